@@ -1,0 +1,163 @@
+"""Plain fp64 CPU oracle for Frechet profile commit-set selection.
+
+TEST INFRASTRUCTURE ONLY.  The oracle checks the CUDA library; only ``tests/``,
+``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline / reference arm may import
+it.  The product package never imports it, and it imports nothing from the product.
+
+The arithmetic lives in ``fdllm_oracle.c`` (plain C, double precision, the steps of the
+paper's Algorithm 1 in order).  This module only compiles that file with gcc and
+marshals numpy arrays through ctypes.
+
+Parameter conventions (same meaning as the library's public interface):
+  mode  0 = profile (Frechet, Sec. 3), 1 = factor, 2 = threshold.
+  param profile: f with margin delta = 1 - f (Cor. factor-reduction); factor: f;
+        threshold: tau.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+PROFILE, FACTOR, THRESHOLD = 0, 1, 2
+BF16, FP32 = 0, 1
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+SOURCE = os.path.join(HERE, "fdllm_oracle.c")
+HEADER = os.path.join(HERE, "fdllm_oracle.h")
+_OUT_DIR = os.path.join(HERE, "_build")
+_LIB_PATH = os.path.join(_OUT_DIR, "liboracle.so")
+_lock = threading.Lock()
+_default = None
+
+
+def compile_oracle(src: str, out: str) -> str:
+    """gcc the C oracle at ``src`` into the shared library ``out`` (OpenMP when present)."""
+    os.makedirs(os.path.dirname(out), exist_ok=True)
+    base = ["gcc", "-O2", "-std=c11", "-ffp-contract=off", "-fPIC", "-shared",
+            "-I", HERE, src, "-o", out + ".tmp", "-lm"]
+    try:
+        subprocess.run(base[:1] + ["-fopenmp"] + base[1:], check=True,
+                       capture_output=True, text=True)
+    except subprocess.CalledProcessError:
+        subprocess.run(base, check=True, capture_output=True, text=True)
+    os.replace(out + ".tmp", out)
+    return out
+
+
+def build_oracle(force: bool = False) -> str:
+    """Compile the committed oracle if its library is missing or stale; return its path."""
+    fresh = (os.path.exists(_LIB_PATH)
+             and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(SOURCE)
+             and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(HEADER))
+    if fresh and not force:
+        return _LIB_PATH
+    return compile_oracle(SOURCE, _LIB_PATH)
+
+
+def _ptr(a: np.ndarray) -> int:
+    return a.ctypes.data
+
+
+def _logits_view(logits: np.ndarray):
+    """Accept fp32 arrays or bf16 given as raw uint16 bits; return (array, dtype code)."""
+    a = np.ascontiguousarray(logits)
+    if a.dtype == np.uint16:
+        return a, BF16
+    if a.dtype == np.float32:
+        return a, FP32
+    raise TypeError("oracle logits must be float32 or uint16 (bf16 bits), got %s" % a.dtype)
+
+
+class Oracle:
+    """ctypes front end of one compiled oracle library."""
+
+    def __init__(self, lib_path: str):
+        lib = ctypes.CDLL(lib_path)
+        p, i64, i32, d = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_double
+        lib.oracle_confidence.argtypes = [p, i32, i64, i64, i64, p, p, p, i32]
+        lib.oracle_confidence.restype = i64
+        lib.oracle_frechet_scan.argtypes = [p, i64, p, p, p]
+        lib.oracle_frechet_scan.restype = None
+        lib.oracle_select_from_conf.argtypes = [p, p, i64, i64, p, i32, d, p, p, p, p]
+        lib.oracle_select_from_conf.restype = i64
+        self.lib = lib
+        self.path = lib_path
+
+    def confidence(self, logits: np.ndarray, mask: np.ndarray, nthreads: int = 1):
+        """Per masked position: (conf float64 [B,L], tok int32 [B,L], invalid row count).
+
+        Unmasked positions hold conf = 0 and tok = -1 (the oracle does not write them)."""
+        a, code = _logits_view(logits)
+        B, L, V = a.shape
+        m = np.ascontiguousarray(mask, dtype=np.uint8).reshape(B, L)
+        conf = np.zeros((B, L), np.float64)
+        tok = np.full((B, L), -1, np.int32)
+        bad = self.lib.oracle_confidence(_ptr(a), code, B, L, V, _ptr(m), _ptr(conf),
+                                         _ptr(tok), int(nthreads))
+        return conf, tok, int(bad)
+
+    def frechet_scan(self, c_sorted):
+        """(L_n, U_n, G_n) for n = 1..m of a descending profile (Eq. frechet_Ln_Un)."""
+        c = np.ascontiguousarray(c_sorted, dtype=np.float64)
+        m = c.shape[0]
+        Ln, Un, Gn = (np.zeros(m, np.float64) for _ in range(3))
+        self.lib.oracle_frechet_scan(_ptr(c), m, _ptr(Ln), _ptr(Un), _ptr(Gn))
+        return Ln, Un, Gn
+
+    def select_from_conf(self, conf: np.ndarray, tok: np.ndarray, mask: np.ndarray, mode: int,
+                         param: float, out_tokens: np.ndarray | None = None):
+        """Sort / scan / select / reveal on given confidences.
+
+        Returns dict(tokens, commit, n, margin, mask, invalid_rows); ``mask`` is the updated
+        copy (the input array is left untouched)."""
+        c = np.ascontiguousarray(conf, dtype=np.float64)
+        B, L = c.shape
+        t = np.ascontiguousarray(tok, dtype=np.int32).reshape(B, L)
+        m = np.array(mask, dtype=np.uint8, copy=True).reshape(B, L)
+        toks = (np.full((B, L), -1, np.int32) if out_tokens is None
+                else np.array(out_tokens, dtype=np.int32, copy=True).reshape(B, L))
+        commit = np.zeros((B, L), np.uint8)
+        n = np.zeros(B, np.int32)
+        margin = np.zeros(B, np.float64)
+        bad = self.lib.oracle_select_from_conf(_ptr(c), _ptr(t), B, L, _ptr(m), int(mode),
+                                               float(param), _ptr(toks), _ptr(commit), _ptr(n),
+                                               _ptr(margin))
+        return dict(tokens=toks, commit=commit, n=n, margin=margin, mask=m,
+                    invalid_rows=int(bad))
+
+    def select(self, logits: np.ndarray, mask: np.ndarray, mode: int, param: float,
+               out_tokens: np.ndarray | None = None, nthreads: int = 1):
+        """Whole selection step (Alg. 1 from confidences to reveal) on host logits."""
+        conf, tok, _ = self.confidence(logits, mask, nthreads)
+        res = self.select_from_conf(conf, tok, mask, mode, param, out_tokens)
+        res["conf"] = conf
+        res["tok"] = tok
+        return res
+
+
+def default() -> Oracle:
+    global _default
+    with _lock:
+        if _default is None:
+            _default = Oracle(build_oracle())
+        return _default
+
+
+def confidence(logits, mask, nthreads: int = 1):
+    return default().confidence(logits, mask, nthreads)
+
+
+def frechet_scan(c_sorted):
+    return default().frechet_scan(c_sorted)
+
+
+def select_from_conf(conf, tok, mask, mode, param, out_tokens=None):
+    return default().select_from_conf(conf, tok, mask, mode, param, out_tokens)
+
+
+def select(logits, mask, mode, param, out_tokens=None, nthreads: int = 1):
+    return default().select(logits, mask, mode, param, out_tokens, nthreads)

@@ -1,0 +1,235 @@
+/*
+ * fdllm_oracle.c -- plain fp64 CPU oracle for Frechet profile commit-set selection.
+ *
+ * TEST INFRASTRUCTURE ONLY (see fdllm_oracle.h): slow, obviously correct, and sharing no
+ * code with the CUDA library.  Each function follows the paper's definitions in the order
+ * of Algorithm 1; nothing is blocked, fused or reordered beyond what those state.
+ *
+ * Build: gcc -O2 -ffp-contract=off -fPIC -shared [-fopenmp] fdllm_oracle.c -lm
+ * (-ffp-contract=off keeps a*b+c unfused so that x86 and Arm hosts round alike.)
+ */
+#include "fdllm_oracle.h"
+
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+/* One logit widened to double.  bf16 is the upper half of an IEEE fp32 word, so the
+ * widening is exact. */
+static double logit_at(const void *logits, int dtype, int64_t i)
+{
+    float f;
+    if (dtype == ORACLE_BF16) {
+        uint32_t u = (uint32_t)((const uint16_t *)logits)[i] << 16;
+        memcpy(&f, &u, sizeof f);
+    } else {
+        f = ((const float *)logits)[i];
+    }
+    return (double)f;
+}
+
+/* Sec. 3 "Notation" and the confidence loop of Alg. 1:
+ *   x_hat_i = argmax_v p_i(v),  c_i = max_v p_i(v),  p_i = softmax of the logits of row i.
+ * With M = max_v x_v and S = sum_v exp(x_v - M), max_v p_i(v) = exp(M - M) / S = 1 / S.
+ * Ties in the argmax go to the lowest vocabulary index. */
+static int confidence_of_row(const void *logits, int dtype, int64_t base, int64_t V,
+                             double *c_out, int32_t *tok_out)
+{
+    double M = -INFINITY;
+    int64_t arg = -1;
+    int saw_nan = 0;
+    for (int64_t v = 0; v < V; ++v) {
+        double x = logit_at(logits, dtype, base + v);
+        if (isnan(x)) {
+            saw_nan = 1;
+            continue;
+        }
+        if (arg < 0 || x > M) { /* strict '>' keeps the lowest index among equal maxima */
+            M = x;
+            arg = v;
+        }
+    }
+    if (saw_nan || !isfinite(M)) {
+        *c_out = NAN;
+        *tok_out = -1;
+        return 1;
+    }
+    double S = 0.0;
+    for (int64_t v = 0; v < V; ++v)
+        S += exp(logit_at(logits, dtype, base + v) - M);
+    *c_out = 1.0 / S;
+    *tok_out = (int32_t)arg;
+    return 0;
+}
+
+int64_t oracle_confidence(const void *logits, int dtype, int64_t B, int64_t L, int64_t V,
+                          const uint8_t *mask, double *conf, int32_t *tok, int nthreads)
+{
+    int64_t bad = 0;
+    const int64_t rows = B * L;
+#ifdef _OPENMP
+    if (nthreads < 1)
+        nthreads = 1;
+#pragma omp parallel for schedule(dynamic, 1) reduction(+ : bad) num_threads(nthreads)
+#else
+    (void)nthreads;
+#endif
+    for (int64_t r = 0; r < rows; ++r) {
+        if (!mask[r])
+            continue;
+        bad += confidence_of_row(logits, dtype, r * V, V, &conf[r], &tok[r]);
+    }
+    return bad;
+}
+
+/* Sec. 3 "Frechet profile quantities" / Eq. frechet_Ln_Un, in the paper's own form. */
+void oracle_frechet_scan(const double *c_sorted, int64_t m, double *Ln, double *Un, double *Gn)
+{
+    double sum = 0.0;
+    for (int64_t n = 1; n <= m; ++n) {
+        sum += c_sorted[n - 1];
+        double l = sum - (double)(n - 1);
+        Ln[n - 1] = l > 0.0 ? l : 0.0;
+        Un[n - 1] = 1.0 - c_sorted[n - 1];
+        Gn[n - 1] = Ln[n - 1] - Un[n - 1];
+    }
+}
+
+typedef struct {
+    double c;
+    int32_t pos;
+} candidate;
+
+/* Alg. 1 sort: c_(1) >= c_(2) >= ...; equal confidences keep the lower position first. */
+static int by_confidence_desc(const void *pa, const void *pb)
+{
+    const candidate *a = (const candidate *)pa, *b = (const candidate *)pb;
+    if (a->c > b->c)
+        return -1;
+    if (a->c < b->c)
+        return 1;
+    return (a->pos > b->pos) - (a->pos < b->pos);
+}
+
+int64_t oracle_select_from_conf(const double *conf, const int32_t *tok, int64_t B, int64_t L,
+                                uint8_t *mask, int mode, double param, int32_t *out_tokens,
+                                uint8_t *out_commit, int32_t *out_n, double *margin)
+{
+    int64_t bad = 0;
+    candidate *cand = (candidate *)malloc((size_t)L * sizeof(candidate));
+    double *cs = (double *)malloc((size_t)L * sizeof(double));
+    double *Ln = (double *)malloc((size_t)L * sizeof(double));
+    double *Un = (double *)malloc((size_t)L * sizeof(double));
+    double *Gn = (double *)malloc((size_t)L * sizeof(double));
+    double *q = (double *)malloc((size_t)L * sizeof(double)); /* signed distance to the bound */
+    int *ok = (int *)malloc((size_t)L * sizeof(int));
+
+    for (int64_t b = 0; b < B; ++b) {
+        const int64_t row0 = b * L;
+        int64_t m = 0;
+        int invalid = 0;
+        for (int64_t l = 0; l < L; ++l) {
+            out_commit[row0 + l] = 0;
+            if (!mask[row0 + l])
+                continue;
+            double c = conf[row0 + l];
+            if (!(c > 0.0 && c <= 1.0))
+                invalid = 1;
+            cand[m].c = c;
+            cand[m].pos = (int32_t)l;
+            ++m;
+        }
+        if (margin)
+            margin[b] = INFINITY;
+        if (invalid) {
+            out_n[b] = -1;
+            ++bad;
+            continue;
+        }
+        if (m == 0) { /* Alg. 1 never reaches a block without masked positions */
+            out_n[b] = 0;
+            continue;
+        }
+
+        qsort(cand, (size_t)m, sizeof(candidate), by_confidence_desc);
+        for (int64_t j = 0; j < m; ++j)
+            cs[j] = cand[j].c;
+
+        /* Alg. 1 scan: one acceptance test per prefix size n = 1..m. */
+        if (mode == ORACLE_PROFILE) {
+            const double delta = 1.0 - param; /* matched margin, Cor. factor-reduction */
+            oracle_frechet_scan(cs, m, Ln, Un, Gn);
+            for (int64_t n = 1; n <= m; ++n) {
+                ok[n - 1] = Gn[n - 1] > delta; /* G_n > delta (Sec. 3) */
+                q[n - 1] = Gn[n - 1] - delta;
+            }
+        } else if (mode == ORACLE_FACTOR) {
+            const double f = param;
+            for (int64_t n = 1; n <= m; ++n) {
+                double r = (double)(n + 1) * (1.0 - cs[n - 1]); /* (n+1)(1 - c_(n)) < f */
+                ok[n - 1] = r < f;
+                q[n - 1] = f - r;
+            }
+        } else { /* threshold: S = {i : c_i >= tau} (Sec. 2, confidence-aware decoding) */
+            const double tau = param;
+            for (int64_t n = 1; n <= m; ++n) {
+                ok[n - 1] = cs[n - 1] >= tau;
+                q[n - 1] = cs[n - 1] - tau;
+            }
+        }
+
+        /* Alg. 1 select: n* = max{n : accepted}; n* = 1 when the set is empty. */
+        int64_t nstar = 0;
+        for (int64_t n = 1; n <= m; ++n)
+            if (ok[n - 1])
+                nstar = n;
+        if (nstar == 0)
+            nstar = 1;
+
+        /* Alg. 1 reveal: the n* most confident masked positions take their argmax token. */
+        for (int64_t j = 0; j < nstar; ++j) {
+            const int64_t at = row0 + cand[j].pos;
+            out_tokens[at] = tok[at];
+            out_commit[at] = 1;
+            mask[at] = 0;
+        }
+        out_n[b] = (int32_t)nstar;
+
+        if (margin) {
+            double mg = fabs(q[nstar - 1]);
+            if (nstar < m) {
+                double next = fabs(q[nstar]);
+                if (next < mg)
+                    mg = next;
+                double gap = cs[nstar - 1] - cs[nstar];
+                if (gap > 0.0 && gap < mg)
+                    mg = gap;
+            }
+            margin[b] = mg;
+        }
+    }
+
+    free(cand);
+    free(cs);
+    free(Ln);
+    free(Un);
+    free(Gn);
+    free(q);
+    free(ok);
+    return bad;
+}
+
+int64_t oracle_select(const void *logits, int dtype, int64_t B, int64_t L, int64_t V,
+                      uint8_t *mask, int mode, double param, int32_t *out_tokens,
+                      uint8_t *out_commit, int32_t *out_n, double *margin, double *conf,
+                      int32_t *tok, int nthreads)
+{
+    int64_t bad_rows = oracle_confidence(logits, dtype, B, L, V, mask, conf, tok, nthreads);
+    (void)bad_rows;
+    return oracle_select_from_conf(conf, tok, B, L, mask, mode, param, out_tokens, out_commit,
+                                   out_n, margin);
+}

@@ -1,0 +1,72 @@
+/*
+ * fdllm_oracle.h -- plain fp64 CPU oracle for Frechet profile commit-set selection.
+ *
+ * TEST INFRASTRUCTURE ONLY.  This oracle exists to check the CUDA path.  Only the
+ * test suite, the smoke check and the benchmark's CPU-baseline / reference arm may
+ * load it.  The product path (the CUDA library) never calls, links or includes it,
+ * and this oracle includes nothing from the product.
+ *
+ * Everything is computed in double precision with plain loops, in the order of the
+ * paper's Algorithm 1 ("Fast-dLLM++: Frechet Profile Decoding"):
+ *   confidence/argmax per masked position -> sort -> scan of L_n, U_n, G_n -> n* -> reveal.
+ *
+ * Conventions shared with the CUDA library's public interface (not its code):
+ *   logits  [B, L, V] row-major, V contiguous; dtype 0 = bf16 (raw uint16 bits), 1 = fp32.
+ *   mask    uint8 [B, L], 1 = masked; updated in place by the reveal (committed -> 0).
+ *   mode    0 = profile (Frechet), 1 = factor, 2 = threshold.
+ *   param   profile: f, with margin delta = 1 - f (matched parameter, Cor. factor-reduction);
+ *           factor: f;  threshold: tau.
+ */
+#ifndef FDLLM_ORACLE_H
+#define FDLLM_ORACLE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum { ORACLE_BF16 = 0, ORACLE_FP32 = 1 };
+enum { ORACLE_PROFILE = 0, ORACLE_FACTOR = 1, ORACLE_THRESHOLD = 2 };
+
+/* Per masked position (b,l): x_hat = lowest v attaining max_v logit, c = max_v softmax(v)
+ * (Sec. 3 "Notation", Alg. 1 confidence loop).  conf/tok are written only at masked
+ * positions.  Rows whose logits contain NaN, or whose maximum is +inf or -inf, get
+ * conf = NaN and tok = -1.  Returns the number of such rows.  nthreads <= 1 runs serially. */
+int64_t oracle_confidence(const void *logits, int dtype, int64_t B, int64_t L, int64_t V,
+                          const uint8_t *mask, double *conf, int32_t *tok, int nthreads);
+
+/* The Frechet profile quantities of Sec. 3 / Eq. frechet_Ln_Un for a profile already
+ * sorted in descending order: for n = 1..m,
+ *   L_n = max{0, sum_{j<=n} c_(j) - (n-1)},  U_n = 1 - c_(n),  G_n = L_n - U_n.
+ * Outputs are indexed n-1. */
+void oracle_frechet_scan(const double *c_sorted, int64_t m, double *Ln, double *Un, double *Gn);
+
+/* Selection from given confidences (Alg. 1 sort, scan, select, reveal).
+ * For every batch row b: m = number of masked positions.
+ *   m == 0            -> out_n[b] = 0, nothing committed.
+ *   any masked conf not in (0, 1] (NaN included) -> out_n[b] = -1, nothing committed.
+ *   otherwise         -> n* = max{n : rule accepts n}, or 1 if no n is accepted;
+ *                        the n* most confident masked positions (ties: lower position
+ *                        first) get out_tokens = tok, out_commit = 1, mask = 0.
+ * out_commit is fully written; out_tokens only at committed positions.
+ * margin[b] (nullable) = decision margin of the row: the smallest of |rule(n) - bound| at
+ * n = n* and n = n*+1 and of the confidence gap c_(n*) - c_(n*+1) when it is non-zero;
+ * +inf when nothing can flip (m == 0, invalid row, or no such term).
+ * Returns the number of invalid rows. */
+int64_t oracle_select_from_conf(const double *conf, const int32_t *tok, int64_t B, int64_t L,
+                                uint8_t *mask, int mode, double param, int32_t *out_tokens,
+                                uint8_t *out_commit, int32_t *out_n, double *margin);
+
+/* oracle_confidence followed by oracle_select_from_conf.  conf/tok are caller scratch of
+ * B*L entries; they come back holding the per-position confidences and argmax tokens. */
+int64_t oracle_select(const void *logits, int dtype, int64_t B, int64_t L, int64_t V,
+                      uint8_t *mask, int mode, double param, int32_t *out_tokens,
+                      uint8_t *out_commit, int32_t *out_n, double *margin, double *conf,
+                      int32_t *tok, int nthreads);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FDLLM_ORACLE_H */

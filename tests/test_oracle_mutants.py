@@ -1,0 +1,63 @@
+"""Planted mistakes in copies of the oracle must each fail at least one pin.
+
+Each mutant is a one-line change to a temporary copy of oracle/fdllm_oracle.c (the
+committed file is never touched): a dropped or shifted term, a wrong sign or index, a
+flipped comparison, a reversed sort.  The copy is compiled with the same gcc flags and the
+whole pin set of ``oracle_pins`` runs against it; a mutant that passes every pin would mean
+the pins cannot see that class of mistake.
+"""
+import os
+import shutil
+
+import pytest
+
+import oracle
+from oracle_pins import ALL_PINS
+
+MUTANTS = {
+    "lower_bound_drops_minus_one": ("sum - (double)(n - 1)", "sum - (double)(n)"),
+    "upper_bound_uses_strongest": ("Un[n - 1] = 1.0 - c_sorted[n - 1]",
+                                   "Un[n - 1] = 1.0 - c_sorted[0]"),
+    "score_sign_flipped": ("Gn[n - 1] = Ln[n - 1] - Un[n - 1]",
+                           "Gn[n - 1] = Ln[n - 1] + Un[n - 1]"),
+    "no_clip_at_zero": ("Ln[n - 1] = l > 0.0 ? l : 0.0", "Ln[n - 1] = l"),
+    "margin_not_strict": ("ok[n - 1] = Gn[n - 1] > delta", "ok[n - 1] = Gn[n - 1] >= delta"),
+    "delta_not_matched": ("const double delta = 1.0 - param", "const double delta = param"),
+    "factor_drops_plus_one": ("(double)(n + 1) * (1.0 - cs[n - 1])",
+                              "(double)(n) * (1.0 - cs[n - 1])"),
+    "factor_not_strict": ("ok[n - 1] = r < f", "ok[n - 1] = r <= f"),
+    "threshold_strict": ("ok[n - 1] = cs[n - 1] >= tau", "ok[n - 1] = cs[n - 1] > tau"),
+    "no_progress_fallback": ("if (nstar == 0)\n            nstar = 1;", ""),
+    "first_failure_off_by_one": ("out_tokens[at] = tok[at];\n            out_commit[at] = 1;",
+                                 "out_tokens[at] = tok[at];\n            out_commit[at] = j > 0 || nstar == 1;"),
+    "sort_ascending": ("if (a->c > b->c)\n        return -1;", "if (a->c > b->c)\n        return 1;"),
+    "ties_prefer_higher_position": ("return (a->pos > b->pos) - (a->pos < b->pos);",
+                                    "return (a->pos < b->pos) - (a->pos > b->pos);"),
+    "argmax_last_of_ties": ("if (arg < 0 || x > M)", "if (arg < 0 || x >= M)"),
+    "confidence_is_sum": ("*c_out = 1.0 / S;", "*c_out = S / (double)V;"),
+    "exp_sign_flipped": ("S += exp(logit_at(logits, dtype, base + v) - M);",
+                         "S += exp(M - logit_at(logits, dtype, base + v));"),
+    "bf16_widened_wrong": ("(uint32_t)((const uint16_t *)logits)[i] << 16",
+                           "(uint32_t)((const uint16_t *)logits)[i] << 15"),
+    "nan_not_flagged": ("if (saw_nan || !isfinite(M))", "if (!isfinite(M))"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_planted_mistake_is_caught(name, tmp_path):
+    old, new = MUTANTS[name]
+    with open(oracle.SOURCE) as fh:
+        src = fh.read()
+    assert src.count(old) == 1, "mutation anchor not found once: %r" % old
+    shutil.copy(oracle.HEADER, tmp_path / os.path.basename(oracle.HEADER))
+    mutated = tmp_path / "mutant.c"
+    mutated.write_text(src.replace(old, new))
+    lib = oracle.compile_oracle(str(mutated), str(tmp_path / "libmutant.so"))
+    mut = oracle.Oracle(lib)
+    failed = []
+    for pin in ALL_PINS:
+        try:
+            pin(mut)
+        except (AssertionError, ValueError, IndexError, OverflowError, FloatingPointError):
+            failed.append(pin.__name__)
+    assert failed, "planted mistake %s passed every pin" % name
