@@ -1,0 +1,435 @@
+#!/usr/bin/env python3
+"""Benchmark of the per-step commit-set selection (Frechet profile decoding) on GB300.
+
+One step = one full selection (vocab reduction + sort / scan / select / reveal) over one
+batch of synthetic LLaDA-shaped logits (V = 126464).  Default workload: the large-batch
+serving step, B = 64 rows of an active block of L = 32 positions, 50-100 % masked, bf16,
+profile rule with f = 1 (delta = 0).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                  [--workload NAME] [--no-graph]
+
+Prints one JSON line (rank 0).  Under torchrun (N > 1) every rank runs its own batch on its
+own GPU (weak scaling, no data exchange); the time is the max over ranks.
+
+--impl reference times the fp64 CPU oracle (the reference arm of this benchmark) on the
+host cores, each step a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import datetime
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = ("decode-step selections/sec and logits HBM GB/s (fraction of GB300 peak) at "
+          "V=126464")
+UNIT = "selections/s"
+FALLBACK_HBM_GBS = 6800.0
+PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "vocab_reduce_serving_b64_l32_bf16.md")
+KERNEL_SOURCE = os.path.join(ROOT, "paper_2606_02955_gb300", "csrc", "vocab_reduce.cu")
+
+
+# ----------------------------------------------------------------------------- host logic
+def aggregate(rows_per_rank: int, steps: int, times_s: list[float]) -> dict:
+    """Whole-job throughput from per-rank timings: every rank decides rows_per_rank rows per
+    step; the job takes as long as its slowest rank."""
+    t = max(times_s)
+    n = len(times_s)
+    return {"value": rows_per_rank * steps * n / t, "seconds": t, "n_ranks": n}
+
+
+def rank_seed(base: int, rank: int) -> int:
+    """Each rank draws its own batch (weak scaling: independent problems per GPU)."""
+    return base + 7919 * rank
+
+
+def peak_hbm_gbs():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as fh:
+            return float(json.load(fh)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def ncu_traffic():
+    """DRAM traffic per vocab-reduction launch from the committed ncu summary, only while
+    the kernel source is the one the counters were taken on."""
+    try:
+        text = open(PROFILE_SUMMARY).read()
+        sha = hashlib.sha256(open(KERNEL_SOURCE, "rb").read()).hexdigest()
+    except OSError:
+        return None
+    m_sha = re.search(r"source_sha256:\s*([0-9a-f]{64})", text)
+    m_t = re.search(r"traffic_bytes_per_launch:\s*([0-9]+)", text)
+    if not (m_sha and m_t) or m_sha.group(1) != sha:
+        return None
+    return int(m_t.group(1))
+
+
+_REASON_BITS = {
+    0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_cap",
+    0x8: "hw_slowdown", 0x10: "sync_boost", 0x20: "sw_thermal_slowdown",
+    0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown",
+    0x100: "display_clock_setting",
+}
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons while work runs."""
+
+    def __init__(self, gpu_index: int, period_ms: int = 50):
+        self.gpu = gpu_index
+        self.period = period_ms
+        self.samples = []  # (t, sm_mhz, max_mhz, reasons_bitmask)
+        self.proc = None
+        self.thread = None
+
+    def start(self):
+        cmd = ["nvidia-smi", "-i", str(self.gpu),
+               "--query-gpu=clocks.sm,clocks.max.sm,clocks_event_reasons.active",
+               "--format=csv,noheader,nounits", "-lms", str(self.period)]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL,
+                                         text=True)
+        except OSError:
+            self.proc = None
+            return self
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 3:
+                continue
+            try:
+                self.samples.append((time.time(), float(parts[0]), float(parts[1]),
+                                     int(parts[2], 16)))
+            except ValueError:
+                continue
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+        if self.thread is not None:
+            self.thread.join(timeout=5)
+
+    def summary(self, t0: float, t1: float) -> dict:
+        inside = [s for s in self.samples if t0 <= s[0] <= t1]
+        used = inside if inside else self.samples
+        if not used:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"],
+                    "samples_in_timed_region": 0}
+        mask = 0
+        for s in used:
+            mask |= s[3]
+        reasons = [name for bit, name in _REASON_BITS.items() if mask & bit and bit != 0x1]
+        return {"sm_mhz": statistics.median(s[1] for s in used),
+                "sm_max_mhz": max(s[2] for s in used), "reasons": reasons,
+                "samples_in_timed_region": len(inside)}
+
+
+# ----------------------------------------------------------------------------- our arm
+def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
+    import numpy as np
+    import torch
+
+    import fdllm_synth as syn
+    import paper_2606_02955_gb300 as fd
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+
+    w = syn.WORKLOADS[args.workload]
+    seed = rank_seed(1234, rank)
+    n_buf = max(1, args.buffers)
+    bufs = [syn.make_logits(w, seed=seed + i, device=dev) for i in range(n_buf)]
+    mask0_np = syn.make_mask(w, seed=seed)
+    mask0 = torch.from_numpy(mask0_np).to(dev)
+    masked_rows = int(mask0_np.sum())
+    alg_bytes = masked_rows * w.V * w.elem_bytes
+    mode = {"profile": fd.PROFILE, "factor": fd.FACTOR, "threshold": fd.THRESHOLD}[args.mode]
+
+    mask = mask0.clone()
+    tok = torch.full((w.B, w.L), -1, dtype=torch.int32, device=dev)
+    commit = torch.empty((w.B, w.L), dtype=torch.uint8, device=dev)
+    n_out = torch.empty((w.B,), dtype=torch.int32, device=dev)
+    conf = torch.empty((w.B, w.L), dtype=torch.float32, device=dev)
+    amax = torch.empty((w.B, w.L), dtype=torch.int32, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def step(i):
+        mask.copy_(mask0, non_blocking=True)  # steady state: same masked rows every step
+        fd.fdllm_select(bufs[i % n_buf], mask, args.param, mode, tok, commit, n_out,
+                        stream=stream)
+
+    def k1_only(i):
+        fd.fdllm_confidence(bufs[i % n_buf], mask0, conf, amax, stream=stream)
+
+    def make_runner(fn, per_replay):
+        """A callable running `per_replay` consecutive steps (one CUDA graph replay)."""
+        with torch.cuda.stream(stream):
+            for i in range(max(3, per_replay)):  # warm: allocations, attributes
+                fn(i)
+        stream.synchronize()
+        if args.no_graph:
+            def run(r):
+                with torch.cuda.stream(stream):
+                    for i in range(per_replay):
+                        fn(r * per_replay + i)
+            return run
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for i in range(per_replay):
+                fn(i)
+
+        def run(_r):
+            g.replay()
+        return run
+
+    per_replay = n_buf
+    replays = max(1, -(-args.steps // per_replay))
+    steps = replays * per_replay
+    warm_replays = max(1, -(-args.warmup // per_replay))
+
+    def timed(run, n_rep):
+        for r in range(warm_replays):
+            with torch.cuda.stream(stream):
+                run(r)
+        stream.synchronize()
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        t_wall0 = time.time()
+        e0.record(stream)
+        with torch.cuda.stream(stream):
+            for r in range(n_rep):
+                run(r)
+        e1.record(stream)
+        e1.synchronize()
+        t_wall1 = time.time()
+        torch.cuda.synchronize()
+        if dist is not None:
+            dist.barrier()
+        return e0.elapsed_time(e1) / 1e3, t_wall0, t_wall1
+
+    sampler = ClockSampler(local_rank).start() if rank == 0 else None
+    step_run = make_runner(step, per_replay)
+    t_step, tw0, tw1 = timed(step_run, replays)
+    k1_run = make_runner(k1_only, per_replay)
+    t_k1, _, _ = timed(k1_run, replays)
+    if sampler is not None:
+        time.sleep(0.12)
+        sampler.stop()
+
+    times = [t_step]
+    if dist is not None:
+        tt = torch.tensor([t_step], dtype=torch.float64, device=dev)
+        gathered = [torch.zeros_like(tt) for _ in range(world)]
+        dist.all_gather(gathered, tt)
+        times = [float(x.item()) for x in gathered]
+    agg = aggregate(w.B, steps, times)
+    ms_per_step = agg["seconds"] / steps * 1e3
+
+    # end to end: the public call with pinned host buffers, copies inside the timed region
+    e2e = None
+    if not args.skip_e2e:
+        h_logits = torch.empty(bufs[0].shape, dtype=bufs[0].dtype, pin_memory=True)
+        h_logits.copy_(bufs[0])
+        h_mask = torch.from_numpy(mask0_np.copy()).pin_memory()
+        h_tok = torch.full((w.B, w.L), -1, dtype=torch.int32).pin_memory()
+        h_commit = torch.empty((w.B, w.L), dtype=torch.uint8).pin_memory()
+        h_n = torch.empty((w.B,), dtype=torch.int32).pin_memory()
+        for _ in range(2):
+            h_mask.copy_(torch.from_numpy(mask0_np))
+            fd.fdllm_select(h_logits, h_mask, args.param, mode, h_tok, h_commit, h_n)
+        e2e_steps = max(3, min(20, args.steps // 50))
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(e2e_steps):
+            h_mask.copy_(torch.from_numpy(mask0_np))
+            fd.fdllm_select(h_logits, h_mask, args.param, mode, h_tok, h_commit, h_n)
+        t_e2e = time.perf_counter() - t0
+        e2e = {"value": w.B * e2e_steps / t_e2e, "unit": UNIT,
+               "h2d_bytes_per_step": h_logits.numel() * h_logits.element_size()
+               + h_mask.numel() + h_tok.numel() * 4,
+               "d2h_bytes_per_step": h_tok.numel() * 4 + h_commit.numel() + h_n.numel() * 4
+               + h_mask.numel(),
+               "steps": e2e_steps}
+        del h_logits
+
+    result = None
+    if rank == 0:
+        peak, peak_kind = peak_hbm_gbs()
+        k1_s = t_k1 / steps
+        achieved = alg_bytes / k1_s / 1e9
+        traffic = ncu_traffic()
+        clocks = sampler.summary(tw0, tw1) if sampler is not None else None
+        result = {
+            "metric": METRIC, "value": agg["value"], "unit": UNIT, "n_gpus": world,
+            "steps": steps, "warmup": warm_replays * per_replay,
+            "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
+            "config": {
+                "workload": w.name, "description": w.description, "B": w.B, "L": w.L,
+                "V": w.V, "rule": args.mode, "param": args.param,
+                "masked_rows_per_step": masked_rows,
+                "logits_bytes_per_step": alg_bytes,
+                "logits_gbs_per_step": alg_bytes / (ms_per_step * 1e-3) / 1e9,
+                "l2_policy": "inputs larger than L2: %d rotating logits buffers of %.0f MB "
+                             "(%.2f GB > 129 MB L2)" % (n_buf, bufs[0].numel() *
+                                                        bufs[0].element_size() / 1e6,
+                                                        n_buf * bufs[0].numel() *
+                                                        bufs[0].element_size() / 1e9),
+                "cuda_graph": not args.no_graph,
+                "parallelism": "dp%d (independent batches, no collective)" % world,
+            },
+            "roofline": {
+                "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": achieved / peak, "traffic": traffic,
+                "kernel": "vocab_reduce (a1), timed with its finalize pass",
+                "kernel_us": k1_s * 1e6, "peak_source": peak_kind,
+                "algorithmic_bytes_per_launch": alg_bytes,
+            },
+            "clocks": clocks,
+            "gpu_launches": 2 * steps,
+            "e2e": e2e,
+        }
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
+    return result
+
+
+# ----------------------------------------------------------------------------- oracle arm
+def oracle_sample_rows(args) -> int:
+    return max(1, min(args.sample_rows, 64))
+
+
+def run_oracle_timed(args, steps: int, warmup: int, budget_s: float | None):
+    """The CPU oracle on a bounded sample of the workload: `sample_rows` batch rows drawn by
+    the same seeded recipe, on all host cores.  Runs `steps` steps, or for `budget_s`
+    seconds (at least one step) when a budget is given."""
+    import dataclasses
+
+    import fdllm_synth as syn
+    import oracle
+
+    w = syn.WORKLOADS[args.workload]
+    rows = oracle_sample_rows(args)
+    ws = dataclasses.replace(w, B=rows)
+    host = syn.host_bits(syn.make_logits(ws, seed=1234, device="cpu"))
+    mask = syn.make_mask(ws, seed=1234)
+    threads = os.cpu_count() or 1
+    mode = {"profile": oracle.PROFILE, "factor": oracle.FACTOR,
+            "threshold": oracle.THRESHOLD}[args.mode]
+    orc = oracle.default()
+    for _ in range(warmup):
+        orc.select(host, mask, mode, args.param, nthreads=threads)
+    t0 = time.perf_counter()
+    done = 0
+    while True:
+        orc.select(host, mask, mode, args.param, nthreads=threads)
+        done += 1
+        elapsed = time.perf_counter() - t0
+        if budget_s is not None and elapsed >= budget_s:
+            break
+        if budget_s is None and done >= steps:
+            break
+    t = time.perf_counter() - t0
+    cpu = "unknown"
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.lower().startswith(("model name", "cpu model")):
+                cpu = line.split(":", 1)[1].strip()
+                break
+    except OSError:
+        pass
+    return {
+        "value": rows * done / t, "unit": UNIT, "cores": threads, "kind": "oracle",
+        "sample": "%d batch rows of %s drawn by its recipe (%d masked positions of V=%d) "
+                  "per step, %d steps, fp64 C oracle with OpenMP over positions"
+                  % (rows, w.name, int(mask.sum()), w.V, done),
+        "seconds": t, "steps": done, "cpu": cpu,
+    }
+
+
+def run_reference(args, rank: int, world: int) -> dict | None:
+    if rank != 0:
+        return None
+    base = run_oracle_timed(args, args.steps, args.warmup, None)
+    import fdllm_synth as syn
+    w = syn.WORKLOADS[args.workload]
+    return {
+        "impl": "reference", "metric": METRIC, "value": base["value"], "unit": UNIT,
+        "n_gpus": world, "steps": base["steps"], "warmup": args.warmup,
+        "ms_per_step": base["seconds"] / base["steps"] * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "B": w.B, "L": w.L, "V": w.V, "rule": args.mode,
+                   "param": args.param, "sample_rows": oracle_sample_rows(args)},
+        "cpu_baseline": base,
+        "e2e": {"value": base["value"], "unit": UNIT, "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+
+
+# ----------------------------------------------------------------------------- main
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="serving_b64_l32_bf16")
+    ap.add_argument("--mode", choices=["profile", "factor", "threshold"], default="profile")
+    ap.add_argument("--param", type=float, default=1.0)
+    ap.add_argument("--buffers", type=int, default=4)
+    ap.add_argument("--no-graph", action="store_true")
+    ap.add_argument("--skip-e2e", action="store_true")
+    ap.add_argument("--skip-cpu-baseline", action="store_true")
+    ap.add_argument("--sample-rows", type=int, default=4,
+                    help="batch rows per oracle step (reference arm / CPU baseline)")
+    ap.add_argument("--cpu-budget-s", type=float, default=10.0)
+    args = ap.parse_args(argv)
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        out = run_reference(args, rank, world)
+    else:
+        out = run_ours(args, rank, world, local_rank)
+        if out is not None and world == 1 and not args.skip_cpu_baseline:
+            out["cpu_baseline"] = run_oracle_timed(args, 1, 1, args.cpu_budget_s)
+    if out is not None:
+        out["timestamp"] = datetime.datetime.now(datetime.timezone.utc).isoformat()
+        print(json.dumps(out), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,151 @@
+/*
+ * fdllm.h -- C interface of the GB300 (sm_103a) commit-set selection library for
+ * Frechet profile decoding of masked diffusion LLMs (Fast-dLLM++).
+ *
+ * One decode step of the paper's Algorithm 1, from logits at the masked positions of the
+ * active block to the committed tokens and the updated mask:
+ *   (a1) per masked position i: x_hat_i = argmax_v p_i(v) (lowest v on ties) and the
+ *        confidence c_i = max_v p_i(v) = exp(M_i - logsumexp_i), p_i = softmax of row i
+ *        (Sec. 3 "Notation"; Alg. 1 confidence loop);
+ *   (a2) sort the masked confidences of each batch row in descending order, equal
+ *        confidences lower position first (Alg. 1 sort);
+ *   (a3) for every prefix size n: L_n = max{0, sum_{j<=n} c_(j) - (n-1)}, U_n = 1 - c_(n),
+ *        G_n = L_n - U_n (Sec. 3 "Frechet profile quantities", Eq. frechet_Ln_Un);
+ *   (a4) n* = max{n : G_n > delta}, n* = 1 when no n qualifies (Sec. 3; Alg. 1 select);
+ *   (a5) reveal the n* most confident masked positions (Alg. 1 reveal).
+ * Fast-dLLM's rules are available as alternative modes: factor, accept n iff
+ * (n+1)(1 - c_(n)) < f (Sec. 1, Cor. factor-reduction); threshold, commit {i : c_i >= tau}
+ * or the single most confident position when that set is empty (Sec. 2).
+ *
+ * Conventions for every entry point:
+ *   - Pointers named logits, mask, out_*, conf, argmax and workspace are DEVICE pointers
+ *     owned by the caller; the library never frees them.  `stream` is a cudaStream_t
+ *     (NULL = legacy default stream) passed as void* so this header needs no CUDA headers.
+ *   - logits is [B, L, V] row-major with V contiguous; dtype FDLLM_BF16 (bfloat16) or
+ *     FDLLM_FP32.  The base must be 16-byte aligned and V * sizeof(dtype) a multiple of 16
+ *     (V % 8 == 0 for bf16, V % 4 == 0 for fp32); otherwise FDLLM_ERR_ALIGN.  A vocabulary
+ *     that is not a multiple can be padded with -inf columns, which change nothing.
+ *   - mask is uint8 [B, L], nonzero = masked.  Only masked positions are read from logits.
+ *   - Limits: 1 <= B, 1 <= L <= FDLLM_MAX_L, B * L <= FDLLM_MAX_ROWS, V >= 1.
+ *   - Work is enqueued asynchronously on `stream`; the return value reports only argument
+ *     and launch errors, detected on the host.  Per-row data errors are reported in out_n
+ *     (see FDLLM_ROW_NONFINITE).
+ *   - All kernels are deterministic: the same inputs on the same GPU model give
+ *     bit-identical outputs.
+ */
+#ifndef FDLLM_H
+#define FDLLM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define FDLLM_MAX_L 1024       /* positions per batch row (one CTA sorts a row in smem) */
+#define FDLLM_MAX_ROWS 65536   /* B * L: masked-row compaction lives in shared memory */
+
+typedef enum { FDLLM_BF16 = 0, FDLLM_FP32 = 1 } fdllm_dtype;
+
+typedef enum {
+    FDLLM_PROFILE = 0,   /* Frechet profile rule, Sec. 3: param = f, margin delta = 1 - f */
+    FDLLM_FACTOR = 1,    /* Fast-dLLM factor rule: param = f                              */
+    FDLLM_THRESHOLD = 2  /* Fast-dLLM threshold rule: param = tau                         */
+} fdllm_mode;
+
+typedef enum {
+    FDLLM_OK = 0,
+    FDLLM_ERR_ARG = 1,       /* a null pointer, a size out of range, an unknown enum, a
+                                non-finite param                                         */
+    FDLLM_ERR_ALIGN = 2,     /* logits base not 16-byte aligned or V*sizeof(dtype) % 16 */
+    FDLLM_ERR_NONFINITE = 3, /* reserved for callers mapping out_n == -1 to a status     */
+    FDLLM_ERR_CUDA = 4,      /* a CUDA runtime call or kernel launch failed             */
+    FDLLM_ERR_WORKSPACE = 5, /* caller workspace too small or misaligned                */
+    FDLLM_ERR_DEVICE = 6     /* a kernel's bounded wait gave up (see fdllm_device_status) */
+} fdllm_status;
+
+/* out_n value of a batch row whose masked logits are unusable: a NaN anywhere in a masked
+ * position's row, or a maximum of +inf or -inf.  Such a row commits nothing and its mask
+ * is left unchanged.  (The paper defines confidences only for proper distributions.) */
+#define FDLLM_ROW_NONFINITE (-1)
+/* out_n value of every row when a kernel of the step gave up a bounded wait. */
+#define FDLLM_ROW_DEVICE_ERROR (-2)
+
+/* ---------------------------------------------------------------------------------- */
+/* One whole selection step (steps a1-a5 above; Alg. 1 from the model's logits to the
+ * reveal), with a workspace the library owns.
+ *
+ *   logits      [B, L, V] device, dtype as given, read only at masked positions.
+ *   mask        [B, L] uint8 device, nonzero = masked.  UPDATED IN PLACE: committed
+ *               positions become 0 (Alg. 1 reveal).
+ *   param       profile: f, the rule accepts n iff G_n > delta with delta = 1 - f (the
+ *               matched parameter of Cor. factor-reduction; the paper's operating point
+ *               delta = 0.25 is f = 0.75).  factor: f.  threshold: tau.  Any finite value
+ *               is accepted; the paper states delta in [0, 1] (f in [0, 1]).
+ *   out_tokens  [B, L] int32 device: written ONLY at committed positions, with x_hat.
+ *   out_commit  [B, L] uint8 device: fully written, 1 = committed this step.
+ *   out_n       [B] int32 device: number committed in each row; 0 iff the row had no
+ *               masked position; FDLLM_ROW_NONFINITE / FDLLM_ROW_DEVICE_ERROR as above.
+ *
+ * The library's workspace is allocated on the current device at the first call that
+ * needs more than it holds (cudaMalloc, which synchronises), then reused; make one call
+ * of the largest shape before capturing the step in a CUDA graph.  Calls that share the
+ * library workspace must be ordered on the GPU (one stream, or events); for concurrent
+ * steps use fdllm_select_ws with a workspace per stream. */
+fdllm_status fdllm_select(const void *logits, int dtype, int B, int L, int V, uint8_t *mask,
+                          double param, int mode, int32_t *out_tokens, uint8_t *out_commit,
+                          int32_t *out_n, void *stream);
+
+/* Bytes of caller workspace fdllm_select_ws needs for this shape (a pure host function). */
+size_t fdllm_workspace_bytes(int B, int L, int V, int dtype);
+
+/* fdllm_select with a caller-provided workspace (device, 256-byte aligned, at least
+ * fdllm_workspace_bytes(B, L, V, dtype) bytes).  The workspace must be zero-filled before
+ * its first use; every call that completes leaves it ready for the next call, so it is
+ * zeroed once, not per call.  The library never allocates on this path. */
+fdllm_status fdllm_select_ws(const void *logits, int dtype, int B, int L, int V, uint8_t *mask,
+                             double param, int mode, int32_t *out_tokens, uint8_t *out_commit,
+                             int32_t *out_n, void *workspace, size_t workspace_bytes,
+                             void *stream);
+
+/* Step a1 alone (Sec. 3 "Notation"; Alg. 1 confidence loop): for every masked position,
+ * out_conf = c = max softmax probability (fp32) and out_argmax = x_hat (int32, lowest index
+ * among equal maxima).  Both [B, L] device arrays, written only at masked positions; a
+ * row with non-finite logits (see FDLLM_ROW_NONFINITE) gets out_conf = NaN and
+ * out_argmax = -1.  Uses the library workspace like fdllm_select. */
+fdllm_status fdllm_confidence(const void *logits, int dtype, int B, int L, int V,
+                              const uint8_t *mask, float *out_conf, int32_t *out_argmax,
+                              void *stream);
+
+/* Steps a2-a5 alone (Alg. 1 sort, scan, select, reveal) on given confidences.
+ *   conf    [B, L] fp32 device, read at masked positions; a masked value outside (0, 1]
+ *           (NaN included) makes the row FDLLM_ROW_NONFINITE.
+ *   argmax  [B, L] int32 device, the token revealed at each committed position.
+ * mask, param, mode and the outputs as in fdllm_select.  Needs no workspace. */
+fdllm_status fdllm_select_from_conf(const float *conf, const int32_t *argmax, int B, int L,
+                                    uint8_t *mask, double param, int mode,
+                                    int32_t *out_tokens, uint8_t *out_commit, int32_t *out_n,
+                                    void *stream);
+
+/* Synchronises `stream`, then reports (and clears) the sticky device error of the library
+ * workspace on the current device: FDLLM_ERR_DEVICE if a kernel gave up a bounded wait
+ * since the last call, FDLLM_OK otherwise.  For fdllm_select_ws, pass the workspace to
+ * fdllm_workspace_status instead. */
+fdllm_status fdllm_device_status(void *stream);
+fdllm_status fdllm_workspace_status(void *workspace, void *stream);
+
+/* Frees the library workspace of the current device (synchronises the device). */
+void fdllm_release_workspace(void);
+
+/* A static English description of a status code. */
+const char *fdllm_status_string(int status);
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+int fdllm_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FDLLM_H */

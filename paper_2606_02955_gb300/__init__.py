@@ -1,0 +1,243 @@
+"""Python binding of libfdllm.so: Frechet profile commit-set selection on GB300 (sm_103a).
+
+The functions carry the names of the C interface (include/fdllm.h) and only marshal
+arguments: every step of the selection runs in the library's CUDA kernels.  PyTorch
+supplies device memory and the current stream.  The first call loads the compiled library
+and raises when it has not been built (``paper_2606_02955_gb300.build``); there is no
+fallback implementation.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+from .build import LIB_PATH
+
+__all__ = [
+    "BF16", "FP32", "PROFILE", "FACTOR", "THRESHOLD", "ROW_NONFINITE", "ROW_DEVICE_ERROR",
+    "FdllmError", "fdllm_select", "fdllm_select_ws", "fdllm_workspace_bytes",
+    "fdllm_confidence", "fdllm_select_from_conf", "fdllm_device_status",
+    "fdllm_workspace_status", "fdllm_release_workspace", "fdllm_status_string",
+    "fdllm_version", "library_path",
+]
+
+BF16, FP32 = 0, 1
+PROFILE, FACTOR, THRESHOLD = 0, 1, 2
+ROW_NONFINITE, ROW_DEVICE_ERROR = -1, -2
+MODES = {"profile": PROFILE, "factor": FACTOR, "threshold": THRESHOLD}
+
+_lib = None
+
+
+def _load():
+    """Load libfdllm.so once; a missing library is an error, never a fallback."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(
+            "libfdllm.so is not built (%s); run paper_2606_02955_gb300.build.build_library() "
+            "or __graft_entry__.build()" % LIB_PATH)
+    lib = ctypes.CDLL(LIB_PATH)
+    p, i, d, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_double, ctypes.c_size_t
+    lib.fdllm_select.argtypes = [p, i, i, i, i, p, d, i, p, p, p, p]
+    lib.fdllm_select.restype = i
+    lib.fdllm_select_ws.argtypes = [p, i, i, i, i, p, d, i, p, p, p, p, sz, p]
+    lib.fdllm_select_ws.restype = i
+    lib.fdllm_workspace_bytes.argtypes = [i, i, i, i]
+    lib.fdllm_workspace_bytes.restype = sz
+    lib.fdllm_confidence.argtypes = [p, i, i, i, i, p, p, p, p]
+    lib.fdllm_confidence.restype = i
+    lib.fdllm_select_from_conf.argtypes = [p, p, i, i, p, d, i, p, p, p, p]
+    lib.fdllm_select_from_conf.restype = i
+    lib.fdllm_device_status.argtypes = [p]
+    lib.fdllm_device_status.restype = i
+    lib.fdllm_workspace_status.argtypes = [p, p]
+    lib.fdllm_workspace_status.restype = i
+    lib.fdllm_release_workspace.argtypes = []
+    lib.fdllm_release_workspace.restype = None
+    lib.fdllm_status_string.argtypes = [i]
+    lib.fdllm_status_string.restype = ctypes.c_char_p
+    lib.fdllm_version.argtypes = []
+    lib.fdllm_version.restype = i
+    _lib = lib
+    return lib
+
+
+class FdllmError(RuntimeError):
+    def __init__(self, status: int, call: str):
+        super().__init__("%s failed: status %d (%s)" % (call, status, fdllm_status_string(status)))
+        self.status = status
+
+
+def library_path() -> str:
+    return LIB_PATH
+
+
+def fdllm_status_string(status: int) -> str:
+    return _load().fdllm_status_string(int(status)).decode()
+
+
+def fdllm_version() -> int:
+    return _load().fdllm_version()
+
+
+def _check(status: int, call: str):
+    if status != 0:
+        raise FdllmError(status, call)
+
+
+def _mode(mode) -> int:
+    return MODES[mode] if isinstance(mode, str) else int(mode)
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return BF16
+    if t.dtype == torch.float32:
+        return FP32
+    raise TypeError("logits must be bfloat16 or float32, got %s" % t.dtype)
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def _dev(t: torch.Tensor, name: str, dtype=None, shape=None):
+    if not t.is_cuda:
+        raise ValueError("%s must be a CUDA tensor" % name)
+    if not t.is_contiguous():
+        raise ValueError("%s must be contiguous" % name)
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError("%s must be %s, got %s" % (name, dtype, t.dtype))
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError("%s must have shape %s, got %s" % (name, tuple(shape), tuple(t.shape)))
+    return t.data_ptr()
+
+
+def _outputs(B, L, device, out_tokens, out_commit, out_n):
+    if out_tokens is None:
+        out_tokens = torch.full((B, L), -1, dtype=torch.int32, device=device)
+    if out_commit is None:
+        out_commit = torch.empty((B, L), dtype=torch.uint8, device=device)
+    if out_n is None:
+        out_n = torch.empty((B,), dtype=torch.int32, device=device)
+    return out_tokens, out_commit, out_n
+
+
+def fdllm_select(logits: torch.Tensor, mask: torch.Tensor, param: float, mode=PROFILE,
+                 out_tokens=None, out_commit=None, out_n=None, stream=None):
+    """One selection step (fdllm_select).  ``logits`` [B, L, V] bf16/fp32, ``mask`` [B, L]
+    uint8 (updated in place).  Returns (out_tokens, out_commit, out_n).
+
+    Device tensors run asynchronously on ``stream`` (default: current stream).  With host
+    tensors the call copies the inputs to the current CUDA device (pinned memory makes the
+    copies asynchronous), runs the step, copies the outputs and the updated mask back and
+    synchronises: the end-to-end form of the call."""
+    if not logits.is_cuda:
+        return _select_from_host(logits, mask, param, mode, out_tokens, out_commit, out_n)
+    B, L, V = logits.shape
+    lp = _dev(logits, "logits")
+    mp = _dev(mask, "mask", torch.uint8, (B, L))
+    out_tokens, out_commit, out_n = _outputs(B, L, logits.device, out_tokens, out_commit, out_n)
+    st = _load().fdllm_select(lp, _dtype_code(logits), B, L, V, mp, float(param), _mode(mode),
+                           _dev(out_tokens, "out_tokens", torch.int32, (B, L)),
+                           _dev(out_commit, "out_commit", torch.uint8, (B, L)),
+                           _dev(out_n, "out_n", torch.int32, (B,)), _stream(stream))
+    _check(st, "fdllm_select")
+    return out_tokens, out_commit, out_n
+
+
+def _select_from_host(logits, mask, param, mode, out_tokens, out_commit, out_n):
+    dev = torch.device("cuda", torch.cuda.current_device())
+    d_logits = logits.to(dev, non_blocking=True)
+    d_mask = mask.to(dev, non_blocking=True)
+    B, L, _ = logits.shape
+    d_tok = (torch.full((B, L), -1, dtype=torch.int32, device=dev) if out_tokens is None
+             else out_tokens.to(dev, non_blocking=True))
+    t, c, n = fdllm_select(d_logits, d_mask, param, mode, d_tok)
+    pin = logits.is_pinned()
+    host = lambda x: torch.empty(x.shape, dtype=x.dtype, pin_memory=pin)
+    h_tok = out_tokens if out_tokens is not None else host(t)
+    h_commit = out_commit if out_commit is not None else host(c)
+    h_n = out_n if out_n is not None else host(n)
+    h_tok.copy_(t, non_blocking=True)
+    h_commit.copy_(c, non_blocking=True)
+    h_n.copy_(n, non_blocking=True)
+    mask.copy_(d_mask, non_blocking=True)
+    torch.cuda.current_stream().synchronize()
+    return h_tok, h_commit, h_n
+
+
+def fdllm_workspace_bytes(B: int, L: int, V: int, dtype=BF16) -> int:
+    return int(_load().fdllm_workspace_bytes(B, L, V, dtype))
+
+
+def fdllm_select_ws(logits: torch.Tensor, mask: torch.Tensor, param: float, mode,
+                    workspace: torch.Tensor, out_tokens=None, out_commit=None, out_n=None,
+                    stream=None):
+    """fdllm_select with a caller workspace (a zero-filled uint8 CUDA tensor of at least
+    fdllm_workspace_bytes bytes, 256-byte aligned as torch allocations are)."""
+    B, L, V = logits.shape
+    out_tokens, out_commit, out_n = _outputs(B, L, logits.device, out_tokens, out_commit, out_n)
+    st = _load().fdllm_select_ws(_dev(logits, "logits"), _dtype_code(logits), B, L, V,
+                              _dev(mask, "mask", torch.uint8, (B, L)), float(param), _mode(mode),
+                              _dev(out_tokens, "out_tokens", torch.int32, (B, L)),
+                              _dev(out_commit, "out_commit", torch.uint8, (B, L)),
+                              _dev(out_n, "out_n", torch.int32, (B,)),
+                              _dev(workspace, "workspace", torch.uint8),
+                              workspace.numel(), _stream(stream))
+    _check(st, "fdllm_select_ws")
+    return out_tokens, out_commit, out_n
+
+
+def fdllm_confidence(logits: torch.Tensor, mask: torch.Tensor, out_conf=None, out_argmax=None,
+                     stream=None):
+    """Step a1 alone: (conf fp32 [B, L], argmax int32 [B, L]) written at masked positions
+    (unwritten positions of freshly allocated outputs hold NaN / -1)."""
+    B, L, V = logits.shape
+    if out_conf is None:
+        out_conf = torch.full((B, L), float("nan"), dtype=torch.float32, device=logits.device)
+    if out_argmax is None:
+        out_argmax = torch.full((B, L), -1, dtype=torch.int32, device=logits.device)
+    st = _load().fdllm_confidence(_dev(logits, "logits"), _dtype_code(logits), B, L, V,
+                               _dev(mask, "mask", torch.uint8, (B, L)),
+                               _dev(out_conf, "out_conf", torch.float32, (B, L)),
+                               _dev(out_argmax, "out_argmax", torch.int32, (B, L)),
+                               _stream(stream))
+    _check(st, "fdllm_confidence")
+    return out_conf, out_argmax
+
+
+def fdllm_select_from_conf(conf: torch.Tensor, argmax: torch.Tensor, mask: torch.Tensor,
+                           param: float, mode=PROFILE, out_tokens=None, out_commit=None,
+                           out_n=None, stream=None):
+    """Steps a2-a5 alone on given confidences; returns (out_tokens, out_commit, out_n)."""
+    B, L = conf.shape
+    out_tokens, out_commit, out_n = _outputs(B, L, conf.device, out_tokens, out_commit, out_n)
+    st = _load().fdllm_select_from_conf(_dev(conf, "conf", torch.float32, (B, L)),
+                                     _dev(argmax, "argmax", torch.int32, (B, L)), B, L,
+                                     _dev(mask, "mask", torch.uint8, (B, L)), float(param),
+                                     _mode(mode),
+                                     _dev(out_tokens, "out_tokens", torch.int32, (B, L)),
+                                     _dev(out_commit, "out_commit", torch.uint8, (B, L)),
+                                     _dev(out_n, "out_n", torch.int32, (B,)), _stream(stream))
+    _check(st, "fdllm_select_from_conf")
+    return out_tokens, out_commit, out_n
+
+
+def fdllm_device_status(stream=None) -> int:
+    """Synchronises and returns (clearing it) the library workspace's sticky device status."""
+    return _load().fdllm_device_status(_stream(stream))
+
+
+def fdllm_workspace_status(workspace: torch.Tensor, stream=None) -> int:
+    return _load().fdllm_workspace_status(_dev(workspace, "workspace", torch.uint8), _stream(stream))
+
+
+def fdllm_release_workspace() -> None:
+    _load().fdllm_release_workspace()

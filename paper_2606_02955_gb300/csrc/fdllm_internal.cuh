@@ -1,0 +1,177 @@
+// fdllm_internal.cuh -- what the kernels and the C interface share: argument blocks,
+// workspace pieces, launch entry points and the per-row combination of unit results.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <cstdint>
+
+namespace fdllm {
+
+// ------------------------------------------------------------------ vocab reduction (a1)
+// Each row of logits is cut into units_per_row units of unit_vecs 16-byte vectors (the last
+// unit may be shorter), with units_per_row = ceil(row_bytes / kUnitTargetBytes).  A unit is
+// reduced by one CTA in a fixed order, so a row's result depends only on its bytes.  The
+// CTA streams a unit through a ring of shared-memory chunk buffers.
+constexpr int kSegQueue = 8;  // unit results queued from math warps to the epilogue warp
+constexpr int64_t kUnitTargetBytes = 65536;
+constexpr int kMaxGrid = 1024;
+constexpr int kMaxRows = 65536;
+constexpr int kMaskWords = kMaxRows / 32;
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr uint32_t kNoIdx = 0xFFFFFFFFu;
+
+// Reduction of one unit: max logit M, S = sum of 2^(x*log2e - fl(M*log2e)) over the unit
+// (fl = rounding to fp32) and the row-relative index of the first logit equal to M.
+struct UnitPartial {
+    float M;
+    float S;
+    uint32_t idx;
+    uint32_t pad;
+};
+
+struct VocabReduceArgs {
+    const uint8_t *logits;   // [rows, V] element size esize
+    const uint8_t *mask;     // [rows]
+    int64_t rows;            // B * L
+    int64_t row_bytes;       // V * esize
+    int64_t vec_per_row;     // row_bytes / 16
+    int32_t units_per_row;
+    int32_t unit_vecs;
+    UnitPartial *partials;   // [rows][units_per_row]; written for masked rows
+    uint32_t *next_unit;     // work counter: zero on entry, reset by the consumer kernel
+    uint32_t *status;        // sticky device error bits
+};
+
+struct UnitPlan {
+    int32_t units_per_row;
+    int32_t unit_vecs;
+};
+
+inline UnitPlan plan_units(int64_t row_bytes)
+{
+    const int64_t vpr = row_bytes / 16;
+    int64_t upr = (row_bytes + kUnitTargetBytes - 1) / kUnitTargetBytes;
+    if (upr < 1)
+        upr = 1;
+    const int64_t uv = (vpr + upr - 1) / upr;
+    return UnitPlan{(int32_t)upr, (int32_t)uv};
+}
+
+// Enqueue the vocab reduction on all SMs.
+cudaError_t launch_vocab_reduce(const VocabReduceArgs &a, int esize, cudaStream_t stream);
+
+// Per masked position: combine its unit partials, write (c, x_hat); resets next_unit.
+// Launched as a programmatic dependent of the vocab reduction.
+struct FinalizeArgs {
+    const uint8_t *mask;
+    int64_t rows;
+    int32_t units_per_row;
+    const UnitPartial *partials;
+    float *out_conf;
+    int32_t *out_tok;
+    uint32_t *next_unit;
+};
+
+cudaError_t launch_finalize(const FinalizeArgs &a, cudaStream_t stream);
+
+// ------------------------------------------------------------------ profile select (a2-a5)
+struct ProfileSelectArgs {
+    // Source of (c, x_hat): unit partials (from the vocab reduction, which this kernel then
+    // follows as a programmatic dependent launch) when `partials` is non-null, otherwise the
+    // given conf/tok arrays.
+    int32_t units_per_row;
+    const UnitPartial *partials;
+    uint32_t *next_unit;     // reset to zero when partials are consumed
+    const float *conf;       // [B, L]
+    const int32_t *tok;      // [B, L]
+    uint8_t *mask;           // [B, L], updated in place
+    int B;
+    int L;
+    int mode;
+    double param;
+    int32_t *out_tokens;     // [B, L]
+    uint8_t *out_commit;     // [B, L]
+    int32_t *out_n;          // [B]
+    const uint32_t *status;  // nullable: nonzero -> every row reports a device error
+};
+
+cudaError_t launch_profile_select(const ProfileSelectArgs &a, cudaStream_t stream);
+
+// ------------------------------------------------------------------ device helpers
+#ifdef __CUDACC__
+__device__ __forceinline__ float ex2_mufu(float x)
+{
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// S re-based from reference a2 to b2 (both already scaled by log2e): S * 2^(a2 - b2).
+__device__ __forceinline__ float rebase(float S, float a2, float b2)
+{
+    return S != 0.0f ? S * ex2_mufu(a2 - b2) : 0.0f;  // keeps NaN, avoids 0 * inf
+}
+
+// Position result from its units, folded in unit order (a fixed order, so identical rows
+// give identical bits): c = min(1/S, 1) (the max term alone is 1) and x_hat = the first
+// index attaining the max; c = NaN, x_hat = -1 when the row holds a NaN or its maximum is
+// +inf or -inf.
+__device__ __forceinline__ void combine_position(const UnitPartial *p, int upr, float &c,
+                                                 int32_t &tok)
+{
+    float Mj[8], Sj[8];
+    uint32_t Ij[8];
+    float M = -__int_as_float(0x7F800000);
+    float S = 0.0f;
+    uint32_t idx = kNoIdx;
+    for (int j0 = 0; j0 < upr; j0 += 8) {
+        const int cnt = upr - j0 < 8 ? upr - j0 : 8;
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+            if (j < cnt) {
+                const int4 r = __ldcg(reinterpret_cast<const int4 *>(p + j0 + j));
+                Mj[j] = __int_as_float(r.x);
+                Sj[j] = __int_as_float(r.y);
+                Ij[j] = (uint32_t)r.z;
+            }
+        float Mb = M;
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+            if (j < cnt)
+                Mb = fmaxf(Mb, Mj[j]);
+        const float Mb2 = Mb * kLog2e;
+        float Sb = rebase(S, M * kLog2e, Mb2);
+        uint32_t ib = (M == Mb) ? idx : kNoIdx;
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+            if (j < cnt) {
+                Sb += rebase(Sj[j], Mj[j] * kLog2e, Mb2);
+                if (Mj[j] == Mb && ib == kNoIdx)
+                    ib = Ij[j];
+            }
+        M = Mb;
+        S = Sb;
+        idx = ib;
+    }
+    c = __int_as_float(0x7FC00000);
+    tok = -1;
+    const bool finite = fabsf(M) <= 3.402823466e38f && fabsf(S) <= 3.402823466e38f;
+    if (!finite || !(S > 0.0f) || idx == kNoIdx)
+        return;
+    tok = (int32_t)idx;
+    c = fminf(1.0f / S, 1.0f);
+}
+
+// Programmatic dependent launch: the dependent grid's wait for the primary grid's results,
+// and the primary's permission for the dependent grid to start launching.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents()
+{
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+#endif
+
+}  // namespace fdllm

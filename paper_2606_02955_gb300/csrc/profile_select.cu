@@ -1,0 +1,222 @@
+// profile_select.cu -- steps a2-a5 of the selection for one batch row per CTA (paper
+// Algorithm 1: sort, scan, select, reveal):
+//   a2  sort the masked (c, position) pairs by c descending, position ascending: one 64-bit
+//       key per thread, bitonic network (warp shuffles for partner distance < 32, shared
+//       memory above);
+//   a3  prefix sums in fp64 over the sorted order (warp shuffles, then across warps):
+//       P_n = sum_{j<=n} (1 - c_(j)), so L_n = max{0, 1 - P_n} (= sum c - (n-1), Sec. 3),
+//       U_n = 1 - c_(n), G_n = L_n - U_n; factor: (n+1)(1 - c_(n)) < f; threshold: c_(n) >= tau;
+//   a4  n* = max{n : rule accepts n} (a block max, the literal definition), 1 if none;
+//   a5  reveal the first n* sorted positions: token, commit flag, mask cleared.
+// The row has L <= 1024 positions, so this is latency-bound work on a few KB.
+#include <cstdint>
+
+#include "fdllm_internal.cuh"
+
+namespace fdllm {
+namespace {
+
+constexpr uint64_t kPadKey = ~0ull;  // sorts after every real key
+
+// Masked: (~bits(c)) << 32 | pos — for c in (0, 1] larger c gives a smaller key, and equal
+// c falls back to the position.  Unmasked: 0xFFFFFFFF << 32 | pos, after every masked key.
+__device__ __forceinline__ uint64_t make_key(bool masked, float c, int pos)
+{
+    const uint32_t hi = masked ? ~__float_as_uint(c) : 0xFFFFFFFFu;
+    return ((uint64_t)hi << 32) | (uint32_t)pos;
+}
+
+__device__ __forceinline__ float key_conf(uint64_t key)
+{
+    return __uint_as_float(~(uint32_t)(key >> 32));
+}
+
+template <int T>
+__device__ __forceinline__ uint64_t bitonic_sort(uint64_t key, uint64_t *sk)
+{
+    const int t = threadIdx.x;
+#pragma unroll 1
+    for (int k = 2; k <= T; k <<= 1) {
+#pragma unroll 1
+        for (int j = k >> 1; j > 0; j >>= 1) {
+            uint64_t other;
+            if (j >= 32) {
+                sk[t] = key;
+                __syncthreads();
+                other = sk[t ^ j];
+                __syncthreads();
+            } else {
+                other = __shfl_xor_sync(0xFFFFFFFFu, key, j);
+            }
+            const bool ascending = (t & k) == 0;
+            const bool lower = (t & j) == 0;
+            const uint64_t lo = key < other ? key : other;
+            const uint64_t hi = key < other ? other : key;
+            key = (lower == ascending) ? lo : hi;
+        }
+    }
+    return key;
+}
+
+template <int T>
+__device__ __forceinline__ double block_inclusive_scan(double v, double *warp_tot)
+{
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const double u = __shfl_up_sync(0xFFFFFFFFu, v, o);
+        if (lane >= o)
+            v += u;
+    }
+    if constexpr (T > 32) {
+        if (lane == 31)
+            warp_tot[w] = v;
+        __syncthreads();
+        if (w == 0) {
+            double x = lane < T / 32 ? warp_tot[lane] : 0.0;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const double u = __shfl_up_sync(0xFFFFFFFFu, x, o);
+                if (lane >= o)
+                    x += u;
+            }
+            if (lane < T / 32)
+                warp_tot[lane] = x;  // inclusive over warps
+        }
+        __syncthreads();
+        if (w > 0)
+            v += warp_tot[w - 1];
+    }
+    return v;
+}
+
+template <int T>
+__device__ __forceinline__ int block_max(int v, int *warp_red)
+{
+    v = __reduce_max_sync(0xFFFFFFFFu, v);
+    if constexpr (T > 32) {
+        const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+        __syncthreads();  // warp_red may still be read from an earlier use
+        if (lane == 0)
+            warp_red[w] = v;
+        __syncthreads();
+        int x = lane < T / 32 ? warp_red[lane] : 0;
+        v = __reduce_max_sync(0xFFFFFFFFu, x);
+    }
+    return v;
+}
+
+template <int T>
+__global__ void __launch_bounds__(T) profile_select_kernel(const ProfileSelectArgs a)
+{
+    __shared__ uint64_t sk[T > 32 ? T : 1];
+    __shared__ int32_t s_tok[T];
+    __shared__ double warp_tot[32];
+    __shared__ int warp_red[32];
+
+    const int t = threadIdx.x;
+    const int L = a.L;
+    const int64_t base = (int64_t)blockIdx.x * L;
+
+    // (c, x_hat) of this thread's position: folded from the vocab reduction's unit
+    // partials, or read from the given arrays.
+    if (a.partials != nullptr)
+        pdl_wait();  // the vocab reduction's partials are complete and visible
+    const bool masked = t < L && a.mask[base + t] != 0;
+    float c = 0.0f;
+    int32_t tok = -1;
+    if (masked) {
+        if (a.partials != nullptr) {
+            combine_position(a.partials + (base + t) * a.units_per_row, a.units_per_row, c,
+                             tok);
+        } else {
+            c = a.conf[base + t];
+            tok = a.tok[base + t];
+        }
+    }
+    s_tok[t] = tok;
+    if (a.partials != nullptr && a.next_unit != nullptr && blockIdx.x == 0 && t == 0)
+        *a.next_unit = 0;  // the vocab reduction before this kernel has finished
+    const bool bad = masked && !(c > 0.0f && c <= 1.0f);  // NaN fails both
+    uint64_t key = t < L ? make_key(masked, c, t) : kPadKey;
+
+    const int m = __syncthreads_count(masked);
+    const int any_bad = __syncthreads_or(bad);
+    const bool dev_err = a.status != nullptr && *((volatile const uint32_t *)a.status) != 0;
+
+    key = bitonic_sort<T>(key, sk);
+
+    // Thread t now holds the (t+1)-th most confident masked position when t < m.
+    const int n = t + 1;
+    const bool live = t < m;
+    const double cn = live ? (double)key_conf(key) : 1.0;
+    const double one_minus = live ? 1.0 - cn : 0.0;
+    const double P = block_inclusive_scan<T>(one_minus, warp_tot);
+
+    bool ok = false;
+    if (live) {
+        if (a.mode == 0) {  // profile: G_n > delta, delta = 1 - f
+            const double delta = 1.0 - a.param;
+            const double Ln = fmax(0.0, 1.0 - P);
+            const double Un = 1.0 - cn;
+            ok = (Ln - Un) > delta;
+        } else if (a.mode == 1) {  // factor: (n+1)(1 - c_(n)) < f
+            ok = (double)(n + 1) * (1.0 - cn) < a.param;
+        } else {  // threshold: c_(n) >= tau
+            ok = cn >= a.param;
+        }
+    }
+    int nstar = block_max<T>(ok ? n : 0, warp_red);
+    if (m > 0 && nstar == 0)
+        nstar = 1;  // progress convention
+    if (any_bad)
+        nstar = -1;
+    if (dev_err)
+        nstar = -2;
+
+    if (t < L) {
+        const int pos = (int)(key & 0xFFFFFFFFu);
+        const bool commit = t < nstar;  // nstar <= m, so only masked keys qualify
+        a.out_commit[base + pos] = commit ? 1 : 0;
+        if (commit) {
+            a.out_tokens[base + pos] = s_tok[pos];
+            a.mask[base + pos] = 0;
+        }
+    }
+    if (t == 0)
+        a.out_n[blockIdx.x] = nstar;
+}
+
+template <int T>
+cudaError_t launch_t(const ProfileSelectArgs &a, cudaStream_t stream)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)a.B);
+    cfg.blockDim = dim3(T);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = a.partials != nullptr ? 1 : 0;  // a dependent of the vocab reduction
+    return cudaLaunchKernelEx(&cfg, profile_select_kernel<T>, a);
+}
+
+}  // namespace
+
+cudaError_t launch_profile_select(const ProfileSelectArgs &a, cudaStream_t stream)
+{
+    if (a.L <= 32)
+        return launch_t<32>(a, stream);
+    if (a.L <= 64)
+        return launch_t<64>(a, stream);
+    if (a.L <= 128)
+        return launch_t<128>(a, stream);
+    if (a.L <= 256)
+        return launch_t<256>(a, stream);
+    if (a.L <= 512)
+        return launch_t<512>(a, stream);
+    return launch_t<1024>(a, stream);
+}
+
+}  // namespace fdllm

@@ -1,0 +1,610 @@
+// vocab_reduce.cu -- step a1 of the selection: for every masked position, the argmax token
+// x_hat (lowest index on ties) and the confidence c = max_v softmax(v) = exp(M - lse)
+// (paper Sec. 3 "Notation"; Algorithm 1, confidence loop).
+//
+// Design (an HBM-bound streaming reduction; no tensor cores):
+//  * Work = the masked rows only.  Every CTA compacts the mask into a bitmap plus word prefix
+//    counts in shared memory and maps the r-th masked row to its global row.
+//  * Each row is cut into fixed units (about 64 KB, see plan_units); the units of all masked
+//    rows form one queue served by an atomic counter, so CTAs that run faster take more
+//    units and the tail is at most one unit.  A unit is reduced by one CTA in a fixed order,
+//    so a row's result depends only on its bytes (identical rows give identical bits, for any
+//    batch composition).
+//  * Warp 0 (one lane) streams each unit through a kStages-deep ring of kChunkBytes buffers
+//    with 1-D bulk copies (cp.async.bulk, completion on mbarriers); chunk metadata travels
+//    with the stage.
+//  * NW math warps read the ring with conflict-free 16-byte shared loads.  Per lane: running
+//    max and the index of its first vector; per warp: a lagging reference `ref` for the sum
+//    of 2^(x*log2e - ref2), raised (with one rescale) only when a logit exceeds it by
+//    kRebaseSlack, so a logit costs half a packed f32x2 FMA, one MUFU ex2 and half a packed
+//    f32x2 add; the vector max uses packed bf16x2 max for bf16.
+//  * At the end of a unit each math warp reduces its lanes (redux + shuffles) and queues
+//    (M, S, vec) for the epilogue warp, which combines the warps in a fixed order and stores
+//    the unit's partial.  The consumer kernel (profile select, or finalize) folds a position's
+//    units in unit order and resolves the argmax element inside the winning 16-byte vector.
+#include <cfloat>
+#include <cmath>
+#include <cstdio>
+#include <cstdlib>
+
+#include "fdllm_internal.cuh"
+#include "ptx.cuh"
+
+namespace fdllm {
+namespace {
+
+// A warp raises its sum reference only when a logit exceeds it by this much (natural-log
+// units); lane sums then stay below (terms per lane) * e^8, far from fp32 overflow.
+constexpr float kRebaseSlack = 8.0f;
+constexpr uint32_t kEndMarker = 0xFFFFFFFFu;
+
+__device__ __forceinline__ float fmax_nan(float a, float b)
+{
+    float r;
+    asm("max.NaN.f32 %0, %1, %2;" : "=f"(r) : "f"(a), "f"(b));
+    return r;
+}
+
+// Monotone map of floats onto unsigned integers (for warp max via redux).
+__device__ __forceinline__ uint32_t ordered(float f)
+{
+    const uint32_t b = __float_as_uint(f);
+    return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+
+__device__ __forceinline__ float unordered(uint32_t k)
+{
+    return __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
+}
+
+__device__ __forceinline__ uint32_t hmax2_nan(uint32_t a, uint32_t b)
+{
+    uint32_t d;
+    asm("max.NaN.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+    return d;
+}
+
+// Packed fp32 pairs (Blackwell f32x2 arithmetic); element order inside a pair is irrelevant
+// here because every operation is elementwise.
+__device__ __forceinline__ uint64_t pack2(float lo, float hi)
+{
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+
+__device__ __forceinline__ void unpack2(uint64_t v, float &lo, float &hi)
+{
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+
+__device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c)
+{
+    uint64_t d;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+    return d;
+}
+
+__device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b)
+{
+    uint64_t d;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+
+__device__ __forceinline__ uint64_t fmul2(uint64_t a, uint64_t b)
+{
+    uint64_t d;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+
+template <int ESIZE>
+struct VecOps;
+
+template <>
+struct VecOps<2> {  // 8 x bf16 per 16-byte vector; widening to fp32 is exact
+    static constexpr uint32_t kPadWord = 0xFF80FF80u;  // two bf16 -inf
+    // max of the 8 logits; NaN if any is NaN
+    __device__ __forceinline__ static float vmax(const uint4 &r)
+    {
+        const uint32_t m = hmax2_nan(hmax2_nan(r.x, r.y), hmax2_nan(r.z, r.w));
+        return fmax_nan(__uint_as_float(m << 16), __uint_as_float(m & 0xFFFF0000u));
+    }
+    __device__ __forceinline__ static uint64_t pair(uint32_t w)
+    {
+        return pack2(__uint_as_float(w << 16), __uint_as_float(w & 0xFFFF0000u));
+    }
+    __device__ __forceinline__ static void pairs(const uint4 &r, uint64_t (&p)[4])
+    {
+        p[0] = pair(r.x);
+        p[1] = pair(r.y);
+        p[2] = pair(r.z);
+        p[3] = pair(r.w);
+    }
+    // first element of the vector equal to M (8 if none)
+    __device__ __forceinline__ static uint32_t first_index(const uint4 &r, float M)
+    {
+        const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+        uint32_t hit = 8;
+#pragma unroll
+        for (int e = 7; e >= 0; --e) {
+            const uint32_t bits = (e & 1) ? (w[e >> 1] & 0xFFFF0000u) : (w[e >> 1] << 16);
+            if (__uint_as_float(bits) == M)
+                hit = e;
+        }
+        return hit;
+    }
+    static constexpr int kPairs = 4;
+    static constexpr int kElems = 8;
+};
+
+template <>
+struct VecOps<4> {  // 4 x fp32 per 16-byte vector
+    static constexpr uint32_t kPadWord = 0xFF800000u;  // fp32 -inf
+    __device__ __forceinline__ static float vmax(const uint4 &r)
+    {
+        return fmax_nan(fmax_nan(__uint_as_float(r.x), __uint_as_float(r.y)),
+                        fmax_nan(__uint_as_float(r.z), __uint_as_float(r.w)));
+    }
+    __device__ __forceinline__ static void pairs(const uint4 &r, uint64_t (&p)[2])
+    {
+        p[0] = ((uint64_t)r.y << 32) | r.x;
+        p[1] = ((uint64_t)r.w << 32) | r.z;
+    }
+    __device__ __forceinline__ static uint32_t first_index(const uint4 &r, float M)
+    {
+        const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+        uint32_t hit = 4;
+#pragma unroll
+        for (int e = 3; e >= 0; --e)
+            if (__uint_as_float(w[e]) == M)
+                hit = e;
+        return hit;
+    }
+    static constexpr int kPairs = 2;
+    static constexpr int kElems = 4;
+};
+
+// Partials held by lanes [0, count) (each S relative to its own M) -> one partial, combined
+// by a fixed butterfly.
+__device__ __forceinline__ UnitPartial warp_combine(UnitPartial p, bool valid)
+{
+    if (!valid) {
+        p.M = -INFINITY;
+        p.S = 0.0f;
+        p.idx = kNoIdx;
+    }
+    const float M = unordered(__reduce_max_sync(0xFFFFFFFFu, ordered(p.M)));
+    float s = rebase(p.S, p.M * kLog2e, M * kLog2e);
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1)
+        s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
+    UnitPartial r;
+    r.M = M;
+    r.S = s;
+    r.idx = __reduce_min_sync(0xFFFFFFFFu, p.M == M ? p.idx : kNoIdx);
+    r.pad = 0;
+    return r;
+}
+
+// Global row of the r-th masked row: the word holding it by binary search over the
+// exclusive word prefix counts, then the bit by rank within the word.
+__device__ __forceinline__ int64_t masked_row(uint32_t r, const uint32_t *bits,
+                                              const uint32_t *pref, int nwords)
+{
+    int lo = 0, hi = nwords - 1;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (pref[mid] <= r)
+            lo = mid;
+        else
+            hi = mid - 1;
+    }
+    const int bit = (int)__fns(bits[lo], 0, (int)(r - pref[lo]) + 1);
+    return (int64_t)lo * 32 + bit;
+}
+
+struct ChunkMeta {
+    uint32_t n;         // vectors in the chunk; 0 marks the end of the CTA's work
+    uint32_t vec_base;  // row-relative index of the chunk's first vector
+    uint32_t last;      // nonzero: last chunk of its unit
+    uint32_t pidx;      // partial slot of the unit: global row * units_per_row + unit
+};
+
+template <int NW, int STAGES>
+struct Smem {
+    uint64_t full[STAGES];
+    uint64_t empty[STAGES];
+    uint64_t seg_full[kSegQueue];
+    uint64_t seg_empty[kSegQueue];
+    ChunkMeta meta[STAGES];
+    UnitPartial seg[kSegQueue][NW];
+    uint32_t seg_pidx[kSegQueue];
+    uint32_t bits[kMaskWords];
+    uint32_t pref[kMaskWords + 1];
+};
+
+template <int NW, int STAGES, int CHUNK>
+constexpr size_t smem_bytes()
+{
+    return (size_t)STAGES * CHUNK + sizeof(Smem<NW, STAGES>);
+}
+
+// ESIZE: bytes per logit; NW: math warps; STAGES x CHUNK: the shared-memory ring;
+// EVICT: L2 evict-first hint on the stream.
+template <int ESIZE, int NW, int STAGES, int CHUNK, bool EVICT>
+__global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const VocabReduceArgs a)
+{
+    constexpr int kStages = STAGES;
+    constexpr int kChunkBytes = CHUNK;
+    constexpr int kChunkVecs = CHUNK / 16;
+    extern __shared__ __align__(128) uint8_t smem_raw[];
+    uint8_t *ring = smem_raw;
+    Smem<NW, STAGES> &sm =
+        *reinterpret_cast<Smem<NW, STAGES> *>(smem_raw + (size_t)kStages * kChunkBytes);
+    constexpr int kWarps = NW + 2;
+    using Ops = VecOps<ESIZE>;
+    constexpr int kP = Ops::kPairs;
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+
+    // The consumer kernel may start launching now; it waits for this grid's results.
+    if (threadIdx.x == 0)
+        pdl_launch_dependents();
+    // The producer's first unit request overlaps the mask compaction below.
+    uint32_t first_unit = 0;
+    if (threadIdx.x == 0)
+        first_unit = atomicAdd(a.next_unit, 1u);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(&sm.full[s], 1);
+            mbar_init(&sm.empty[s], NW);
+        }
+        for (int q = 0; q < kSegQueue; ++q) {
+            mbar_init(&sm.seg_full[q], NW);
+            mbar_init(&sm.seg_empty[q], 1);
+        }
+        fence_mbar_init();
+    }
+
+    // Mask -> bitmap (one ballot per 32 rows, four words in flight per warp) -> exclusive
+    // prefix count per word.
+    const int nwords = (int)((a.rows + 31) / 32);
+    for (int w0 = warp; w0 < nwords; w0 += 4 * kWarps) {
+        bool m[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int w = w0 + i * kWarps;
+            const int64_t r = (int64_t)w * 32 + lane;
+            m[i] = w < nwords && r < a.rows && a.mask[r] != 0;
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const uint32_t b = __ballot_sync(0xFFFFFFFFu, m[i]);
+            if (lane == 0 && w0 + i * kWarps < nwords)
+                sm.bits[w0 + i * kWarps] = b;
+        }
+    }
+    __syncthreads();
+    if (warp == 0) {
+        const int per = (nwords + 31) / 32;
+        const int w0 = lane * per;
+        uint32_t local = 0;
+        for (int k = 0; k < per; ++k)
+            if (w0 + k < nwords)
+                local += __popc(sm.bits[w0 + k]);
+        uint32_t incl = local;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t t = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+            if (lane >= o)
+                incl += t;
+        }
+        uint32_t run = incl - local;
+        for (int k = 0; k < per; ++k)
+            if (w0 + k < nwords) {
+                sm.pref[w0 + k] = run;
+                run += __popc(sm.bits[w0 + k]);
+            }
+        if (lane == 31)
+            sm.pref[nwords] = incl;
+    }
+    __syncthreads();
+
+    const uint32_t upr = (uint32_t)a.units_per_row;
+    const uint32_t total = sm.pref[nwords] * upr;  // host checks rows * upr < 2^31
+    if (total == 0)
+        return;  // (first_unit >= total then, so nothing was claimed)
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer (one lane)
+        if (lane != 0)
+            return;
+        uint64_t policy = 0;
+        if (EVICT)
+            policy = make_evict_first_policy();
+        uint32_t k = 0;
+        uint32_t u = first_unit;
+        while (u < total) {
+            const uint32_t u_next = atomicAdd(a.next_unit, 1u);  // in flight while u streams
+            const uint32_t r = u / upr, j = u - r * upr;
+            const int64_t grow = masked_row(r, sm.bits, sm.pref, nwords);
+            const int64_t v0 = (int64_t)j * a.unit_vecs;
+            const int64_t v1 = min(v0 + (int64_t)a.unit_vecs, a.vec_per_row);
+            const uint8_t *rowp = a.logits + grow * a.row_bytes;
+            for (int64_t v = v0; v < v1; v += kChunkVecs) {
+                const uint32_t n = (uint32_t)min((int64_t)kChunkVecs, v1 - v);
+                const uint32_t s = k % kStages;
+                if (k >= kStages && !mbar_wait(&sm.empty[s], ((k / kStages) - 1) & 1, a.status))
+                    return;  // math warps stopped; issued copies complete on their own
+                ChunkMeta cm;
+                cm.n = n;
+                cm.vec_base = (uint32_t)v;
+                cm.last = (v + n == v1) ? 1u : 0u;
+                cm.pidx = (uint32_t)(grow * upr + j);
+                sm.meta[s] = cm;
+                mbar_arrive_expect_tx(&sm.full[s], n * 16u);
+                if (EVICT)
+                    bulk_copy_g2s_hint(ring + (size_t)s * kChunkBytes, rowp + v * 16, n * 16u,
+                                       &sm.full[s], policy);
+                else
+                    bulk_copy_g2s(ring + (size_t)s * kChunkBytes, rowp + v * 16, n * 16u,
+                                  &sm.full[s]);
+                ++k;
+            }
+            u = u_next;
+        }
+        const uint32_t s = k % kStages;
+        if (k >= kStages && !mbar_wait(&sm.empty[s], ((k / kStages) - 1) & 1, a.status))
+            return;
+        ChunkMeta end;
+        end.n = 0;
+        end.vec_base = 0;
+        end.last = 1;
+        end.pidx = kEndMarker;
+        sm.meta[s] = end;
+        mbar_arrive(&sm.full[s]);
+    } else if (warp <= NW) {
+        // ------------------------------------------------------------ math warps
+        const int mw = warp - 1;
+        const int ct = threadIdx.x - 32;
+        constexpr int kPer = kChunkVecs / (NW * 32);
+        static_assert(kChunkVecs % (NW * 32) == 0, "chunk must split evenly over math warps");
+        const uint64_t log2e2 = pack2(kLog2e, kLog2e);
+        float m = -INFINITY;     // lane max (the first logit attaining it wins ties)
+        float mnan = -INFINITY;  // lane max propagating NaN (NaN detection, rebase trigger)
+        uint32_t idx = kNoIdx;   // row-relative index of that first logit
+        uint64_t acc[kP];
+        float ref = -FLT_MAX, ref2 = -FLT_MAX;  // warp-uniform reference
+#pragma unroll
+        for (int q = 0; q < kP; ++q)
+            acc[q] = 0;
+        uint32_t seg = 0;
+        for (uint32_t k = 0;; ++k) {
+            const uint32_t st = k % kStages;
+            if (!mbar_wait(&sm.full[st], (k / kStages) & 1, a.status))
+                return;
+            const ChunkMeta cm = sm.meta[st];
+            if (cm.n != 0) {
+                const uint4 *buf =
+                    reinterpret_cast<const uint4 *>(ring + (size_t)st * kChunkBytes);
+                const uint4 pad = make_uint4(Ops::kPadWord, Ops::kPadWord, Ops::kPadWord,
+                                             Ops::kPadWord);
+                uint4 raw[kPer];
+#pragma unroll
+                for (int it = 0; it < kPer; ++it) {
+                    const int v = ct + it * NW * 32;
+                    raw[it] = v < (int)cm.n ? buf[v] : pad;
+                }
+                // chunk max and its first vector (tree; the earlier vector wins ties)
+                float vm[kPer];
+                int vi[kPer];
+#pragma unroll
+                for (int it = 0; it < kPer; ++it) {
+                    vm[it] = Ops::vmax(raw[it]);
+                    vi[it] = it;
+                    mnan = fmax_nan(mnan, vm[it]);
+                }
+#pragma unroll
+                for (int w = 1; w < kPer; w *= 2)
+#pragma unroll
+                    for (int it = 0; it + w < kPer; it += 2 * w)
+                        if (vm[it + w] > vm[it]) {
+                            vm[it] = vm[it + w];
+                            vi[it] = vi[it + w];
+                        }
+                if (vm[0] > m) {  // rare after a unit's first chunk
+                    // the winning vector is still in the ring (the stage is not released yet)
+                    const int v = ct + vi[0] * NW * 32;
+                    m = vm[0];
+                    idx = (cm.vec_base + (uint32_t)v) * Ops::kElems +
+                          Ops::first_index(buf[v], m);
+                }
+                if (__any_sync(0xFFFFFFFFu, mnan > ref + kRebaseSlack)) {
+                    const float wmax = unordered(__reduce_max_sync(0xFFFFFFFFu, ordered(mnan)));
+                    const float r2 = wmax * kLog2e;
+                    const float f = ex2_mufu(ref2 - r2);
+                    const uint64_t f2 = pack2(f, f);
+#pragma unroll
+                    for (int q = 0; q < kP; ++q)
+                        acc[q] = fmul2(acc[q], f2);
+                    ref = wmax;
+                    ref2 = r2;
+                }
+                const uint64_t nref2 = pack2(-ref2, -ref2);
+#pragma unroll
+                for (int it = 0; it < kPer; ++it) {
+                    uint64_t p[kP];
+                    Ops::pairs(raw[it], p);
+#pragma unroll
+                    for (int q = 0; q < kP; ++q) {
+                        float t0, t1;
+                        unpack2(ffma2(p[q], log2e2, nref2), t0, t1);
+                        acc[q] = fadd2(acc[q], pack2(ex2_mufu(t0), ex2_mufu(t1)));
+                    }
+                }
+            }
+            __syncwarp();
+            if (cm.n != 0 && lane == 0)
+                mbar_arrive(&sm.empty[st]);
+            if (!cm.last)
+                continue;
+            // end of a unit (or of the CTA's work): hand the warp's result to the epilogue
+            const uint32_t q = seg % kSegQueue;
+            if (seg >= kSegQueue &&
+                !mbar_wait(&sm.seg_empty[q], ((seg / kSegQueue) - 1) & 1, a.status))
+                return;
+            float S = 0.0f;
+#pragma unroll
+            for (int j = 0; j < kP; ++j) {
+                float lo, hi;
+                unpack2(acc[j], lo, hi);
+                S += lo + hi;
+            }
+#pragma unroll
+            for (int o = 16; o >= 1; o >>= 1)
+                S += __shfl_xor_sync(0xFFFFFFFFu, S, o);
+            UnitPartial p;
+            p.M = unordered(__reduce_max_sync(0xFFFFFFFFu, ordered(m)));
+            // NaN anywhere poisons the sum; a warp that saw no finite logit adds exactly 0.
+            const bool bad = __any_sync(0xFFFFFFFFu, mnan != mnan);
+            p.S = bad ? __int_as_float(0x7FC00000)
+                      : (p.M == -INFINITY ? 0.0f : rebase(S, ref2, p.M * kLog2e));
+            p.idx = __reduce_min_sync(0xFFFFFFFFu, m == p.M ? idx : kNoIdx);
+            p.pad = 0;
+            if (lane == 0) {
+                sm.seg[q][mw] = p;
+                if (mw == 0)
+                    sm.seg_pidx[q] = cm.pidx;
+                mbar_arrive(&sm.seg_full[q]);
+            }
+            if (cm.n == 0)
+                return;
+            ++seg;
+            m = -INFINITY;
+            mnan = -INFINITY;
+            idx = kNoIdx;
+            ref = -FLT_MAX;
+            ref2 = -FLT_MAX;
+#pragma unroll
+            for (int j = 0; j < kP; ++j)
+                acc[j] = 0;
+        }
+    } else {
+        // ------------------------------------------------------------ epilogue warp
+        for (uint32_t seg = 0;; ++seg) {
+            const uint32_t q = seg % kSegQueue;
+            if (!mbar_wait(&sm.seg_full[q], (seg / kSegQueue) & 1, a.status))
+                return;
+            const uint32_t pidx = sm.seg_pidx[q];
+            UnitPartial p = {-INFINITY, 0.0f, kNoIdx, 0};
+            if (lane < NW)
+                p = sm.seg[q][lane];
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(&sm.seg_empty[q]);
+            if (pidx == kEndMarker)
+                return;
+            p = warp_combine(p, lane < NW);
+            if (lane == 0)
+                a.partials[pidx] = p;
+        }
+    }
+}
+
+__global__ void finalize_kernel(const FinalizeArgs a)
+{
+    pdl_wait();  // the vocab reduction's partials are complete and visible
+    if (blockIdx.x == 0 && threadIdx.x == 0)
+        *a.next_unit = 0;
+    const int64_t row = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (row >= a.rows || a.mask[row] == 0)
+        return;
+    float c;
+    int32_t tok;
+    combine_position(a.partials + row * a.units_per_row, a.units_per_row, c, tok);
+    a.out_conf[row] = c;
+    a.out_tok[row] = tok;
+}
+
+template <int ESIZE, int NW, int STAGES, int CHUNK, bool EVICT>
+cudaError_t launch_variant(const VocabReduceArgs &a, cudaStream_t stream)
+{
+    static int attr_done[64] = {0};
+    static int grid_cache[64] = {0};
+    int dev = 0;
+    cudaError_t err = cudaGetDevice(&dev);
+    if (err != cudaSuccess)
+        return err;
+    if (dev < 0 || dev >= 64)
+        return cudaErrorInvalidDevice;
+    constexpr size_t smem = smem_bytes<NW, STAGES, CHUNK>();
+    static_assert(smem <= 227 * 1024, "ring does not fit in shared memory");
+    auto *kern = vocab_reduce_kernel<ESIZE, NW, STAGES, CHUNK, EVICT>;
+    if (!attr_done[dev]) {
+        err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (err != cudaSuccess)
+            return err;
+        int sms = 0, per_sm = 0;
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, (NW + 2) * 32, smem);
+        int g = sms * (per_sm > 0 ? per_sm : 1);
+        grid_cache[dev] = g < kMaxGrid ? g : kMaxGrid;
+        attr_done[dev] = 1;
+    }
+    kern<<<grid_cache[dev], (NW + 2) * 32, smem, stream>>>(a);
+    return cudaGetLastError();
+}
+
+// Tuning table (math warps, ring stages x chunk bytes, L2 hint).  Entry 0 is the
+// configuration in use; FDLLM_K1_VARIANT=<index> selects another for measurements.
+template <int ESIZE>
+cudaError_t launch_esize(const VocabReduceArgs &a, cudaStream_t stream, int which)
+{
+    switch (which) {
+    case 1: return launch_variant<ESIZE, 16, 6, 32768, false>(a, stream);
+    case 2: return launch_variant<ESIZE, 16, 3, 65536, false>(a, stream);
+    case 3: return launch_variant<ESIZE, 8, 3, 65536, false>(a, stream);
+    case 4: return launch_variant<ESIZE, 16, 8, 24576, false>(a, stream);
+    case 5: return launch_variant<ESIZE, 16, 12, 16384, false>(a, stream);
+    case 6: return launch_variant<ESIZE, 8, 6, 32768, false>(a, stream);
+    case 7: return launch_variant<ESIZE, 16, 6, 32768, true>(a, stream);
+    default: return launch_variant<ESIZE, 16, 3, 65536, true>(a, stream);
+    }
+}
+
+int variant_index()
+{
+    static const int v = [] {
+        const char *e = std::getenv("FDLLM_K1_VARIANT");
+        return e ? std::atoi(e) : 0;
+    }();
+    return v;
+}
+
+}  // namespace
+
+cudaError_t launch_vocab_reduce(const VocabReduceArgs &a, int esize, cudaStream_t stream)
+{
+    const int which = variant_index();
+    return esize == 2 ? launch_esize<2>(a, stream, which) : launch_esize<4>(a, stream, which);
+}
+
+cudaError_t launch_finalize(const FinalizeArgs &a, cudaStream_t stream)
+{
+    const int threads = 256;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)((a.rows + threads - 1) / threads));
+    cfg.blockDim = dim3(threads);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, finalize_kernel, a);
+}
+
+}  // namespace fdllm

@@ -1,0 +1,109 @@
+"""The C interface on the host (no GPU): the library builds, loads, exports every function
+include/fdllm.h declares, and rejects bad arguments before touching the device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "fdllm.h")
+
+OK, ERR_ARG, ERR_ALIGN, ERR_WORKSPACE = 0, 1, 2, 5
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(fdllm_[a-z_]+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib(cuda_lib_path):
+    lib = ctypes.CDLL(cuda_lib_path)
+    p, i, d, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_double, ctypes.c_size_t
+    lib.fdllm_select.argtypes = [p, i, i, i, i, p, d, i, p, p, p, p]
+    lib.fdllm_select_ws.argtypes = [p, i, i, i, i, p, d, i, p, p, p, p, sz, p]
+    lib.fdllm_confidence.argtypes = [p, i, i, i, i, p, p, p, p]
+    lib.fdllm_select_from_conf.argtypes = [p, p, i, i, p, d, i, p, p, p, p]
+    lib.fdllm_workspace_bytes.argtypes = [i, i, i, i]
+    lib.fdllm_workspace_bytes.restype = sz
+    lib.fdllm_status_string.restype = ctypes.c_char_p
+    return lib
+
+
+def test_header_declares_the_interface():
+    names = declared_functions()
+    for must in ("fdllm_select", "fdllm_select_ws", "fdllm_workspace_bytes",
+                 "fdllm_confidence", "fdllm_select_from_conf"):
+        assert must in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    missing = [n for n in declared_functions() if not hasattr(lib, n)]
+    assert not missing, missing
+
+
+def test_version_and_status_strings(lib):
+    assert lib.fdllm_version() >= 100
+    for code in range(0, 7):
+        assert lib.fdllm_status_string(code)
+
+
+def test_workspace_bytes(lib):
+    a = lib.fdllm_workspace_bytes(64, 32, 126464, 0)
+    b = lib.fdllm_workspace_bytes(16, 1024, 126464, 1)
+    assert a % 256 == 0 and b % 256 == 0 and b > a > 8 * 64 * 32
+    assert lib.fdllm_workspace_bytes(0, 32, 126464, 0) == 0
+
+
+# Fake device addresses: the argument checks reject these calls before any CUDA call.
+A16 = 0x10000
+A2 = 0x10002
+
+
+@pytest.mark.parametrize("args,want", [
+    ((A16, 0, 0, 32, 1024), ERR_ARG),          # B = 0
+    ((A16, 0, 2, 0, 1024), ERR_ARG),           # L = 0
+    ((A16, 0, 2, 1025, 1024), ERR_ARG),        # L > 1024
+    ((A16, 0, 128, 1024, 1024), ERR_ARG),      # B * L > 65536
+    ((A16, 0, 2, 32, 0), ERR_ARG),             # V = 0
+    ((A16, 2, 2, 32, 1024), ERR_ARG),          # unknown dtype
+    ((None, 0, 2, 32, 1024), ERR_ARG),         # null logits
+    ((A2, 0, 2, 32, 1024), ERR_ALIGN),         # logits not 16-byte aligned
+    ((A16, 0, 2, 32, 1001), ERR_ALIGN),        # V * 2 not a multiple of 16
+    ((A16, 1, 2, 32, 1002), ERR_ALIGN),        # V * 4 not a multiple of 16
+])
+def test_select_rejects_bad_shapes(lib, args, want):
+    logits, dtype, B, L, V = args
+    st = lib.fdllm_select(logits, dtype, B, L, V, A16, 1.0, 0, A16, A16, A16, None)
+    assert st == want
+
+
+def test_select_rejects_bad_mode_param_and_outputs(lib):
+    call = lambda mode, param, out=A16, mask=A16: lib.fdllm_select(
+        A16, 0, 2, 32, 1024, mask, param, mode, out, A16, A16, None)
+    assert call(3, 1.0) == ERR_ARG
+    assert call(-1, 1.0) == ERR_ARG
+    assert call(0, float("nan")) == ERR_ARG
+    assert call(0, float("inf")) == ERR_ARG
+    assert call(0, 1.0, out=None) == ERR_ARG
+    assert call(0, 1.0, mask=None) == ERR_ARG
+
+
+def test_select_ws_rejects_small_or_misaligned_workspace(lib):
+    need = lib.fdllm_workspace_bytes(2, 32, 1024, 0)
+    f = lambda ws, n: lib.fdllm_select_ws(A16, 0, 2, 32, 1024, A16, 1.0, 0, A16, A16, A16, ws,
+                                          n, None)
+    assert f(None, need) == ERR_WORKSPACE
+    assert f(A16 + 16, need) == ERR_WORKSPACE
+    assert f(A16, need - 1) == ERR_WORKSPACE
+
+
+def test_confidence_and_select_from_conf_reject(lib):
+    assert lib.fdllm_confidence(A2, 0, 2, 32, 1024, A16, A16, A16, None) == ERR_ALIGN
+    assert lib.fdllm_confidence(A16, 0, 2, 32, 1024, None, A16, A16, None) == ERR_ARG
+    assert lib.fdllm_select_from_conf(A16, A16, 2, 2000, A16, 1.0, 0, A16, A16, A16,
+                                      None) == ERR_ARG
+    assert lib.fdllm_select_from_conf(None, A16, 2, 32, A16, 1.0, 0, A16, A16, A16,
+                                      None) == ERR_ARG

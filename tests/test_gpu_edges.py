@@ -1,0 +1,133 @@
+"""Edge cases of the CUDA path against the oracle: empty and single-position rows, maximal
+L and row counts, the smallest vocabulary, -inf and non-finite logits, all-equal logits,
+maxima tied across CTA boundaries and in the ragged tail."""
+import numpy as np
+import pytest
+import torch
+
+import fdllm_synth as syn
+from gpu_util import check_confidence, check_select
+
+pytestmark = pytest.mark.gpu
+PROFILE, FACTOR, THRESHOLD = 0, 1, 2
+
+
+def _bf16(x: np.ndarray) -> torch.Tensor:
+    return torch.from_numpy(x).to(torch.bfloat16).cuda()
+
+
+def test_all_rows_unmasked(fd, orc):
+    logits = torch.randn(4, 16, 1024, device="cuda", dtype=torch.bfloat16)
+    mask = torch.zeros(4, 16, dtype=torch.uint8, device="cuda")
+    tok, commit, n = fd.fdllm_select(logits, mask, 0.75, PROFILE)
+    assert n.cpu().tolist() == [0, 0, 0, 0]
+    assert commit.sum().item() == 0 and mask.sum().item() == 0
+    assert torch.all(tok == -1)
+
+
+@pytest.mark.parametrize("L", [1, 2, 31, 32, 33, 1024])
+def test_row_lengths(fd, orc, L):
+    w = syn.Workload("len", 2, L, 2048, "bf16", 1.0, "target", 0.3, 4.0)
+    logits = syn.make_logits(w, seed=L, device="cuda")
+    mask_np = np.ones((2, L), np.uint8)
+    mask_np[1, ::3] = 0
+    for mode, p in ((PROFILE, 0.75), (FACTOR, 0.75), (THRESHOLD, 0.9)):
+        check_select(fd, orc, logits, mask_np, mode, p)
+
+
+def test_max_rows_and_min_vocab(fd, orc):
+    """B * L = 65536 rows of V = 8 bf16 (one 16-byte vector per row)."""
+    B, L, V = 64, 1024, 8
+    x = np.random.default_rng(1).normal(0, 2, (B, L, V)).astype(np.float32)
+    logits = _bf16(x)
+    mask_np = (np.random.default_rng(2).random((B, L)) < 0.5).astype(np.uint8)
+    check_confidence(fd, orc, logits, mask_np)
+    check_select(fd, orc, logits, mask_np, PROFILE, 0.75)
+
+
+def test_fp32_min_vocab(fd, orc):
+    x = np.random.default_rng(3).normal(0, 2, (3, 40, 4)).astype(np.float32)
+    check_confidence(fd, orc, torch.from_numpy(x).cuda(), np.ones((3, 40), np.uint8))
+
+
+def test_equal_logits_give_uniform_confidence(fd):
+    V = 126464
+    logits = torch.full((1, 3, V), 0.5, device="cuda", dtype=torch.bfloat16)
+    conf, tok = fd.fdllm_confidence(logits, torch.ones(1, 3, dtype=torch.uint8, device="cuda"))
+    assert torch.all(tok == 0)
+    assert torch.allclose(conf.double(), torch.full_like(conf.double(), 1.0 / V), rtol=1e-5,
+                          atol=0)
+
+
+def test_nonfinite_rows(fd, orc):
+    V = 4096
+    x = np.random.default_rng(4).normal(0, 1, (3, 4, V)).astype(np.float32)
+    x[0, 1, 100] = np.nan       # row 0 invalid
+    x[1, 2, :] = -np.inf        # row 1 invalid (max is -inf)
+    x[2, 0, ::2] = -np.inf      # row 2 fine: -inf entries contribute nothing
+    x[2, 3, 4000] = np.inf      # ... but +inf makes row 2 invalid too
+    logits = torch.from_numpy(x).cuda()
+    mask_np = np.ones((3, 4), np.uint8)
+    check_confidence(fd, orc, logits, mask_np)
+    mask = torch.from_numpy(mask_np.copy()).cuda()
+    tok, commit, n = fd.fdllm_select(logits, mask, 0.75, PROFILE)
+    assert n.cpu().tolist() == [fd.ROW_NONFINITE] * 3
+    assert commit.sum().item() == 0 and mask.sum().item() == 12
+    # -inf entries alone are fine
+    x[2, 3, 4000] = 0.0
+    x[0, 1, 100] = 0.0
+    x[1, 2, :] = 0.0
+    logits = torch.from_numpy(x).cuda()
+    check_confidence(fd, orc, logits, mask_np)
+    check_select(fd, orc, logits, mask_np, PROFILE, 0.75)
+
+
+def test_argmax_ties_across_chunks_and_ctas(fd, orc):
+    """Equal maxima far apart in a row (different chunks and, at this size, different CTAs),
+    and maxima in the last, ragged chunk: the lowest index must win."""
+    V = 126464
+    rng = np.random.default_rng(5)
+    x = rng.normal(0, 1, (2, 6, V)).astype(np.float32)
+    x[0, 0, [V - 1, 70000, 9000]] = 20.0
+    x[0, 1, [V - 1]] = 20.0
+    x[0, 2, [0, V - 1]] = 20.0
+    x[0, 3, [8191, 8192, 16384]] = 20.0
+    x[0, 4, [V - 8, V - 7]] = 20.0
+    x[0, 5, :] = 3.0
+    x[1] = x[0, ::-1]
+    for dt in ("bf16", "fp32"):
+        logits = _bf16(x) if dt == "bf16" else torch.from_numpy(x).cuda()
+        _, g_tok, _, _ = check_confidence(fd, orc, logits, np.ones((2, 6), np.uint8))
+        assert g_tok[0, :5].tolist() == [9000, V - 1, 0, 8191, V - 8]
+        assert g_tok[0, 5] == 0
+
+
+def test_large_rows_many_ctas_fp32(fd, orc):
+    """Few long rows: every row spans many CTAs, so the split-row combination decides."""
+    w = syn.Workload("long", 1, 3, 1 << 20, "fp32", 1.0, "target", 0.3, 4.0)
+    logits = syn.make_logits(w, seed=6, device="cuda")
+    check_confidence(fd, orc, logits, np.ones((1, 3), np.uint8))
+
+
+def test_bad_arguments_raise(fd):
+    logits = torch.randn(2, 4, 1000, device="cuda", dtype=torch.bfloat16)
+    mask = torch.ones(2, 4, dtype=torch.uint8, device="cuda")
+    with pytest.raises(fd.FdllmError) as e:
+        fd.fdllm_select(logits, mask, 1.0, 7)
+    assert e.value.status == 1
+    with pytest.raises(fd.FdllmError) as e:
+        fd.fdllm_select(logits, mask, float("nan"), 0)
+    assert e.value.status == 1
+
+
+def test_misaligned_logits_rejected(fd):
+    base = torch.randn(2 * 4 * 1000 + 8, device="cuda", dtype=torch.bfloat16)
+    logits = base[1:1 + 2 * 4 * 1000].view(2, 4, 1000)
+    mask = torch.ones(2, 4, dtype=torch.uint8, device="cuda")
+    with pytest.raises(fd.FdllmError) as e:
+        fd.fdllm_select(logits, mask, 1.0, PROFILE)
+    assert e.value.status == 2
+    with pytest.raises(fd.FdllmError) as e:
+        fd.fdllm_select(torch.randn(2, 4, 999, device="cuda", dtype=torch.bfloat16), mask, 1.0,
+                        PROFILE)
+    assert e.value.status == 2
