@@ -50,6 +50,15 @@ def aggregate(rows_per_rank: int, steps: int, times_s: list[float]) -> dict:
     return {"value": rows_per_rank * steps * n / t, "seconds": t, "n_ranks": n}
 
 
+def gather_times(dist, t_s: float, device) -> list[float]:
+    """Every rank's timed seconds, in rank order (all_gather of one float64 per rank)."""
+    import torch
+    t = torch.tensor([t_s], dtype=torch.float64, device=device)
+    out = [torch.zeros_like(t) for _ in range(dist.get_world_size())]
+    dist.all_gather(out, t)
+    return [float(x.item()) for x in out]
+
+
 def rank_seed(base: int, rank: int) -> int:
     """Each rank draws its own batch (weak scaling: independent problems per GPU)."""
     return base + 7919 * rank
@@ -246,12 +255,7 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
         time.sleep(0.12)
         sampler.stop()
 
-    times = [t_step]
-    if dist is not None:
-        tt = torch.tensor([t_step], dtype=torch.float64, device=dev)
-        gathered = [torch.zeros_like(tt) for _ in range(world)]
-        dist.all_gather(gathered, tt)
-        times = [float(x.item()) for x in gathered]
+    times = gather_times(dist, t_step, dev) if dist is not None else [t_step]
     agg = aggregate(w.B, steps, times)
     ms_per_step = agg["seconds"] / steps * 1e3
 
