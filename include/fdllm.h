@@ -109,6 +109,36 @@ fdllm_status fdllm_select_ws(const void *logits, int dtype, int B, int L, int V,
                              int32_t *out_n, void *workspace, size_t workspace_bytes,
                              void *stream);
 
+/* Scratch of fdllm_select_static: a fixed device array of this many bytes. */
+#define FDLLM_STATIC_SCRATCH_BYTES (8u << 20)
+
+/* fdllm_select without any allocation, for callers that must not allocate device memory
+ * while they run steps: a serving process that reserves all of its memory up front and
+ * forbids allocation afterwards, code running under an external allocator that owns the
+ * device (a framework's memory pool, a fixed memory budget), or a caller that cannot hand
+ * the library a workspace of its own.  (The paper has no counterpart: this is a property
+ * of the library, not of the method.)
+ *
+ * Arguments and results are exactly those of fdllm_select.  The scratch memory is a fixed
+ * array of FDLLM_STATIC_SCRATCH_BYTES bytes compiled into the library; every GPU that loads
+ * the library holds it until the process exits.  A shape whose scratch need,
+ * fdllm_workspace_bytes(B, L, V, dtype), exceeds that size is rejected with
+ * FDLLM_ERR_WORKSPACE before anything is enqueued.  8 MiB covers, for example, every bf16
+ * shape with V <= 126464 (up to B * L = 65536 rows) and fp32 V = 126464 up to
+ * B * L = 32768 rows.
+ * The call allocates nothing: no cudaMalloc, no cudaFree, no allocating library routine.
+ *
+ * The first call on a device looks up the array's device address (cudaGetSymbolAddress)
+ * with that device current and caches it; make that first call before any stream capture.
+ * Every call clears the array's status word and work counter on `stream` before its
+ * kernels run.  All calls on a device share the one array, which keeps the last call's
+ * contents: calls whose work overlaps on the GPU (different streams without ordering
+ * between them) race on it and produce wrong results; order such calls on one stream or
+ * with events. */
+fdllm_status fdllm_select_static(const void *logits, int dtype, int B, int L, int V,
+                                 uint8_t *mask, double param, int mode, int32_t *out_tokens,
+                                 uint8_t *out_commit, int32_t *out_n, void *stream);
+
 /* Step a1 alone (Sec. 3 "Notation"; Alg. 1 confidence loop): for every masked position,
  * out_conf = c = max softmax probability (fp32) and out_argmax = x_hat (int32, lowest index
  * among equal maxima).  Both [B, L] device arrays, written only at masked positions; a

@@ -182,6 +182,31 @@ fdllm_status read_and_clear_status(uint32_t *status, cudaStream_t stream)
     return FDLLM_ERR_DEVICE;
 }
 
+// Scratch for fdllm_select_static: a fixed array in device memory that every GPU loading
+// this library holds until the process exits, so that a selection step needs no
+// allocation at call time.  Host code only ever sees a host-side stand-in for the symbol;
+// the device address comes from cudaGetSymbolAddress, looked up once per device.
+static __device__ __align__(256) uint8_t g_static_scratch[FDLLM_STATIC_SCRATCH_BYTES];
+
+void *g_static_scratch_addr[kMaxDevices] = {nullptr};
+std::mutex g_static_mutex;
+
+fdllm_status static_scratch_address(void **out)
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices)
+        return FDLLM_ERR_CUDA;
+    std::lock_guard<std::mutex> lock(g_static_mutex);
+    if (g_static_scratch_addr[dev] == nullptr) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || p == nullptr)
+            return FDLLM_ERR_CUDA;
+        g_static_scratch_addr[dev] = p;
+    }
+    *out = g_static_scratch_addr[dev];
+    return FDLLM_OK;
+}
+
 }  // namespace
 }  // namespace fdllm
 
@@ -228,6 +253,30 @@ fdllm_status fdllm_select(const void *logits, int dtype, int B, int L, int V, ui
     st = owned_workspace(lay.total, s, &ws);
     if (st != FDLLM_OK)
         return st;
+    return run_select(logits, dtype, B, L, V, mask, param, mode, out_tokens, out_commit, out_n,
+                      static_cast<uint8_t *>(ws), lay, s);
+}
+
+fdllm_status fdllm_select_static(const void *logits, int dtype, int B, int L, int V,
+                                 uint8_t *mask, double param, int mode, int32_t *out_tokens,
+                                 uint8_t *out_commit, int32_t *out_n, void *stream)
+{
+    fdllm_status st = check_select_args(logits, dtype, B, L, V, mask, param, mode, out_tokens,
+                                        out_commit, out_n);
+    if (st != FDLLM_OK)
+        return st;
+    const Layout lay = layout_for((int64_t)B * L, (int64_t)V * esize_of(dtype));
+    if (lay.total > (size_t)FDLLM_STATIC_SCRATCH_BYTES)
+        return FDLLM_ERR_WORKSPACE;  // shape needs more scratch than the fixed array holds
+    void *ws = nullptr;
+    st = static_scratch_address(&ws);
+    if (st != FDLLM_OK)
+        return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    // The array keeps the previous call's contents: zero the status word and the work
+    // counter (the header block) before the kernels read them.
+    if (cudaMemsetAsync(ws, 0, kAlign, s) != cudaSuccess)
+        return FDLLM_ERR_CUDA;
     return run_select(logits, dtype, B, L, V, mask, param, mode, out_tokens, out_commit, out_n,
                       static_cast<uint8_t *>(ws), lay, s);
 }
