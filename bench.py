@@ -329,6 +329,59 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
     return result
 
 
+# ----------------------------------------------------------------------------- loop mode
+def run_loop(args) -> dict:
+    """Selection + commit repeated until no mask remains, for the profile and the factor
+    rule (f = args.param): steps taken and per-step selection latency.  Logits are
+    regenerated from (seed, step) before each step, outside the timed region; each step's
+    selection is timed with CUDA events on its stream."""
+    import numpy as np
+    import torch
+
+    import fdllm_synth as syn
+    import paper_2606_02955_gb300 as fd
+
+    w = syn.WORKLOADS[args.workload]
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.Stream(device=dev)
+    out = {}
+    for mode_name, mode in (("profile", fd.PROFILE), ("factor", fd.FACTOR)):
+        mask = torch.from_numpy(syn.make_mask(w, seed=4321)).to(dev)
+        tok = torch.full((w.B, w.L), -1, dtype=torch.int32, device=dev)
+        commit = torch.empty((w.B, w.L), dtype=torch.uint8, device=dev)
+        n = torch.empty((w.B,), dtype=torch.int32, device=dev)
+        times, masked, step = [], [], 0
+        while True:
+            remaining = int(mask.sum().item())
+            if remaining == 0 or step >= w.L + 1:
+                break
+            logits = syn.make_logits(w, seed=4321, device=dev, step=step)
+            torch.cuda.synchronize()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            fd.fdllm_select(logits, mask, args.param, mode, tok, commit, n, stream=stream)
+            e1.record(stream)
+            e1.synchronize()
+            times.append(e0.elapsed_time(e1))
+            masked.append(remaining)
+            del logits
+            step += 1
+        t = np.array(times)
+        first_bytes = masked[0] * w.V * w.elem_bytes
+        out[mode_name] = {
+            "steps": step, "finished": remaining == 0,
+            "per_step_ms_median": float(np.median(t)), "per_step_ms_mean": float(t.mean()),
+            "first_step_ms": float(t[0]), "total_selection_ms": float(t.sum()),
+            "first_step_logits_gbs": first_bytes / (t[0] * 1e-3) / 1e9,
+            "tokens_per_step": float(w.B * w.L / max(step, 1)),
+        }
+    return {"metric": "full-sequence loop: steps until no mask remains and per-step "
+                      "selection latency", "workload": w.name, "B": w.B, "L": w.L, "V": w.V,
+            "dtype": w.dtype, "param": args.param, "data": "synthetic", "results": out}
+
+
 # ----------------------------------------------------------------------------- oracle arm
 def oracle_sample_rows(args) -> int:
     return max(1, min(args.sample_rows, 64))
@@ -418,7 +471,15 @@ def main(argv=None):
     ap.add_argument("--sample-rows", type=int, default=4,
                     help="batch rows per oracle step (reference arm / CPU baseline)")
     ap.add_argument("--cpu-budget-s", type=float, default=10.0)
+    ap.add_argument("--loop", action="store_true",
+                    help="run the selection until no mask remains (profile vs factor) and "
+                         "report steps and per-step latency instead of the throughput line")
     args = ap.parse_args(argv)
+    if args.loop:
+        if args.workload == "serving_b64_l32_bf16":
+            args.workload = "full_seq_b16_l1024_fp32"
+        print(json.dumps(run_loop(args)), flush=True)
+        return
 
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
