@@ -50,13 +50,22 @@ struct UnitPlan {
     int32_t unit_vecs;
 };
 
+// Unit lengths are rounded up to a multiple of kUnitAlignVecs vectors (8 KB), so that every
+// unit but a row's last one fills whole chunks; the unit count is then recomputed so that
+// no unit is empty.
+constexpr int64_t kUnitAlignVecs = 512;
+
 inline UnitPlan plan_units(int64_t row_bytes)
 {
     const int64_t vpr = row_bytes / 16;
     int64_t upr = (row_bytes + kUnitTargetBytes - 1) / kUnitTargetBytes;
     if (upr < 1)
         upr = 1;
-    const int64_t uv = (vpr + upr - 1) / upr;
+    int64_t uv = (vpr + upr - 1) / upr;
+    uv = (uv + kUnitAlignVecs - 1) / kUnitAlignVecs * kUnitAlignVecs;
+    upr = (vpr + uv - 1) / uv;
+    if (upr < 1)
+        upr = 1;
     return UnitPlan{(int32_t)upr, (int32_t)uv};
 }
 

@@ -26,6 +26,7 @@
 #include <cmath>
 #include <cstdio>
 #include <cstdlib>
+#include <type_traits>
 
 #include "fdllm_internal.cuh"
 #include "ptx.cuh"
@@ -381,6 +382,65 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
 #pragma unroll
         for (int q = 0; q < kP; ++q)
             acc[q] = 0;
+
+        // One chunk: vector maxima and the first maximal logit, the reference update, then
+        // 2^(x*log2e - ref2) accumulated.  FULL: every vector of the chunk exists.
+        auto process_chunk = [&](auto full_tag, const uint4 *buf, const ChunkMeta &cm) {
+            constexpr bool FULL = decltype(full_tag)::value;
+            const uint4 pad = make_uint4(Ops::kPadWord, Ops::kPadWord, Ops::kPadWord,
+                                         Ops::kPadWord);
+            uint4 raw[kPer];
+#pragma unroll
+            for (int it = 0; it < kPer; ++it) {
+                const int v = ct + it * NW * 32;
+                raw[it] = (FULL || v < (int)cm.n) ? buf[v] : pad;
+            }
+            float vm[kPer];
+            int vi[kPer];
+#pragma unroll
+            for (int it = 0; it < kPer; ++it) {
+                vm[it] = Ops::vmax(raw[it]);
+                vi[it] = it;
+                mnan = fmax_nan(mnan, vm[it]);
+            }
+#pragma unroll
+            for (int w = 1; w < kPer; w *= 2)
+#pragma unroll
+                for (int it = 0; it + w < kPer; it += 2 * w)
+                    if (vm[it + w] > vm[it]) {
+                        vm[it] = vm[it + w];
+                        vi[it] = vi[it + w];
+                    }
+            if (vm[0] > m) {  // rare after a unit's first chunk
+                // the winning vector is still in the ring (the stage is not released yet)
+                const int v = ct + vi[0] * NW * 32;
+                m = vm[0];
+                idx = (cm.vec_base + (uint32_t)v) * Ops::kElems + Ops::first_index(buf[v], m);
+            }
+            if (__any_sync(0xFFFFFFFFu, mnan > ref + kRebaseSlack)) {
+                const float wmax = unordered(__reduce_max_sync(0xFFFFFFFFu, ordered(mnan)));
+                const float r2 = wmax * kLog2e;
+                const float f = ex2_mufu(ref2 - r2);
+                const uint64_t f2 = pack2(f, f);
+#pragma unroll
+                for (int q = 0; q < kP; ++q)
+                    acc[q] = fmul2(acc[q], f2);
+                ref = wmax;
+                ref2 = r2;
+            }
+            const uint64_t nref2 = pack2(-ref2, -ref2);
+#pragma unroll
+            for (int it = 0; it < kPer; ++it) {
+                uint64_t p[kP];
+                Ops::pairs(raw[it], p);
+#pragma unroll
+                for (int q = 0; q < kP; ++q) {
+                    float t0, t1;
+                    unpack2(ffma2(p[q], log2e2, nref2), t0, t1);
+                    acc[q] = fadd2(acc[q], pack2(ex2_mufu(t0), ex2_mufu(t1)));
+                }
+            }
+        };
         uint32_t seg = 0;
         for (uint32_t k = 0;; ++k) {
             const uint32_t st = k % kStages;
@@ -390,61 +450,10 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
             if (cm.n != 0) {
                 const uint4 *buf =
                     reinterpret_cast<const uint4 *>(ring + (size_t)st * kChunkBytes);
-                const uint4 pad = make_uint4(Ops::kPadWord, Ops::kPadWord, Ops::kPadWord,
-                                             Ops::kPadWord);
-                uint4 raw[kPer];
-#pragma unroll
-                for (int it = 0; it < kPer; ++it) {
-                    const int v = ct + it * NW * 32;
-                    raw[it] = v < (int)cm.n ? buf[v] : pad;
-                }
-                // chunk max and its first vector (tree; the earlier vector wins ties)
-                float vm[kPer];
-                int vi[kPer];
-#pragma unroll
-                for (int it = 0; it < kPer; ++it) {
-                    vm[it] = Ops::vmax(raw[it]);
-                    vi[it] = it;
-                    mnan = fmax_nan(mnan, vm[it]);
-                }
-#pragma unroll
-                for (int w = 1; w < kPer; w *= 2)
-#pragma unroll
-                    for (int it = 0; it + w < kPer; it += 2 * w)
-                        if (vm[it + w] > vm[it]) {
-                            vm[it] = vm[it + w];
-                            vi[it] = vi[it + w];
-                        }
-                if (vm[0] > m) {  // rare after a unit's first chunk
-                    // the winning vector is still in the ring (the stage is not released yet)
-                    const int v = ct + vi[0] * NW * 32;
-                    m = vm[0];
-                    idx = (cm.vec_base + (uint32_t)v) * Ops::kElems +
-                          Ops::first_index(buf[v], m);
-                }
-                if (__any_sync(0xFFFFFFFFu, mnan > ref + kRebaseSlack)) {
-                    const float wmax = unordered(__reduce_max_sync(0xFFFFFFFFu, ordered(mnan)));
-                    const float r2 = wmax * kLog2e;
-                    const float f = ex2_mufu(ref2 - r2);
-                    const uint64_t f2 = pack2(f, f);
-#pragma unroll
-                    for (int q = 0; q < kP; ++q)
-                        acc[q] = fmul2(acc[q], f2);
-                    ref = wmax;
-                    ref2 = r2;
-                }
-                const uint64_t nref2 = pack2(-ref2, -ref2);
-#pragma unroll
-                for (int it = 0; it < kPer; ++it) {
-                    uint64_t p[kP];
-                    Ops::pairs(raw[it], p);
-#pragma unroll
-                    for (int q = 0; q < kP; ++q) {
-                        float t0, t1;
-                        unpack2(ffma2(p[q], log2e2, nref2), t0, t1);
-                        acc[q] = fadd2(acc[q], pack2(ex2_mufu(t0), ex2_mufu(t1)));
-                    }
-                }
+                if (cm.n == (uint32_t)kChunkVecs)
+                    process_chunk(std::true_type{}, buf, cm);
+                else
+                    process_chunk(std::false_type{}, buf, cm);
             }
             __syncwarp();
             if (cm.n != 0 && lane == 0)
@@ -564,13 +573,9 @@ template <int ESIZE>
 cudaError_t launch_esize(const VocabReduceArgs &a, cudaStream_t stream, int which)
 {
     switch (which) {
-    case 1: return launch_variant<ESIZE, 16, 6, 32768, false>(a, stream);
-    case 2: return launch_variant<ESIZE, 16, 3, 65536, false>(a, stream);
-    case 3: return launch_variant<ESIZE, 8, 3, 65536, false>(a, stream);
-    case 4: return launch_variant<ESIZE, 16, 8, 24576, false>(a, stream);
-    case 5: return launch_variant<ESIZE, 16, 12, 16384, false>(a, stream);
-    case 6: return launch_variant<ESIZE, 8, 6, 32768, false>(a, stream);
-    case 7: return launch_variant<ESIZE, 16, 6, 32768, true>(a, stream);
+    case 1: return launch_variant<ESIZE, 16, 3, 65536, false>(a, stream);
+    case 2: return launch_variant<ESIZE, 8, 3, 65536, true>(a, stream);
+    case 3: return launch_variant<ESIZE, 16, 6, 32768, true>(a, stream);
     default: return launch_variant<ESIZE, 16, 3, 65536, true>(a, stream);
     }
 }
