@@ -181,7 +181,9 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
     alg_bytes = masked_rows * w.V * w.elem_bytes
     mode = {"profile": fd.PROFILE, "factor": fd.FACTOR, "threshold": fd.THRESHOLD}[args.mode]
 
-    mask = mask0.clone()
+    # one mask buffer per logits buffer, all restored by a single copy per replay
+    masks = mask0.unsqueeze(0).repeat(n_buf, 1, 1).contiguous()
+    masks0 = masks.clone()
     tok = torch.full((w.B, w.L), -1, dtype=torch.int32, device=dev)
     commit = torch.empty((w.B, w.L), dtype=torch.uint8, device=dev)
     n_out = torch.empty((w.B,), dtype=torch.int32, device=dev)
@@ -190,9 +192,10 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
     stream = torch.cuda.Stream(device=dev)
 
     def step(i):
-        mask.copy_(mask0, non_blocking=True)  # steady state: same masked rows every step
-        fd.fdllm_select(bufs[i % n_buf], mask, args.param, mode, tok, commit, n_out,
-                        stream=stream)
+        if i % n_buf == 0:  # steady state: the same masked rows every step
+            masks.copy_(masks0, non_blocking=True)
+        fd.fdllm_select(bufs[i % n_buf], masks[i % n_buf], args.param, mode, tok, commit,
+                        n_out, stream=stream)
 
     def k1_only(i):
         fd.fdllm_confidence(bufs[i % n_buf], mask0, conf, amax, stream=stream)

@@ -41,7 +41,8 @@ struct VocabReduceArgs {
     int32_t units_per_row;
     int32_t unit_vecs;
     UnitPartial *partials;   // [rows][units_per_row]; written for masked rows
-    uint32_t *next_unit;     // work counter: zero on entry, reset by the consumer kernel
+    uint32_t *next_unit;     // work queue past the first gridDim.x units: zero on entry,
+                             // reset by the consumer kernel
     uint32_t *status;        // sticky device error bits
 };
 
@@ -69,7 +70,8 @@ inline UnitPlan plan_units(int64_t row_bytes)
     return UnitPlan{(int32_t)upr, (int32_t)uv};
 }
 
-// Enqueue the vocab reduction on all SMs.
+// Enqueue the vocab reduction on all SMs, as a programmatic dependent of the previous
+// kernel on the stream.
 cudaError_t launch_vocab_reduce(const VocabReduceArgs &a, int esize, cudaStream_t stream);
 
 // Per masked position: combine its unit partials, write (c, x_hat); resets next_unit.

@@ -122,6 +122,8 @@ __global__ void __launch_bounds__(T) profile_select_kernel(const ProfileSelectAr
     // partials, or read from the given arrays.
     if (a.partials != nullptr)
         pdl_wait();  // the vocab reduction's partials are complete and visible
+    if (threadIdx.x == 0)
+        pdl_launch_dependents();  // a following vocab reduction may start its prologue
     const bool masked = t < L && a.mask[base + t] != 0;
     float c = 0.0f;
     int32_t tok = -1;

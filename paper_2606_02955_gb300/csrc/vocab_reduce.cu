@@ -250,14 +250,6 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
 
-    // The consumer kernel may start launching now; it waits for this grid's results.
-    if (threadIdx.x == 0)
-        pdl_launch_dependents();
-    // The producer's first unit request overlaps the mask compaction below.
-    uint32_t first_unit = 0;
-    if (threadIdx.x == 0)
-        first_unit = atomicAdd(a.next_unit, 1u);
-
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             mbar_init(&sm.full[s], 1);
@@ -269,6 +261,12 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
         }
         fence_mbar_init();
     }
+    // Launched as a programmatic dependent of the previous kernel: its writes (mask, logits,
+    // this workspace's counter) are visible after this wait.  The consumer kernel of this
+    // grid may start launching now; it waits for this grid's results itself.
+    pdl_wait();
+    if (threadIdx.x == 0)
+        pdl_launch_dependents();
 
     // Mask -> bitmap (one ballot per 32 rows, four words in flight per warp) -> exclusive
     // prefix count per word.
@@ -317,7 +315,7 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
     const uint32_t upr = (uint32_t)a.units_per_row;
     const uint32_t total = sm.pref[nwords] * upr;  // host checks rows * upr < 2^31
     if (total == 0)
-        return;  // (first_unit >= total then, so nothing was claimed)
+        return;
 
     if (warp == 0) {
         // ------------------------------------------------------------ producer (one lane)
@@ -326,10 +324,13 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
         uint64_t policy = 0;
         if (EVICT)
             policy = make_evict_first_policy();
+        // Unit blockIdx.x first (no atomic before the first copy), then the work queue,
+        // which hands out units gridDim.x, gridDim.x + 1, ...
         uint32_t k = 0;
-        uint32_t u = first_unit;
+        uint32_t u = blockIdx.x;
         while (u < total) {
-            const uint32_t u_next = atomicAdd(a.next_unit, 1u);  // in flight while u streams
+            // the next unit's request is in flight while u streams
+            const uint32_t u_next = gridDim.x + atomicAdd(a.next_unit, 1u);
             const uint32_t r = u / upr, j = u - r * upr;
             const int64_t grow = masked_row(r, sm.bits, sm.pref, nwords);
             const int64_t v0 = (int64_t)j * a.unit_vecs;
@@ -526,6 +527,8 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
 __global__ void finalize_kernel(const FinalizeArgs a)
 {
     pdl_wait();  // the vocab reduction's partials are complete and visible
+    if (threadIdx.x == 0)
+        pdl_launch_dependents();  // a following vocab reduction may start its prologue
     if (blockIdx.x == 0 && threadIdx.x == 0)
         *a.next_unit = 0;
     const int64_t row = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -563,8 +566,17 @@ cudaError_t launch_variant(const VocabReduceArgs &a, cudaStream_t stream)
         grid_cache[dev] = g < kMaxGrid ? g : kMaxGrid;
         attr_done[dev] = 1;
     }
-    kern<<<grid_cache[dev], (NW + 2) * 32, smem, stream>>>(a);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid_cache[dev]);
+    cfg.blockDim = dim3((NW + 2) * 32);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, a);
 }
 
 // Tuning table (math warps, ring stages x chunk bytes, L2 hint).  Entry 0 is the
