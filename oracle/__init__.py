@@ -84,6 +84,8 @@ class Oracle:
         lib.oracle_frechet_scan.restype = None
         lib.oracle_select_from_conf.argtypes = [p, p, i64, i64, p, i32, d, p, p, p, p]
         lib.oracle_select_from_conf.restype = i64
+        lib.oracle_select_robust_from_conf.argtypes = [p, p, i64, i64, p, d, d, p, p, p, p, p]
+        lib.oracle_select_robust_from_conf.restype = i64
         self.lib = lib
         self.path = lib_path
 
@@ -128,6 +130,37 @@ class Oracle:
                                                _ptr(margin))
         return dict(tokens=toks, commit=commit, n=n, margin=margin, mask=m,
                     invalid_rows=int(bad))
+
+    def select_robust_from_conf(self, conf: np.ndarray, tok: np.ndarray, mask: np.ndarray,
+                                param: float, eta: float, eta_pos: np.ndarray | None = None,
+                                out_tokens: np.ndarray | None = None):
+        """Calibration-robust profile selection (App. C) on given confidences; eta_pos
+        (per position, [B, L]) replaces the uniform eta when given.  Same result dict as
+        select_from_conf."""
+        c = np.ascontiguousarray(conf, dtype=np.float64)
+        B, L = c.shape
+        t = np.ascontiguousarray(tok, dtype=np.int32).reshape(B, L)
+        m = np.array(mask, dtype=np.uint8, copy=True).reshape(B, L)
+        e = None if eta_pos is None else np.ascontiguousarray(eta_pos, np.float64).reshape(B, L)
+        toks = (np.full((B, L), -1, np.int32) if out_tokens is None
+                else np.array(out_tokens, dtype=np.int32, copy=True).reshape(B, L))
+        commit = np.zeros((B, L), np.uint8)
+        n = np.zeros(B, np.int32)
+        margin = np.zeros(B, np.float64)
+        bad = self.lib.oracle_select_robust_from_conf(
+            _ptr(c), _ptr(t), B, L, _ptr(m), float(param), float(eta),
+            None if e is None else _ptr(e), _ptr(toks), _ptr(commit), _ptr(n), _ptr(margin))
+        return dict(tokens=toks, commit=commit, n=n, margin=margin, mask=m,
+                    invalid_rows=int(bad))
+
+    def select_robust(self, logits: np.ndarray, mask: np.ndarray, param: float, eta: float,
+                      eta_pos: np.ndarray | None = None, nthreads: int = 1):
+        """Whole calibration-robust step on host logits."""
+        conf, tok, _ = self.confidence(logits, mask, nthreads)
+        res = self.select_robust_from_conf(conf, tok, mask, param, eta, eta_pos)
+        res["conf"] = conf
+        res["tok"] = tok
+        return res
 
     def select(self, logits: np.ndarray, mask: np.ndarray, mode: int, param: float,
                out_tokens: np.ndarray | None = None, nthreads: int = 1):

@@ -223,6 +223,92 @@ int64_t oracle_select_from_conf(const double *conf, const int32_t *tok, int64_t 
     return bad;
 }
 
+int64_t oracle_select_robust_from_conf(const double *conf, const int32_t *tok, int64_t B,
+                                       int64_t L, uint8_t *mask, double param, double eta,
+                                       const double *eta_pos, int32_t *out_tokens,
+                                       uint8_t *out_commit, int32_t *out_n, double *margin)
+{
+    int64_t bad = 0;
+    candidate *cand = (candidate *)malloc((size_t)L * sizeof(candidate));
+    double *cs = (double *)malloc((size_t)L * sizeof(double));
+    double *Ln = (double *)malloc((size_t)L * sizeof(double));
+    double *Un = (double *)malloc((size_t)L * sizeof(double));
+    double *Gn = (double *)malloc((size_t)L * sizeof(double));
+    const double delta = 1.0 - param; /* matched margin, Cor. factor-reduction */
+
+    for (int64_t b = 0; b < B; ++b) {
+        const int64_t row0 = b * L;
+        int64_t m = 0;
+        int invalid = 0;
+        double clip_gap = INFINITY; /* closest distance of a c_hat to its clipping point */
+        for (int64_t l = 0; l < L; ++l) {
+            out_commit[row0 + l] = 0;
+            if (!mask[row0 + l])
+                continue;
+            const double c_hat = conf[row0 + l];
+            if (!(c_hat > 0.0 && c_hat <= 1.0))
+                invalid = 1;
+            const double eta_i = eta_pos ? eta_pos[row0 + l] : eta;
+            /* App. C: the lower confidence max{0, c_hat - eta} */
+            const double c_low = c_hat - eta_i > 0.0 ? c_hat - eta_i : 0.0;
+            if (fabs(c_hat - eta_i) < clip_gap)
+                clip_gap = fabs(c_hat - eta_i);
+            cand[m].c = c_low;
+            cand[m].pos = (int32_t)l;
+            ++m;
+        }
+        if (margin)
+            margin[b] = INFINITY;
+        if (invalid) {
+            out_n[b] = -1;
+            ++bad;
+            continue;
+        }
+        if (m == 0) {
+            out_n[b] = 0;
+            continue;
+        }
+        qsort(cand, (size_t)m, sizeof(candidate), by_confidence_desc);
+        for (int64_t j = 0; j < m; ++j)
+            cs[j] = cand[j].c;
+        /* Eq. robust_L_U on the top-n prefix: the same scan as Sec. 3 on c_low */
+        oracle_frechet_scan(cs, m, Ln, Un, Gn);
+        int64_t nstar = 0;
+        for (int64_t n = 1; n <= m; ++n)
+            if (Gn[n - 1] > delta)
+                nstar = n;
+        if (nstar == 0)
+            nstar = 1;
+        for (int64_t j = 0; j < nstar; ++j) {
+            const int64_t at = row0 + cand[j].pos;
+            out_tokens[at] = tok[at];
+            out_commit[at] = 1;
+            mask[at] = 0;
+        }
+        out_n[b] = (int32_t)nstar;
+        if (margin) {
+            double mg = fabs(Gn[nstar - 1] - delta);
+            if (nstar < m) {
+                double next = fabs(Gn[nstar] - delta);
+                if (next < mg)
+                    mg = next;
+                double gap = cs[nstar - 1] - cs[nstar];
+                if (gap > 0.0 && gap < mg)
+                    mg = gap;
+            }
+            if (clip_gap < mg)
+                mg = clip_gap;
+            margin[b] = mg;
+        }
+    }
+    free(cand);
+    free(cs);
+    free(Ln);
+    free(Un);
+    free(Gn);
+    return bad;
+}
+
 int64_t oracle_select(const void *logits, int dtype, int64_t B, int64_t L, int64_t V,
                       uint8_t *mask, int mode, double param, int32_t *out_tokens,
                       uint8_t *out_commit, int32_t *out_n, double *margin, double *conf,

@@ -58,6 +58,18 @@ int64_t oracle_select_from_conf(const double *conf, const int32_t *tok, int64_t 
                                 uint8_t *mask, int mode, double param, int32_t *out_tokens,
                                 uint8_t *out_commit, int32_t *out_n, double *margin);
 
+/* Calibration-robust profile selection (App. C, Eq. robust_L_U) on given confidences:
+ * lower confidences c_low_i = max{0, c_hat_i - eta_i} with eta_i = eta_pos[i] when eta_pos
+ * is given, else the uniform eta; then the profile rule of Sec. 3 on c_low: rank the masked
+ * positions by c_low descending (ties: lower position first), L = max{0, sum c_low - (n-1)},
+ * U = 1 - c_low_(n), accept n iff L - U > delta = 1 - param, n* = max accepted or 1.
+ * Validity, empty rows, outputs and return value as oracle_select_from_conf.  margin[b] also
+ * covers min_i |c_hat_i - eta_i| over the row's masked positions (clipping can reorder). */
+int64_t oracle_select_robust_from_conf(const double *conf, const int32_t *tok, int64_t B,
+                                       int64_t L, uint8_t *mask, double param, double eta,
+                                       const double *eta_pos, int32_t *out_tokens,
+                                       uint8_t *out_commit, int32_t *out_n, double *margin);
+
 /* oracle_confidence followed by oracle_select_from_conf.  conf/tok are caller scratch of
  * B*L entries; they come back holding the per-position confidences and argmax tokens. */
 int64_t oracle_select(const void *logits, int dtype, int64_t B, int64_t L, int64_t V,

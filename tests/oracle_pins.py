@@ -380,9 +380,104 @@ def pin_end_to_end(o):
             assert r["n"][b] == (max(ks) if ks else 1)
 
 
+def _robust_profiles(rng, count, m_max, dyadic, eta_lo=0.0):
+    out = []
+    for _ in range(count):
+        m = int(rng.integers(1, m_max + 1))
+        lo = int(np.ceil(eta_lo * dyadic))
+        out.append(list(map(float, rng.integers(max(lo, 1), dyadic + 1, m) / dyadic)))
+    return out
+
+
+def _run_robust(o, profiles, param, eta, eta_pos=None):
+    B = len(profiles)
+    L = max(len(p) for p in profiles)
+    conf = np.zeros((B, L))
+    mask = np.zeros((B, L), np.uint8)
+    tok = np.arange(B * L, dtype=np.int32).reshape(B, L)
+    for b, p in enumerate(profiles):
+        conf[b, :len(p)] = p
+        mask[b, :len(p)] = 1
+    r = o.select_robust_from_conf(conf, tok, mask, param, eta, eta_pos)
+    return r["n"], [set(np.nonzero(r["commit"][b])[0].tolist()) for b in range(B)], r
+
+
+def pin_robust_zero_eta_is_profile(o):
+    """App. C with eta = 0 is the plain profile rule (c_low = c_hat)."""
+    rng = np.random.default_rng(29)
+    profiles = _random_profiles(rng, 200, 24)
+    for f in (1.0, 0.75, 0.5):
+        n_r, s_r, _ = _run_robust(o, profiles, f, 0.0)
+        n_p, s_p, _ = run_profiles(o, profiles, PROFILE, f)
+        assert np.array_equal(n_r, n_p) and s_r == s_p
+
+
+def pin_robust_calibration_penalty(o):
+    """Cor. calibration-penalty: with uniform eta and no clipping (every c_hat >= eta),
+    G^(eta)_n = G_hat_n - (n+1) eta where the robust lower bound is active, and both sides
+    reject otherwise (delta >= 0), so n*_robust = max{n : G_hat_n - (n+1) eta > delta}.
+    Dyadic values keep every comparison exact."""
+    rng = np.random.default_rng(31)
+    for eta in (1 / 64, 1 / 16, 3 / 32):
+        profiles = _robust_profiles(rng, 150, 12, 256, eta_lo=eta)
+        for f in (1.0, 0.75, 0.5):
+            delta = 1.0 - f
+            n_r, _, _ = _run_robust(o, profiles, f, eta)
+            for b, p in enumerate(profiles):
+                c = np.array(sorted(p, reverse=True))
+                _, _, G = o.frechet_scan(c)
+                acc = [n for n in range(1, len(c) + 1) if G[n - 1] - (n + 1) * eta > delta]
+                assert n_r[b] == (max(acc) if acc else 1), (p, eta, f)
+
+
+def _G_low(cs):
+    k = len(cs)
+    return max(0.0, sum(cs) - (k - 1)) - (1.0 - min(cs))
+
+
+def pin_robust_bruteforce(o):
+    """Eq. robust_L_U over all subsets with per-position allowances: n* is the largest size
+    with an admissible subset, and the committed set attains the best robust score."""
+    rng = np.random.default_rng(37)
+    B, m = 120, 7
+    profiles = [list(map(float, rng.integers(1, 65, m) / 64)) for _ in range(B)]
+    eta_pos = rng.integers(0, 9, (B, m)) / 64
+    for f in (1.0, 0.75):
+        delta = 1.0 - f
+        n_r, sets, _ = _run_robust(o, profiles, f, 0.0, eta_pos)
+        for b, p in enumerate(profiles):
+            low = [max(0.0, p[i] - eta_pos[b, i]) for i in range(m)]
+            best = {k: max(_G_low([low[i] for i in S])
+                           for S in itertools.combinations(range(m), k))
+                    for k in range(1, m + 1)}
+            ks = [k for k in range(1, m + 1) if best[k] > delta]
+            want = max(ks) if ks else 1
+            assert n_r[b] == want, (p, eta_pos[b], f)
+            if ks:
+                assert _G_low([low[i] for i in sorted(sets[b])]) == best[want]
+
+
+def pin_robust_monotone_and_clipped(o):
+    """A larger allowance never commits more (uniform eta); when every confidence is at or
+    below eta all lower confidences are 0 and the progress convention commits the lowest
+    position."""
+    rng = np.random.default_rng(41)
+    profiles = _random_profiles(rng, 200, 20)
+    prev = None
+    for eta in (0.0, 0.01, 0.05, 0.1, 0.3):
+        n_r, _, _ = _run_robust(o, profiles, 1.0, eta)
+        if prev is not None:
+            assert np.all(n_r <= prev)
+        prev = n_r
+    low = [[0.2, 0.1, 0.3], [0.05]]
+    n_r, sets, _ = _run_robust(o, low, 0.75, 0.3)
+    assert list(n_r) == [1, 1] and sets == [{0}, {0}]
+
+
 ALL_PINS = [
     pin_confidence_vs_torch, pin_confidence_closed_forms, pin_nonfinite, pin_hand_worked,
     pin_bruteforce_subsets, pin_equal_confidence_reduction, pin_heterogeneity_bonus,
     pin_matched_dominance, pin_greedy_equivalence, pin_monotone_prefix, pin_special_cases,
-    pin_reveal_and_ties, pin_end_to_end,
+    pin_reveal_and_ties, pin_end_to_end, pin_robust_zero_eta_is_profile,
+    pin_robust_calibration_penalty, pin_robust_bruteforce, pin_robust_monotone_and_clipped,
 ]

@@ -40,18 +40,35 @@ MUTANTS = {
     "bf16_widened_wrong": ("(uint32_t)((const uint16_t *)logits)[i] << 16",
                            "(uint32_t)((const uint16_t *)logits)[i] << 15"),
     "nan_not_flagged": ("if (saw_nan || !isfinite(M))", "if (!isfinite(M))"),
+    "robust_no_clipping": ("const double c_low = c_hat - eta_i > 0.0 ? c_hat - eta_i : 0.0;",
+                           "const double c_low = c_hat - eta_i;"),
+    "robust_eta_added": ("const double c_low = c_hat - eta_i > 0.0 ? c_hat - eta_i : 0.0;",
+                         "const double c_low = c_hat + eta_i;"),
+    "robust_ranks_by_c_hat": ("cand[m].c = c_low;", "cand[m].c = c_hat;"),
+    "robust_eta_ignored": ("const double eta_i = eta_pos ? eta_pos[row0 + l] : eta;",
+                           "const double eta_i = 0.0;"),
+    # (old, new, occurrence): the robust selector repeats some lines of the plain one
+    "robust_no_progress_fallback": ("if (nstar == 0)\n            nstar = 1;", "", 1),
+    "robust_margin_not_strict": ("if (Gn[n - 1] > delta)", "if (Gn[n - 1] >= delta)"),
+    "robust_delta_not_matched": ("const double delta = 1.0 - param;", "const double delta = param;",
+                                 1),
 }
 
 
 @pytest.mark.parametrize("name", sorted(MUTANTS))
 def test_planted_mistake_is_caught(name, tmp_path):
-    old, new = MUTANTS[name]
+    old, new, *occ = MUTANTS[name]
+    which = occ[0] if occ else 0
     with open(oracle.SOURCE) as fh:
         src = fh.read()
-    assert src.count(old) == 1, "mutation anchor not found once: %r" % old
+    assert src.count(old) > which, "mutation anchor not found: %r" % old
+    at = -1
+    for _ in range(which + 1):
+        at = src.index(old, at + 1)
+    src = src[:at] + new + src[at + len(old):]
     shutil.copy(oracle.HEADER, tmp_path / os.path.basename(oracle.HEADER))
     mutated = tmp_path / "mutant.c"
-    mutated.write_text(src.replace(old, new))
+    mutated.write_text(src)
     lib = oracle.compile_oracle(str(mutated), str(tmp_path / "libmutant.so"))
     mut = oracle.Oracle(lib)
     failed = []
