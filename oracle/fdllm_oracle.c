@@ -104,6 +104,33 @@ typedef struct {
     int32_t pos;
 } candidate;
 
+/* Decision margin contribution of the ranking (for parity checks): the smallest positive
+ * confidence gap whose sign decides which positions fill the first n* ranks.  Without a tie
+ * at the boundary that is c_(n*) - c_(n*+1).  When a block of equal confidences straddles
+ * the boundary (ranks a..b with a <= n* < b), the block is committed partly, in position
+ * order, so the gaps to its neighbours above and below decide instead. */
+static double ranking_gap(const double *cs, int64_t m, int64_t nstar)
+{
+    double mg = INFINITY;
+    if (nstar >= m)
+        return mg;
+    const double v = cs[nstar - 1];
+    if (cs[nstar] != v) {
+        const double gap = v - cs[nstar];
+        return gap > 0.0 ? gap : mg;
+    }
+    int64_t a = nstar, b = nstar; /* 1-based ranks of the tie block */
+    while (a > 1 && cs[a - 2] == v)
+        --a;
+    while (b < m && cs[b] == v)
+        ++b;
+    if (a > 1 && cs[a - 2] - v < mg)
+        mg = cs[a - 2] - v;
+    if (b < m && v - cs[b] < mg)
+        mg = v - cs[b];
+    return mg;
+}
+
 /* Alg. 1 sort: c_(1) >= c_(2) >= ...; equal confidences keep the lower position first. */
 static int by_confidence_desc(const void *pa, const void *pb)
 {
@@ -201,14 +228,11 @@ int64_t oracle_select_from_conf(const double *conf, const int32_t *tok, int64_t 
 
         if (margin) {
             double mg = fabs(q[nstar - 1]);
-            if (nstar < m) {
-                double next = fabs(q[nstar]);
-                if (next < mg)
-                    mg = next;
-                double gap = cs[nstar - 1] - cs[nstar];
-                if (gap > 0.0 && gap < mg)
-                    mg = gap;
-            }
+            if (nstar < m && fabs(q[nstar]) < mg)
+                mg = fabs(q[nstar]);
+            const double gap = ranking_gap(cs, m, nstar);
+            if (gap < mg)
+                mg = gap;
             margin[b] = mg;
         }
     }
@@ -288,14 +312,11 @@ int64_t oracle_select_robust_from_conf(const double *conf, const int32_t *tok, i
         out_n[b] = (int32_t)nstar;
         if (margin) {
             double mg = fabs(Gn[nstar - 1] - delta);
-            if (nstar < m) {
-                double next = fabs(Gn[nstar] - delta);
-                if (next < mg)
-                    mg = next;
-                double gap = cs[nstar - 1] - cs[nstar];
-                if (gap > 0.0 && gap < mg)
-                    mg = gap;
-            }
+            if (nstar < m && fabs(Gn[nstar] - delta) < mg)
+                mg = fabs(Gn[nstar] - delta);
+            const double gap = ranking_gap(cs, m, nstar);
+            if (gap < mg)
+                mg = gap;
             if (clip_gap < mg)
                 mg = clip_gap;
             margin[b] = mg;

@@ -51,8 +51,9 @@ void oracle_frechet_scan(const double *c_sorted, int64_t m, double *Ln, double *
  *                        first) get out_tokens = tok, out_commit = 1, mask = 0.
  * out_commit is fully written; out_tokens only at committed positions.
  * margin[b] (nullable) = decision margin of the row: the smallest of |rule(n) - bound| at
- * n = n* and n = n*+1 and of the confidence gap c_(n*) - c_(n*+1) when it is non-zero;
- * +inf when nothing can flip (m == 0, invalid row, or no such term).
+ * n = n* and n = n*+1 and of the ranking gap that decides which positions fill the first n*
+ * ranks (c_(n*) - c_(n*+1); when equal confidences straddle the boundary, the gaps from
+ * that tie block to its neighbours); +inf when nothing can flip (m == 0, invalid row).
  * Returns the number of invalid rows. */
 int64_t oracle_select_from_conf(const double *conf, const int32_t *tok, int64_t B, int64_t L,
                                 uint8_t *mask, int mode, double param, int32_t *out_tokens,
