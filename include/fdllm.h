@@ -109,6 +109,24 @@ fdllm_status fdllm_select_ws(const void *logits, int dtype, int B, int L, int V,
                              int32_t *out_n, void *workspace, size_t workspace_bytes,
                              void *stream);
 
+/* The profile rule on calibration-robust confidences (App. C, "Calibration-Robust Frechet
+ * Certificates"): every masked confidence c_hat is replaced by the lower confidence
+ * c_low = max{0, c_hat - eta_i} (Eq. robust_L_U), the masked positions are ranked by c_low
+ * (ties: lower position first), L_eta(n) = max{0, sum_{j<=n} c_low_(j) - (n-1)},
+ * U_eta(n) = 1 - c_low_(n), n is accepted iff L_eta(n) - U_eta(n) > delta = 1 - param, and
+ * n* = max accepted, or 1 (the paper defines the robust certificate; this selection rule on
+ * it is the library's reading).  With uniform eta and no clipping the score is the plain
+ * one minus (n+1) eta (Cor. calibration-penalty).
+ *   eta               uniform allowance (finite; the paper takes eta >= 0), used when
+ *                     eta_per_position is NULL.
+ *   eta_per_position  [B, L] fp32 device array of per-position allowances, or NULL.
+ * Everything else as fdllm_select (the same library workspace).  eta = 0 gives exactly
+ * fdllm_select's profile rule. */
+fdllm_status fdllm_select_robust(const void *logits, int dtype, int B, int L, int V,
+                                 uint8_t *mask, double param, double eta,
+                                 const float *eta_per_position, int32_t *out_tokens,
+                                 uint8_t *out_commit, int32_t *out_n, void *stream);
+
 /* Scratch of fdllm_select_static: a fixed device array of this many bytes. */
 #define FDLLM_STATIC_SCRATCH_BYTES (8u << 20)
 

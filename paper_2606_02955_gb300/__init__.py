@@ -20,7 +20,7 @@ __all__ = [
     "FdllmError", "fdllm_select", "fdllm_select_ws", "fdllm_workspace_bytes",
     "fdllm_confidence", "fdllm_select_from_conf", "fdllm_device_status",
     "fdllm_workspace_status", "fdllm_release_workspace", "fdllm_status_string",
-    "fdllm_version", "library_path", "fdllm_select_static",
+    "fdllm_version", "library_path", "fdllm_select_static", "fdllm_select_robust",
 ]
 
 BF16, FP32 = 0, 1
@@ -46,6 +46,8 @@ def _load():
     lib.fdllm_select.restype = i
     lib.fdllm_select_ws.argtypes = [p, i, i, i, i, p, d, i, p, p, p, p, sz, p]
     lib.fdllm_select_ws.restype = i
+    lib.fdllm_select_robust.argtypes = [p, i, i, i, i, p, d, d, p, p, p, p, p]
+    lib.fdllm_select_robust.restype = i
     lib.fdllm_select_static.argtypes = [p, i, i, i, i, p, d, i, p, p, p, p]
     lib.fdllm_select_static.restype = i
     lib.fdllm_workspace_bytes.argtypes = [i, i, i, i]
@@ -173,6 +175,26 @@ def _select_from_host(logits, mask, param, mode, out_tokens, out_commit, out_n):
     mask.copy_(d_mask, non_blocking=True)
     torch.cuda.current_stream().synchronize()
     return h_tok, h_commit, h_n
+
+
+def fdllm_select_robust(logits: torch.Tensor, mask: torch.Tensor, param: float, eta: float = 0.0,
+                        eta_per_position=None, out_tokens=None, out_commit=None, out_n=None,
+                        stream=None):
+    """Calibration-robust profile selection (App. C): confidences lowered to
+    max(0, c - eta) (``eta_per_position``: [B, L] fp32 CUDA tensor, else the uniform eta)
+    before the profile rule.  Returns (out_tokens, out_commit, out_n)."""
+    B, L, V = logits.shape
+    out_tokens, out_commit, out_n = _outputs(B, L, logits.device, out_tokens, out_commit, out_n)
+    ep = None if eta_per_position is None else _dev(eta_per_position, "eta_per_position",
+                                                     torch.float32, (B, L))
+    st = _load().fdllm_select_robust(_dev(logits, "logits"), _dtype_code(logits), B, L, V,
+                                     _dev(mask, "mask", torch.uint8, (B, L)), float(param),
+                                     float(eta), ep,
+                                     _dev(out_tokens, "out_tokens", torch.int32, (B, L)),
+                                     _dev(out_commit, "out_commit", torch.uint8, (B, L)),
+                                     _dev(out_n, "out_n", torch.int32, (B,)), _stream(stream))
+    _check(st, "fdllm_select_robust")
+    return out_tokens, out_commit, out_n
 
 
 def fdllm_select_static(logits: torch.Tensor, mask: torch.Tensor, param: float, mode=PROFILE,

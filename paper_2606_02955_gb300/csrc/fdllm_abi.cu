@@ -124,7 +124,8 @@ VocabReduceArgs reduce_args(const void *logits, int dtype, int B, int L, int V,
 
 fdllm_status run_select(const void *logits, int dtype, int B, int L, int V, uint8_t *mask,
                         double param, int mode, int32_t *out_tokens, uint8_t *out_commit,
-                        int32_t *out_n, uint8_t *ws, const Layout &lay, cudaStream_t stream)
+                        int32_t *out_n, uint8_t *ws, const Layout &lay, cudaStream_t stream,
+                        double eta = 0.0, const float *eta_pos = nullptr)
 {
     VocabReduceArgs ra = reduce_args(logits, dtype, B, L, V, mask, ws, lay);
     if (launch_vocab_reduce(ra, esize_of(dtype), stream) != cudaSuccess)
@@ -140,6 +141,8 @@ fdllm_status run_select(const void *logits, int dtype, int B, int L, int V, uint
     pa.L = L;
     pa.mode = mode;
     pa.param = param;
+    pa.eta = eta;
+    pa.eta_pos = eta_pos;
     pa.out_tokens = out_tokens;
     pa.out_commit = out_commit;
     pa.out_n = out_n;
@@ -257,6 +260,27 @@ fdllm_status fdllm_select(const void *logits, int dtype, int B, int L, int V, ui
                       static_cast<uint8_t *>(ws), lay, s);
 }
 
+fdllm_status fdllm_select_robust(const void *logits, int dtype, int B, int L, int V,
+                                 uint8_t *mask, double param, double eta,
+                                 const float *eta_per_position, int32_t *out_tokens,
+                                 uint8_t *out_commit, int32_t *out_n, void *stream)
+{
+    fdllm_status st = check_select_args(logits, dtype, B, L, V, mask, param, FDLLM_PROFILE,
+                                        out_tokens, out_commit, out_n);
+    if (st != FDLLM_OK)
+        return st;
+    if (!std::isfinite(eta))
+        return FDLLM_ERR_ARG;
+    const Layout lay = layout_for((int64_t)B * L, (int64_t)V * esize_of(dtype));
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    void *ws = nullptr;
+    st = owned_workspace(lay.total, s, &ws);
+    if (st != FDLLM_OK)
+        return st;
+    return run_select(logits, dtype, B, L, V, mask, param, kModeRobust, out_tokens, out_commit,
+                      out_n, static_cast<uint8_t *>(ws), lay, s, eta, eta_per_position);
+}
+
 fdllm_status fdllm_select_static(const void *logits, int dtype, int B, int L, int V,
                                  uint8_t *mask, double param, int mode, int32_t *out_tokens,
                                  uint8_t *out_commit, int32_t *out_n, void *stream)
@@ -339,6 +363,8 @@ fdllm_status fdllm_select_from_conf(const float *conf, const int32_t *argmax, in
     pa.L = L;
     pa.mode = mode;
     pa.param = param;
+    pa.eta = 0.0;
+    pa.eta_pos = nullptr;
     pa.out_tokens = out_tokens;
     pa.out_commit = out_commit;
     pa.out_n = out_n;

@@ -89,6 +89,9 @@ struct FinalizeArgs {
 cudaError_t launch_finalize(const FinalizeArgs &a, cudaStream_t stream);
 
 // ------------------------------------------------------------------ profile select (a2-a5)
+// The profile rule on calibration-robust lower confidences max{0, c - eta} (App. C).
+constexpr int kModeRobust = 3;
+
 struct ProfileSelectArgs {
     // Source of (c, x_hat): unit partials (from the vocab reduction, which this kernel then
     // follows as a programmatic dependent launch) when `partials` is non-null, otherwise the
@@ -101,8 +104,10 @@ struct ProfileSelectArgs {
     uint8_t *mask;           // [B, L], updated in place
     int B;
     int L;
-    int mode;
+    int mode;                // 0 profile, 1 factor, 2 threshold, kModeRobust
     double param;
+    double eta;              // kModeRobust: uniform calibration allowance
+    const float *eta_pos;    // kModeRobust: [B, L] per-position allowances, or null
     int32_t *out_tokens;     // [B, L]
     uint8_t *out_commit;     // [B, L]
     int32_t *out_n;          // [B]

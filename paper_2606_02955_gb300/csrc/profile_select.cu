@@ -18,17 +18,20 @@ namespace {
 
 constexpr uint64_t kPadKey = ~0ull;  // sorts after every real key
 
-// Masked: (~bits(c)) << 32 | pos — for c in (0, 1] larger c gives a smaller key, and equal
-// c falls back to the position.  Unmasked: 0xFFFFFFFF << 32 | pos, after every masked key.
+// Masked: (bits(1) - bits(c)) << 32 | pos — for c in [0, 1] larger c gives a smaller key
+// (0 for c = 1, bits(1) for c = 0), and equal c falls back to the position.  Unmasked:
+// 0xFFFFFFFF << 32 | pos, after every masked key.
+constexpr uint32_t kOneBits = 0x3F800000u;
+
 __device__ __forceinline__ uint64_t make_key(bool masked, float c, int pos)
 {
-    const uint32_t hi = masked ? ~__float_as_uint(c) : 0xFFFFFFFFu;
+    const uint32_t hi = masked ? kOneBits - __float_as_uint(c) : 0xFFFFFFFFu;
     return ((uint64_t)hi << 32) | (uint32_t)pos;
 }
 
 __device__ __forceinline__ float key_conf(uint64_t key)
 {
-    return __uint_as_float(~(uint32_t)(key >> 32));
+    return __uint_as_float(kOneBits - (uint32_t)(key >> 32));
 }
 
 template <int T>
@@ -140,7 +143,13 @@ __global__ void __launch_bounds__(T) profile_select_kernel(const ProfileSelectAr
     if (a.partials != nullptr && a.next_unit != nullptr && blockIdx.x == 0 && t == 0)
         *a.next_unit = 0;  // the vocab reduction before this kernel has finished
     const bool bad = masked && !(c > 0.0f && c <= 1.0f);  // NaN fails both
-    uint64_t key = t < L ? make_key(masked, c, t) : kPadKey;
+    // The robust rule ranks and scans lower confidences max{0, c - eta} (App. C).
+    float c_rank = c;
+    if (a.mode == kModeRobust && masked && !bad) {
+        const float eta = a.eta_pos != nullptr ? a.eta_pos[base + t] : (float)a.eta;
+        c_rank = fmaxf(0.0f, c - eta);
+    }
+    uint64_t key = t < L ? make_key(masked, c_rank, t) : kPadKey;
 
     const int m = __syncthreads_count(masked);
     const int any_bad = __syncthreads_or(bad);
@@ -157,7 +166,7 @@ __global__ void __launch_bounds__(T) profile_select_kernel(const ProfileSelectAr
 
     bool ok = false;
     if (live) {
-        if (a.mode == 0) {  // profile: G_n > delta, delta = 1 - f
+        if (a.mode == 0 || a.mode == kModeRobust) {  // profile: G_n > delta, delta = 1 - f
             const double delta = 1.0 - a.param;
             const double Ln = fmax(0.0, 1.0 - P);
             const double Un = 1.0 - cn;

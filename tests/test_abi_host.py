@@ -107,3 +107,14 @@ def test_confidence_and_select_from_conf_reject(lib):
                                       None) == ERR_ARG
     assert lib.fdllm_select_from_conf(None, A16, 2, 32, A16, 1.0, 0, A16, A16, A16,
                                       None) == ERR_ARG
+
+
+def test_select_robust_rejects(lib):
+    p, i, d = ctypes.c_void_p, ctypes.c_int, ctypes.c_double
+    lib.fdllm_select_robust.argtypes = [p, i, i, i, i, p, d, d, p, p, p, p, p]
+    f = lambda eta, B=2, logits=A16: lib.fdllm_select_robust(logits, 0, B, 32, 1024, A16, 1.0,
+                                                             eta, None, A16, A16, A16, None)
+    assert f(float("nan")) == ERR_ARG
+    assert f(float("inf")) == ERR_ARG
+    assert f(0.1, B=0) == ERR_ARG
+    assert f(0.1, logits=A2) == ERR_ALIGN
