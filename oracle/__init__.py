@@ -86,6 +86,10 @@ class Oracle:
         lib.oracle_select_from_conf.restype = i64
         lib.oracle_select_robust_from_conf.argtypes = [p, p, i64, i64, p, d, d, p, p, p, p, p]
         lib.oracle_select_robust_from_conf.restype = i64
+        lib.oracle_bonus_terms.argtypes = [p, i64, p, p]
+        lib.oracle_bonus_terms.restype = None
+        lib.oracle_profile_terms.argtypes = [p, p, i64, i64, p, p, p, p]
+        lib.oracle_profile_terms.restype = None
         self.lib = lib
         self.path = lib_path
 
@@ -109,6 +113,25 @@ class Oracle:
         Ln, Un, Gn = (np.zeros(m, np.float64) for _ in range(3))
         self.lib.oracle_frechet_scan(_ptr(c), m, _ptr(Ln), _ptr(Un), _ptr(Gn))
         return Ln, Un, Gn
+
+    def bonus_terms(self, c_sorted):
+        """(F_n, B_n) for n = 1..m of a descending profile (Eq. heterogeneity_decomp)."""
+        c = np.ascontiguousarray(c_sorted, dtype=np.float64)
+        m = c.shape[0]
+        F, Bn = np.zeros(m), np.zeros(m)
+        self.lib.oracle_bonus_terms(_ptr(c), m, _ptr(F), _ptr(Bn))
+        return F, Bn
+
+    def profile_terms(self, conf: np.ndarray, mask: np.ndarray):
+        """Per batch row at each rank of the sorted masked profile: dict(G, F, B, order)."""
+        c = np.ascontiguousarray(conf, dtype=np.float64)
+        B, L = c.shape
+        m = np.ascontiguousarray(mask, dtype=np.uint8).reshape(B, L)
+        G, F, Bn = (np.zeros((B, L)) for _ in range(3))
+        order = np.zeros((B, L), np.int32)
+        self.lib.oracle_profile_terms(_ptr(c), _ptr(m), B, L, _ptr(G), _ptr(F), _ptr(Bn),
+                                      _ptr(order))
+        return dict(G=G, F=F, B=Bn, order=order)
 
     def select_from_conf(self, conf: np.ndarray, tok: np.ndarray, mask: np.ndarray, mode: int,
                          param: float, out_tokens: np.ndarray | None = None):

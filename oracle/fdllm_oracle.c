@@ -330,6 +330,56 @@ int64_t oracle_select_robust_from_conf(const double *conf, const int32_t *tok, i
     return bad;
 }
 
+/* Eq. heterogeneity_decomp, term by term. */
+void oracle_bonus_terms(const double *c_sorted, int64_t m, double *Fn, double *Bn)
+{
+    for (int64_t n = 1; n <= m; ++n) {
+        const double cn = c_sorted[n - 1];
+        Fn[n - 1] = (double)(n + 1) * cn - (double)n;
+        double bonus = 0.0;
+        for (int64_t j = 1; j <= n - 1; ++j)
+            bonus += c_sorted[j - 1] - cn;
+        Bn[n - 1] = bonus;
+    }
+}
+
+void oracle_profile_terms(const double *conf, const uint8_t *mask, int64_t B, int64_t L,
+                          double *G, double *F, double *Bn, int32_t *order)
+{
+    candidate *cand = (candidate *)malloc((size_t)L * sizeof(candidate));
+    double *cs = (double *)malloc((size_t)L * sizeof(double));
+    double *Lt = (double *)malloc((size_t)L * sizeof(double));
+    double *Ut = (double *)malloc((size_t)L * sizeof(double));
+    for (int64_t b = 0; b < B; ++b) {
+        const int64_t row0 = b * L;
+        int64_t m = 0;
+        for (int64_t l = 0; l < L; ++l) {
+            G[row0 + l] = NAN;
+            F[row0 + l] = NAN;
+            Bn[row0 + l] = NAN;
+            order[row0 + l] = -1;
+            if (!mask[row0 + l])
+                continue;
+            cand[m].c = conf[row0 + l];
+            cand[m].pos = (int32_t)l;
+            ++m;
+        }
+        if (m == 0)
+            continue;
+        qsort(cand, (size_t)m, sizeof(candidate), by_confidence_desc);
+        for (int64_t j = 0; j < m; ++j) {
+            cs[j] = cand[j].c;
+            order[row0 + j] = cand[j].pos;
+        }
+        oracle_frechet_scan(cs, m, Lt, Ut, G + row0);
+        oracle_bonus_terms(cs, m, F + row0, Bn + row0);
+    }
+    free(cand);
+    free(cs);
+    free(Lt);
+    free(Ut);
+}
+
 int64_t oracle_select(const void *logits, int dtype, int64_t B, int64_t L, int64_t V,
                       uint8_t *mask, int mode, double param, int32_t *out_tokens,
                       uint8_t *out_commit, int32_t *out_n, double *margin, double *conf,

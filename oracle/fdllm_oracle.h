@@ -71,6 +71,18 @@ int64_t oracle_select_robust_from_conf(const double *conf, const int32_t *tok, i
                                        const double *eta_pos, int32_t *out_tokens,
                                        uint8_t *out_commit, int32_t *out_n, double *margin);
 
+/* Heterogeneity-bonus terms of a descending profile (Prop. heterogeneity-bonus, Eq.
+ * heterogeneity_decomp): for n = 1..m, F_n = (n+1) c_(n) - n (factor core) and
+ * B_n = sum_{j=1}^{n-1} (c_(j) - c_(n)) (heterogeneity bonus).  Outputs indexed n-1. */
+void oracle_bonus_terms(const double *c_sorted, int64_t m, double *Fn, double *Bn);
+
+/* Per batch row, the masked confidences sorted as in Alg. 1 (descending, ties: lower
+ * position first) and, at rank n = 1..m_b: G[b, n-1] (Eq. frechet_Ln_Un), F[b, n-1],
+ * Bn[b, n-1] (Eq. heterogeneity_decomp) and order[b, n-1] = the position at rank n.  Ranks
+ * beyond m_b hold NaN (order -1).  All arrays [B, L]. */
+void oracle_profile_terms(const double *conf, const uint8_t *mask, int64_t B, int64_t L,
+                          double *G, double *F, double *Bn, int32_t *order);
+
 /* oracle_confidence followed by oracle_select_from_conf.  conf/tok are caller scratch of
  * B*L entries; they come back holding the per-position confidences and argmax tokens. */
 int64_t oracle_select(const void *logits, int dtype, int64_t B, int64_t L, int64_t V,

@@ -474,10 +474,40 @@ def pin_robust_monotone_and_clipped(o):
     assert list(n_r) == [1, 1] and sets == [{0}, {0}]
 
 
+def pin_bonus_terms(o):
+    """Eq. heterogeneity_decomp: F_n and B_n against the hand-worked profiles, and
+    G_n = F_n + B_n whenever L_n > 0 with B_n >= 0 (zero iff the prefix is flat)."""
+    with open(GOLDEN) as fh:
+        cases = json.load(fh)["cases"]
+    for case in cases:
+        F, Bn = o.bonus_terms(np.array(case["c_sorted"]))
+        np.testing.assert_allclose(F, case["F"], atol=1e-12)
+        np.testing.assert_allclose(Bn, case["Bn"], atol=1e-12)
+    rng = np.random.default_rng(43)
+    for p in _random_profiles(rng, 200, 16, dyadic=256):
+        c = np.array(sorted(p, reverse=True))
+        Ln, _, Gn = o.frechet_scan(c)
+        F, Bn = o.bonus_terms(c)
+        assert np.all(Bn >= 0)
+        for n in range(1, len(c) + 1):
+            assert (Bn[n - 1] == 0) == bool(np.all(c[:n] == c[n - 1]))
+            if Ln[n - 1] > 0:
+                assert Gn[n - 1] == F[n - 1] + Bn[n - 1]
+    # the row-level terms follow the selection's order
+    conf = np.array([[0.3, 0.9, 0.0, 0.9, 0.7]])
+    mask = np.array([[1, 1, 0, 1, 1]], np.uint8)
+    t = o.profile_terms(conf, mask)
+    assert t["order"][0].tolist() == [1, 3, 4, 0, -1]
+    _, _, G = o.frechet_scan(np.array([0.9, 0.9, 0.7, 0.3]))
+    np.testing.assert_allclose(t["G"][0, :4], G, atol=0)
+    assert np.isnan(t["G"][0, 4]) and np.isnan(t["B"][0, 4])
+
+
 ALL_PINS = [
     pin_confidence_vs_torch, pin_confidence_closed_forms, pin_nonfinite, pin_hand_worked,
     pin_bruteforce_subsets, pin_equal_confidence_reduction, pin_heterogeneity_bonus,
     pin_matched_dominance, pin_greedy_equivalence, pin_monotone_prefix, pin_special_cases,
     pin_reveal_and_ties, pin_end_to_end, pin_robust_zero_eta_is_profile,
     pin_robust_calibration_penalty, pin_robust_bruteforce, pin_robust_monotone_and_clipped,
+    pin_bonus_terms,
 ]

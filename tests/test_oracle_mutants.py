@@ -47,6 +47,10 @@ MUTANTS = {
     "robust_ranks_by_c_hat": ("cand[m].c = c_low;", "cand[m].c = c_hat;"),
     "robust_eta_ignored": ("const double eta_i = eta_pos ? eta_pos[row0 + l] : eta;",
                            "const double eta_i = 0.0;"),
+    "factor_core_drops_plus_one": ("Fn[n - 1] = (double)(n + 1) * cn - (double)n;",
+                                   "Fn[n - 1] = (double)n * cn - (double)n;"),
+    "bonus_index_shifted": ("bonus += c_sorted[j - 1] - cn;", "bonus += c_sorted[j] - cn;"),
+    "bonus_sign_flipped": ("bonus += c_sorted[j - 1] - cn;", "bonus += cn - c_sorted[j - 1];"),
     # (old, new, occurrence): the robust selector repeats some lines of the plain one
     "robust_no_progress_fallback": ("if (nstar == 0)\n            nstar = 1;", "", 1),
     "robust_margin_not_strict": ("if (Gn[n - 1] > delta)", "if (Gn[n - 1] >= delta)"),
