@@ -179,7 +179,8 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
     mask0 = torch.from_numpy(mask0_np).to(dev)
     masked_rows = int(mask0_np.sum())
     alg_bytes = masked_rows * w.V * w.elem_bytes
-    mode = {"profile": fd.PROFILE, "factor": fd.FACTOR, "threshold": fd.THRESHOLD}[args.mode]
+    mode = {"profile": fd.PROFILE, "factor": fd.FACTOR, "threshold": fd.THRESHOLD,
+            "robust": fd.PROFILE}[args.mode]
 
     # one mask buffer per logits buffer, all restored by a single copy per replay
     masks = mask0.unsqueeze(0).repeat(n_buf, 1, 1).contiguous()
@@ -194,8 +195,12 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
     def step(i):
         if i % n_buf == 0:  # steady state: the same masked rows every step
             masks.copy_(masks0, non_blocking=True)
-        fd.fdllm_select(bufs[i % n_buf], masks[i % n_buf], args.param, mode, tok, commit,
-                        n_out, stream=stream)
+        if args.mode == "robust":
+            fd.fdllm_select_robust(bufs[i % n_buf], masks[i % n_buf], args.param, args.eta,
+                                   None, tok, commit, n_out, stream=stream)
+        else:
+            fd.fdllm_select(bufs[i % n_buf], masks[i % n_buf], args.param, mode, tok, commit,
+                            n_out, stream=stream)
 
     def k1_only(i):
         fd.fdllm_confidence(bufs[i % n_buf], mask0, conf, amax, stream=stream)
@@ -405,15 +410,22 @@ def run_oracle_timed(args, steps: int, warmup: int, budget_s: float | None):
     host = syn.host_bits(syn.make_logits(ws, seed=1234, device="cpu"))
     mask = syn.make_mask(ws, seed=1234)
     threads = os.cpu_count() or 1
-    mode = {"profile": oracle.PROFILE, "factor": oracle.FACTOR,
-            "threshold": oracle.THRESHOLD}[args.mode]
     orc = oracle.default()
+    if args.mode == "robust":
+        def one():
+            orc.select_robust(host, mask, args.param, args.eta, None, nthreads=threads)
+    else:
+        mode = {"profile": oracle.PROFILE, "factor": oracle.FACTOR,
+                "threshold": oracle.THRESHOLD}[args.mode]
+
+        def one():
+            orc.select(host, mask, mode, args.param, nthreads=threads)
     for _ in range(warmup):
-        orc.select(host, mask, mode, args.param, nthreads=threads)
+        one()
     t0 = time.perf_counter()
     done = 0
     while True:
-        orc.select(host, mask, mode, args.param, nthreads=threads)
+        one()
         done += 1
         elapsed = time.perf_counter() - t0
         if budget_s is not None and elapsed >= budget_s:
@@ -465,7 +477,10 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="serving_b64_l32_bf16")
-    ap.add_argument("--mode", choices=["profile", "factor", "threshold"], default="profile")
+    ap.add_argument("--mode", choices=["profile", "factor", "threshold", "robust"],
+                    default="profile")
+    ap.add_argument("--eta", type=float, default=0.02,
+                    help="calibration allowance of the robust rule (App. C)")
     ap.add_argument("--param", type=float, default=1.0)
     ap.add_argument("--buffers", type=int, default=4)
     ap.add_argument("--no-graph", action="store_true")

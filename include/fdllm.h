@@ -176,6 +176,24 @@ fdllm_status fdllm_select_from_conf(const float *conf, const int32_t *argmax, in
                                     int32_t *out_tokens, uint8_t *out_commit, int32_t *out_n,
                                     void *stream);
 
+/* Heterogeneity-bonus diagnostics (Prop. heterogeneity-bonus, Eq. heterogeneity_decomp,
+ * Remark adaptive-factor).  For each batch row, the masked confidences are sorted as the
+ * selection sorts them (descending, ties: lower position first); at rank n = 1..m_b:
+ *   out_G[b, n-1]     = G_n = max{0, sum_{j<=n} c_(j) - (n-1)} - (1 - c_(n))
+ *   out_F[b, n-1]     = F_n = (n+1) c_(n) - n                (factor core)
+ *   out_B[b, n-1]     = B_n = sum_{j<n} (c_(j) - c_(n))       (heterogeneity bonus)
+ *   out_order[b, n-1] = the position holding c_(n)
+ * Ranks n > m_b get NaN (order -1).  G_n = F_n + B_n wherever the lower bound is positive,
+ * and the profile rule with margin delta behaves as the factor rule with the effective
+ * factor f_eff(n) = 1 - delta + B_n.
+ *   conf  [B, L] fp32 device (e.g. from fdllm_confidence), read at masked positions.
+ *   mask  [B, L] uint8 device, nonzero = masked (not modified).
+ *   out_G, out_F, out_B  [B, L] fp64 device, each nullable; out_order [B, L] int32, nullable.
+ * Asynchronous on `stream`; needs no workspace. */
+fdllm_status fdllm_profile_terms(const float *conf, const uint8_t *mask, int B, int L,
+                                 double *out_G, double *out_F, double *out_B,
+                                 int32_t *out_order, void *stream);
+
 /* Synchronises `stream`, then reports (and clears) the sticky device error of the library
  * workspace on the current device: FDLLM_ERR_DEVICE if a kernel gave up a bounded wait
  * since the last call, FDLLM_OK otherwise.  For fdllm_select_ws, pass the workspace to

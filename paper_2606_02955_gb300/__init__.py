@@ -21,6 +21,7 @@ __all__ = [
     "fdllm_confidence", "fdllm_select_from_conf", "fdllm_device_status",
     "fdllm_workspace_status", "fdllm_release_workspace", "fdllm_status_string",
     "fdllm_version", "library_path", "fdllm_select_static", "fdllm_select_robust",
+    "fdllm_profile_terms",
 ]
 
 BF16, FP32 = 0, 1
@@ -56,6 +57,8 @@ def _load():
     lib.fdllm_confidence.restype = i
     lib.fdllm_select_from_conf.argtypes = [p, p, i, i, p, d, i, p, p, p, p]
     lib.fdllm_select_from_conf.restype = i
+    lib.fdllm_profile_terms.argtypes = [p, p, i, i, p, p, p, p, p]
+    lib.fdllm_profile_terms.restype = i
     lib.fdllm_device_status.argtypes = [p]
     lib.fdllm_device_status.restype = i
     lib.fdllm_workspace_status.argtypes = [p, p]
@@ -269,6 +272,21 @@ def fdllm_select_from_conf(conf: torch.Tensor, argmax: torch.Tensor, mask: torch
                                      _dev(out_n, "out_n", torch.int32, (B,)), _stream(stream))
     _check(st, "fdllm_select_from_conf")
     return out_tokens, out_commit, out_n
+
+
+def fdllm_profile_terms(conf: torch.Tensor, mask: torch.Tensor, stream=None):
+    """Heterogeneity-bonus diagnostics by rank of each row's sorted masked profile:
+    dict(G, F, B) fp64 [B, L] and order int32 [B, L] (NaN / -1 beyond the masked count)."""
+    B, L = conf.shape
+    dev = conf.device
+    G, F, Bn = (torch.empty((B, L), dtype=torch.float64, device=dev) for _ in range(3))
+    order = torch.empty((B, L), dtype=torch.int32, device=dev)
+    st = _load().fdllm_profile_terms(_dev(conf, "conf", torch.float32, (B, L)),
+                                     _dev(mask, "mask", torch.uint8, (B, L)), B, L,
+                                     G.data_ptr(), F.data_ptr(), Bn.data_ptr(),
+                                     order.data_ptr(), _stream(stream))
+    _check(st, "fdllm_profile_terms")
+    return dict(G=G, F=F, B=Bn, order=order)
 
 
 def fdllm_device_status(stream=None) -> int:

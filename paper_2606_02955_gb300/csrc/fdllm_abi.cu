@@ -374,6 +374,28 @@ fdllm_status fdllm_select_from_conf(const float *conf, const int32_t *argmax, in
     return FDLLM_OK;
 }
 
+fdllm_status fdllm_profile_terms(const float *conf, const uint8_t *mask, int B, int L,
+                                 double *out_G, double *out_F, double *out_B,
+                                 int32_t *out_order, void *stream)
+{
+    if (B < 1 || L < 1 || L > FDLLM_MAX_L || (int64_t)B * L > FDLLM_MAX_ROWS)
+        return FDLLM_ERR_ARG;
+    if (!conf || !mask)
+        return FDLLM_ERR_ARG;
+    ProfileTermsArgs a;
+    a.conf = conf;
+    a.mask = mask;
+    a.B = B;
+    a.L = L;
+    a.out_G = out_G;
+    a.out_F = out_F;
+    a.out_B = out_B;
+    a.out_order = out_order;
+    return launch_profile_terms(a, static_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? FDLLM_OK
+               : FDLLM_ERR_CUDA;
+}
+
 fdllm_status fdllm_device_status(void *stream)
 {
     int dev = 0;

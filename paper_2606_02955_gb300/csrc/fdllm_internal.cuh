@@ -116,6 +116,19 @@ struct ProfileSelectArgs {
 
 cudaError_t launch_profile_select(const ProfileSelectArgs &a, cudaStream_t stream);
 
+struct ProfileTermsArgs {
+    const float *conf;       // [B, L]
+    const uint8_t *mask;     // [B, L]
+    int B;
+    int L;
+    double *out_G;           // [B, L] by rank, nullable
+    double *out_F;           // [B, L] by rank, nullable
+    double *out_B;           // [B, L] by rank, nullable
+    int32_t *out_order;      // [B, L] position at each rank, nullable
+};
+
+cudaError_t launch_profile_terms(const ProfileTermsArgs &a, cudaStream_t stream);
+
 // ------------------------------------------------------------------ device helpers
 #ifdef __CUDACC__
 __device__ __forceinline__ float ex2_mufu(float x)

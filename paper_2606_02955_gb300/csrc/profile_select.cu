@@ -198,6 +198,47 @@ __global__ void __launch_bounds__(T) profile_select_kernel(const ProfileSelectAr
         a.out_n[blockIdx.x] = nstar;
 }
 
+// Heterogeneity-bonus diagnostics of one batch row per CTA (Prop. heterogeneity-bonus,
+// Eq. heterogeneity_decomp): the masked confidences sorted as in the selection, an fp64
+// inclusive scan S_n = sum_{j<=n} c_(j), and at rank n: G_n = max{0, S_n - (n-1)} - (1 - c_(n)),
+// F_n = (n+1) c_(n) - n and B_n = S_n - n c_(n) (= sum_{j<n} (c_(j) - c_(n))).
+template <int T>
+__global__ void __launch_bounds__(T) profile_terms_kernel(const ProfileTermsArgs a)
+{
+    __shared__ uint64_t sk[T > 32 ? T : 1];
+    __shared__ double warp_tot[32];
+    const int t = threadIdx.x;
+    const int L = a.L;
+    const int64_t base = (int64_t)blockIdx.x * L;
+    const bool masked = t < L && a.mask[base + t] != 0;
+    const float c = masked ? a.conf[base + t] : 0.0f;
+    uint64_t key = t < L ? make_key(masked, c, t) : kPadKey;
+    const int m = __syncthreads_count(masked);
+    key = bitonic_sort<T>(key, sk);
+    const bool live = t < m;
+    const double cn = live ? (double)key_conf(key) : 0.0;
+    const double S = block_inclusive_scan<T>(cn, warp_tot);
+    if (t >= L)
+        return;
+    const double n = (double)(t + 1);
+    const double nan = __longlong_as_double(0x7FF8000000000000ll);
+    if (a.out_G != nullptr)
+        a.out_G[base + t] = live ? fmax(0.0, S - (n - 1.0)) - (1.0 - cn) : nan;
+    if (a.out_F != nullptr)
+        a.out_F[base + t] = live ? (n + 1.0) * cn - n : nan;
+    if (a.out_B != nullptr)
+        a.out_B[base + t] = live ? S - n * cn : nan;
+    if (a.out_order != nullptr)
+        a.out_order[base + t] = live ? (int32_t)(key & 0xFFFFFFFFu) : -1;
+}
+
+template <int T>
+cudaError_t launch_terms_t(const ProfileTermsArgs &a, cudaStream_t stream)
+{
+    profile_terms_kernel<T><<<a.B, T, 0, stream>>>(a);
+    return cudaGetLastError();
+}
+
 template <int T>
 cudaError_t launch_t(const ProfileSelectArgs &a, cudaStream_t stream)
 {
@@ -228,6 +269,21 @@ cudaError_t launch_profile_select(const ProfileSelectArgs &a, cudaStream_t strea
     if (a.L <= 512)
         return launch_t<512>(a, stream);
     return launch_t<1024>(a, stream);
+}
+
+cudaError_t launch_profile_terms(const ProfileTermsArgs &a, cudaStream_t stream)
+{
+    if (a.L <= 32)
+        return launch_terms_t<32>(a, stream);
+    if (a.L <= 64)
+        return launch_terms_t<64>(a, stream);
+    if (a.L <= 128)
+        return launch_terms_t<128>(a, stream);
+    if (a.L <= 256)
+        return launch_terms_t<256>(a, stream);
+    if (a.L <= 512)
+        return launch_terms_t<512>(a, stream);
+    return launch_terms_t<1024>(a, stream);
 }
 
 }  // namespace fdllm
