@@ -194,6 +194,15 @@ fdllm_status fdllm_profile_terms(const float *conf, const uint8_t *mask, int B, 
                                  double *out_G, double *out_F, double *out_B,
                                  int32_t *out_order, void *stream);
 
+/* Health check of the library's failure detection: every wait inside the kernels is
+ * bounded, and a wait that runs out records a device error and lets the kernel return
+ * instead of hanging.  This launches one thread that waits on a barrier nobody completes,
+ * with a limit of `seconds` (0 < seconds <= 10), synchronises `stream` and returns
+ * FDLLM_ERR_DEVICE when the wait ran out and was reported as it should (FDLLM_OK would mean
+ * the wait did not run out).  The device stays usable afterwards.  The paper has no
+ * counterpart. */
+fdllm_status fdllm_check_bounded_wait(double seconds, void *stream);
+
 /* Synchronises `stream`, then reports (and clears) the sticky device error of the library
  * workspace on the current device: FDLLM_ERR_DEVICE if a kernel gave up a bounded wait
  * since the last call, FDLLM_OK otherwise.  For fdllm_select_ws, pass the workspace to

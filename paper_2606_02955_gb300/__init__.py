@@ -21,7 +21,7 @@ __all__ = [
     "fdllm_confidence", "fdllm_select_from_conf", "fdllm_device_status",
     "fdllm_workspace_status", "fdllm_release_workspace", "fdllm_status_string",
     "fdllm_version", "library_path", "fdllm_select_static", "fdllm_select_robust",
-    "fdllm_profile_terms",
+    "fdllm_profile_terms", "fdllm_check_bounded_wait",
 ]
 
 BF16, FP32 = 0, 1
@@ -59,6 +59,8 @@ def _load():
     lib.fdllm_select_from_conf.restype = i
     lib.fdllm_profile_terms.argtypes = [p, p, i, i, p, p, p, p, p]
     lib.fdllm_profile_terms.restype = i
+    lib.fdllm_check_bounded_wait.argtypes = [d, p]
+    lib.fdllm_check_bounded_wait.restype = i
     lib.fdllm_device_status.argtypes = [p]
     lib.fdllm_device_status.restype = i
     lib.fdllm_workspace_status.argtypes = [p, p]
@@ -287,6 +289,12 @@ def fdllm_profile_terms(conf: torch.Tensor, mask: torch.Tensor, stream=None):
                                      order.data_ptr(), _stream(stream))
     _check(st, "fdllm_profile_terms")
     return dict(G=G, F=F, B=Bn, order=order)
+
+
+def fdllm_check_bounded_wait(seconds: float = 0.01, stream=None) -> int:
+    """Makes one kernel wait on a barrier nobody completes; returns the status code
+    (FDLLM_ERR_DEVICE = 6 when the bounded wait ran out and was reported)."""
+    return _load().fdllm_check_bounded_wait(float(seconds), _stream(stream))
 
 
 def fdllm_device_status(stream=None) -> int:

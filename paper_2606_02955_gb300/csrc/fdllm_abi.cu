@@ -191,6 +191,9 @@ fdllm_status read_and_clear_status(uint32_t *status, cudaStream_t stream)
 // the device address comes from cudaGetSymbolAddress, looked up once per device.
 static __device__ __align__(256) uint8_t g_static_scratch[FDLLM_STATIC_SCRATCH_BYTES];
 
+// Status word of fdllm_check_bounded_wait (kept apart from every workspace).
+static __device__ uint32_t g_probe_status;
+
 void *g_static_scratch_addr[kMaxDevices] = {nullptr};
 std::mutex g_static_mutex;
 
@@ -394,6 +397,21 @@ fdllm_status fdllm_profile_terms(const float *conf, const uint8_t *mask, int B, 
     return launch_profile_terms(a, static_cast<cudaStream_t>(stream)) == cudaSuccess
                ? FDLLM_OK
                : FDLLM_ERR_CUDA;
+}
+
+fdllm_status fdllm_check_bounded_wait(double seconds, void *stream)
+{
+    if (!(seconds > 0.0) || seconds > 10.0)
+        return FDLLM_ERR_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    uint32_t *status = nullptr;
+    if (cudaGetSymbolAddress(reinterpret_cast<void **>(&status), g_probe_status) != cudaSuccess)
+        return FDLLM_ERR_CUDA;
+    if (cudaMemsetAsync(status, 0, sizeof(uint32_t), s) != cudaSuccess)
+        return FDLLM_ERR_CUDA;
+    if (launch_bounded_wait_probe(status, (uint64_t)(seconds * 1e9), s) != cudaSuccess)
+        return FDLLM_ERR_CUDA;
+    return read_and_clear_status(status, s);
 }
 
 fdllm_status fdllm_device_status(void *stream)

@@ -74,6 +74,9 @@ inline UnitPlan plan_units(int64_t row_bytes)
 // kernel on the stream.
 cudaError_t launch_vocab_reduce(const VocabReduceArgs &a, int esize, cudaStream_t stream);
 
+// One thread waits, bounded by limit_ns, on an mbarrier that never completes.
+cudaError_t launch_bounded_wait_probe(uint32_t *status, uint64_t limit_ns, cudaStream_t stream);
+
 // Per masked position: combine its unit partials, write (c, x_hat); resets next_unit.
 // Launched as a programmatic dependent of the vocab reduction.
 struct FinalizeArgs {

@@ -60,8 +60,9 @@ __device__ __forceinline__ uint64_t global_timer_ns()
 }
 
 // Waits for the phase of `bar` with the given parity to complete.  Gives up after
-// kWaitLimitNs, sets kDevStatTimeout in *status and returns false.
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, uint32_t *status)
+// limit_ns, sets kDevStatTimeout in *status and returns false.
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, uint32_t *status,
+                                          uint64_t limit_ns = kWaitLimitNs)
 {
     if (mbar_try_wait(bar, parity))
         return true;
@@ -69,7 +70,7 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, uint32
     for (uint32_t it = 1;; ++it) {
         if (mbar_try_wait(bar, parity))
             return true;
-        if ((it & 63u) == 0 && global_timer_ns() - t0 > kWaitLimitNs) {
+        if ((it & 63u) == 0 && global_timer_ns() - t0 > limit_ns) {
             atomicOr(status, kDevStatTimeout);
             return false;
         }

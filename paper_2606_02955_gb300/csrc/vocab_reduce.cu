@@ -601,7 +601,23 @@ int variant_index()
     return v;
 }
 
+// Health check of the bounded waits: one thread waits on an mbarrier that nobody arrives
+// at, so the wait must run out after limit_ns, record kDevStatTimeout and return.
+__global__ void bounded_wait_probe_kernel(uint32_t *status, uint64_t limit_ns)
+{
+    __shared__ uint64_t bar;
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+    mbar_wait(&bar, 0, status, limit_ns);
+}
+
 }  // namespace
+
+cudaError_t launch_bounded_wait_probe(uint32_t *status, uint64_t limit_ns, cudaStream_t stream)
+{
+    bounded_wait_probe_kernel<<<1, 1, 0, stream>>>(status, limit_ns);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_vocab_reduce(const VocabReduceArgs &a, int esize, cudaStream_t stream)
 {

@@ -1,0 +1,36 @@
+"""Failure detection on the GPU without a fault: a kernel wait that nothing completes must
+run out after its limit, be reported as a device error, and leave the device usable."""
+import time
+
+import numpy as np
+import pytest
+import torch
+
+import fdllm_synth as syn
+
+pytestmark = pytest.mark.gpu
+ERR_DEVICE = 6
+
+
+def test_bounded_wait_runs_out_and_device_stays_usable(fd, orc):
+    t0 = time.perf_counter()
+    assert fd.fdllm_check_bounded_wait(0.02) == ERR_DEVICE
+    elapsed = time.perf_counter() - t0
+    assert 0.015 <= elapsed < 2.0
+    assert fd.fdllm_check_bounded_wait(0.02) == ERR_DEVICE  # repeatable
+    # the context is intact: a normal step still runs and its status is clean
+    w = syn.WORKLOADS["target_b8_l32_bf16"]
+    logits = syn.make_logits(w, seed=11, device="cuda")
+    mask_np = syn.make_mask(w, seed=11)
+    tok, commit, n = fd.fdllm_select(logits, torch.from_numpy(mask_np.copy()).cuda(), 0.75,
+                                     fd.PROFILE)
+    torch.cuda.synchronize()
+    assert fd.fdllm_device_status() == 0
+    ref = orc.select(syn.host_bits(logits), mask_np, 0, 0.75)
+    ok = ref["margin"] >= 1e-5
+    assert np.array_equal(n.cpu().numpy()[ok], ref["n"][ok])
+
+
+def test_bounded_wait_rejects_bad_limits(fd):
+    assert fd.fdllm_check_bounded_wait(0.0) == 1
+    assert fd.fdllm_check_bounded_wait(60.0) == 1
