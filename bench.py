@@ -390,6 +390,94 @@ def run_loop(args) -> dict:
             "dtype": w.dtype, "param": args.param, "data": "synthetic", "results": out}
 
 
+def run_decode_loop(args) -> dict:
+    """A whole generation (gen_len tokens per row in blocks of block_len) on the
+    counter-based synthetic forward pass, two ways: the device-resident loop
+    (fdllm_decode_loop: one call, one CUDA graph with a conditional WHILE node) and a
+    host-driven loop (per step: forward launch, fdllm_select, reveal, and a host read of
+    "any masked left").  Both take the same decisions, so the difference in wall time is the
+    cost of the host round trips.  Wall time per generation, median of --repeats."""
+    import time
+
+    import numpy as np
+    import torch
+
+    import fdllm_synth as syn
+    import paper_2606_02955_gb300 as fd
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    B, gen, Lb, V = args.loop_batch, args.gen_len, args.block_len, syn.LLADA_VOCAB
+    seed, peak = 2024, args.peak
+    mode = fd.MODES[args.mode]
+    logits = torch.empty((B, Lb, V), dtype=torch.bfloat16, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def forward(state, mask, out, strm):
+        syn.synth_block_logits_gpu(out, mask, B, Lb, V, seed, step_ptr=state, peak_max=peak,
+                                   stream_ptr=strm)
+
+    def device_loop():
+        return fd.fdllm_decode_loop(forward, logits, gen, args.param, mode)
+
+    seq_h = torch.empty((B, gen), dtype=torch.int32, device=dev)
+    mask = torch.empty((B, Lb), dtype=torch.uint8, device=dev)
+    tok = torch.empty((B, Lb), dtype=torch.int32, device=dev)
+    commit = torch.empty((B, Lb), dtype=torch.uint8, device=dev)
+    n = torch.empty((B,), dtype=torch.int32, device=dev)
+
+    def host_loop():
+        seq_h.fill_(-1)
+        step, nfe = 0, []
+        for blk in range(gen // Lb):
+            mask.fill_(1)
+            k = 0
+            while bool(mask.any().item()):
+                syn.synth_block_logits_gpu(logits.data_ptr(), mask.data_ptr(), B, Lb, V, seed,
+                                           step=step, peak_max=peak,
+                                           stream_ptr=stream.cuda_stream)
+                fd.fdllm_select(logits, mask, args.param, mode, tok, commit, n)
+                view = seq_h[:, blk * Lb:(blk + 1) * Lb]
+                view.copy_(torch.where(commit.bool(), tok, view))
+                step += 1
+                k += 1
+            nfe.append(k)
+        return seq_h, nfe, step
+
+    def timed(fn):
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        r = fn()
+        torch.cuda.synchronize()
+        return time.perf_counter() - t0, r
+
+    for _ in range(max(1, args.warmup_loops)):
+        timed(device_loop)
+        timed(host_loop)
+    dts, hts = [], []
+    for _ in range(args.repeats):
+        dt, (seq_d, nfe_d, steps_d) = timed(device_loop)
+        ht, (seq_hh, nfe_hh, steps_hh) = timed(host_loop)
+        dts.append(dt)
+        hts.append(ht)
+    dms, hms = 1e3 * float(np.median(dts)), 1e3 * float(np.median(hts))
+    identical = bool(torch.equal(seq_d, seq_hh)) and list(nfe_d.cpu().numpy()) == nfe_hh
+    tokens = B * gen
+    return {
+        "metric": "decode loop: generated tokens/s on a synthetic forward pass",
+        "workload": "decode_loop_b%d_gen%d_block%d_bf16" % (B, gen, Lb),
+        "B": B, "gen_len": gen, "block_len": Lb, "V": V, "dtype": "bf16",
+        "mode": args.mode, "param": args.param, "peak": peak, "data": "synthetic",
+        "steps": int(steps_d), "nfe_per_block": [int(x) for x in nfe_d.cpu().numpy()],
+        "device_loop": {"ms_per_generation": dms, "tokens_per_s": tokens / (dms * 1e-3),
+                        "ms_per_step": dms / max(steps_d, 1)},
+        "host_loop": {"ms_per_generation": hms, "tokens_per_s": tokens / (hms * 1e-3),
+                      "ms_per_step": hms / max(steps_hh, 1)},
+        "host_round_trip_us_per_step": 1e3 * (hms - dms) / max(steps_d, 1),
+        "identical_decisions": identical, "repeats": args.repeats,
+    }
+
+
 # ----------------------------------------------------------------------------- oracle arm
 def oracle_sample_rows(args) -> int:
     return max(1, min(args.sample_rows, 64))
@@ -492,7 +580,20 @@ def main(argv=None):
     ap.add_argument("--loop", action="store_true",
                     help="run the selection until no mask remains (profile vs factor) and "
                          "report steps and per-step latency instead of the throughput line")
+    ap.add_argument("--decode-loop", action="store_true",
+                    help="time a whole generation through the device-resident decode loop "
+                         "and through a host-driven loop, instead of the throughput line")
+    ap.add_argument("--loop-batch", type=int, default=8)
+    ap.add_argument("--gen-len", type=int, default=256)
+    ap.add_argument("--block-len", type=int, default=32)
+    ap.add_argument("--peak", type=float, default=20.0,
+                    help="decode loop: largest planted logit height of the synthetic forward")
+    ap.add_argument("--repeats", type=int, default=5)
+    ap.add_argument("--warmup-loops", type=int, default=2)
     args = ap.parse_args(argv)
+    if args.decode_loop:
+        print(json.dumps(run_decode_loop(args)), flush=True)
+        return
     if args.loop:
         if args.workload == "serving_b64_l32_bf16":
             args.workload = "full_seq_b16_l1024_fp32"

@@ -19,8 +19,12 @@ multi-token commits, ties and profile-vs-factor differences are exercised.
 """
 from __future__ import annotations
 
+import ctypes
 import dataclasses
 import math
+import os
+import shutil
+import subprocess
 
 import numpy as np
 import torch
@@ -186,3 +190,47 @@ def host_bits(logits: torch.Tensor) -> np.ndarray:
     if t.dtype == torch.float32:
         return t.numpy()
     raise TypeError(t.dtype)
+
+
+# ----------------------------------------------------------------------------- GPU stand-in
+# Counter-based synthetic logits on the GPU (fdllm_synth_cuda.cu): the forward pass of the
+# decode-loop tests and benchmarks.  The CPU oracle implements the same generator itself.
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SYNTH_SRC = os.path.join(_HERE, "fdllm_synth_cuda.cu")
+_SYNTH_LIB = os.path.join(_HERE, "_build", "libfdllm_synth.so")
+_synth = None
+
+
+def build_synth_cuda(force: bool = False) -> str:
+    if (not force and os.path.exists(_SYNTH_LIB)
+            and os.path.getmtime(_SYNTH_LIB) >= os.path.getmtime(_SYNTH_SRC)):
+        return _SYNTH_LIB
+    nvcc = shutil.which("nvcc") or "/usr/local/cuda/bin/nvcc"
+    os.makedirs(os.path.dirname(_SYNTH_LIB), exist_ok=True)
+    subprocess.run([nvcc, "-gencode", "arch=compute_103a,code=sm_103a", "-O3", "-std=c++17",
+                    "-Xcompiler", "-fPIC", "-shared", _SYNTH_SRC, "-o", _SYNTH_LIB + ".tmp"],
+                   check=True, capture_output=True, text=True)
+    os.replace(_SYNTH_LIB + ".tmp", _SYNTH_LIB)
+    return _SYNTH_LIB
+
+
+def _synth_lib():
+    global _synth
+    if _synth is None:
+        lib = ctypes.CDLL(build_synth_cuda())
+        p, i = ctypes.c_void_p, ctypes.c_int
+        lib.fdllm_synth_block_logits.argtypes = [p, p, i, i, i, ctypes.c_ulonglong, p,
+                                                 ctypes.c_longlong, ctypes.c_double, p]
+        lib.fdllm_synth_block_logits.restype = i
+        _synth = lib
+    return _synth
+
+
+def synth_block_logits_gpu(out_ptr, mask_ptr, B, L, V, seed, step_ptr=None, step=0,
+                           peak_max=16.0, stream_ptr=None):
+    """Enqueue counter-based bf16 logits [B, L, V] (raw device pointers; rows whose mask
+    byte is 0 are skipped; the step is read from step_ptr on the device when given)."""
+    err = _synth_lib().fdllm_synth_block_logits(out_ptr, mask_ptr, B, L, V, int(seed), step_ptr,
+                                                int(step), float(peak_max), stream_ptr)
+    if err != 0:
+        raise RuntimeError("synthetic logits launch failed: %d" % err)

@@ -176,6 +176,43 @@ fdllm_status fdllm_select_from_conf(const float *conf, const int32_t *argmax, in
                                     int32_t *out_tokens, uint8_t *out_commit, int32_t *out_n,
                                     void *stream);
 
+/* Model forward pass used by fdllm_decode_loop.  It must only enqueue stream-ordered GPU
+ * work on `stream`: it is called while the loop body is being captured into a CUDA graph
+ * (once, or twice when the driver rejects the first capture and the body is captured again
+ * without programmatic dependent launches), and the captured work is replayed at every
+ * step.  It must not synchronise or allocate.  It writes logits [B, block_len, V]
+ * of the current block into `logits` for the rows with block_mask != 0.  loop_state is a
+ * device pointer to two int32 values read at run time: [0] the global step (forward passes
+ * so far), [1] the current block.  Return 0 on success. */
+typedef int (*fdllm_forward_fn)(void *user, const int32_t *loop_state,
+                                const uint8_t *block_mask, void *logits, void *stream);
+
+/* Algorithm 1's outer loop on the GPU, with no host round trip per step: for each of
+ * gen_len / block_len blocks, start with the block fully masked and repeat {forward pass;
+ * selection with (mode, param) as in fdllm_select; reveal} while the block has masked
+ * positions (Alg. 1: a block's steps go on until none of its positions is masked), then
+ * move to the next block.
+ * The loop is one CUDA graph with a conditional WHILE node; the forward pass, the two
+ * selection kernels and a controller kernel form its body.
+ *   logits          [B, block_len, V] device buffer the forward pass writes (dtype as given).
+ *   seq_tokens      [B, gen_len] int32 device output: the committed tokens (-1 if none).
+ *   nfe_per_block   [gen_len / block_len] int32 device output: steps (NFE) per block.
+ *   max_steps       bound on the total number of steps; reaching it ends the loop early
+ *                   and returns FDLLM_ERR_DEVICE.
+ *   out_steps       host int: total steps taken.
+ * Synchronous: returns when the generation is finished.  Allocates its own small buffers
+ * and the library workspace (outside the graph).  Limits as fdllm_select with L = block_len;
+ * modes FDLLM_PROFILE, FDLLM_FACTOR and FDLLM_THRESHOLD.  Errors: FDLLM_ERR_ARG for a bad
+ * argument (checked before any device work) or a forward pass that returned nonzero;
+ * FDLLM_ERR_CUDA for a failed graph build or launch.  Uses the library-owned workspace of
+ * fdllm_select: no other selection may run on this device from another thread meanwhile.
+ * Every step commits at least one position of each row that still has masked positions, so
+ * each block ends after at most block_len steps. */
+fdllm_status fdllm_decode_loop(int B, int gen_len, int block_len, int V, int dtype,
+                               double param, int mode, fdllm_forward_fn forward, void *user,
+                               void *logits, int32_t *seq_tokens, int32_t *nfe_per_block,
+                               int max_steps, int *out_steps, void *stream);
+
 /* Heterogeneity-bonus diagnostics (Prop. heterogeneity-bonus, Eq. heterogeneity_decomp,
  * Remark adaptive-factor).  For each batch row, the masked confidences are sorted as the
  * selection sorts them (descending, ties: lower position first); at rank n = 1..m_b:

@@ -90,6 +90,11 @@ class Oracle:
         lib.oracle_bonus_terms.restype = None
         lib.oracle_profile_terms.argtypes = [p, p, i64, i64, p, p, p, p]
         lib.oracle_profile_terms.restype = None
+        u64 = ctypes.c_uint64
+        lib.oracle_synth_block_logits.argtypes = [p, p, i64, i64, i64, u64, u64, d]
+        lib.oracle_synth_block_logits.restype = None
+        lib.oracle_decode_loop.argtypes = [i64, i64, i64, i64, i32, d, u64, d, i64, p, p, p, i32]
+        lib.oracle_decode_loop.restype = i64
         self.lib = lib
         self.path = lib_path
 
@@ -132,6 +137,25 @@ class Oracle:
         self.lib.oracle_profile_terms(_ptr(c), _ptr(m), B, L, _ptr(G), _ptr(F), _ptr(Bn),
                                       _ptr(order))
         return dict(G=G, F=F, B=Bn, order=order)
+
+    def synth_block_logits(self, B, L, V, seed, step, peak_max, mask=None):
+        """Counter-based synthetic bf16 logits (uint16 bits [B, L, V]); unmasked rows zero."""
+        out = np.zeros((B, L, V), np.uint16)
+        m = None if mask is None else np.ascontiguousarray(mask, np.uint8).reshape(B, L)
+        self.lib.oracle_synth_block_logits(_ptr(out), None if m is None else _ptr(m), B, L, V,
+                                           int(seed), int(step), float(peak_max))
+        return out
+
+    def decode_loop(self, B, gen_len, block_len, V, mode, param, seed, peak_max, max_steps,
+                    nthreads: int = 1):
+        """Algorithm 1's outer loop on the synthetic forward: dict(seq, nfe, margin, steps)."""
+        seq = np.zeros((B, gen_len), np.int32)
+        nfe = np.zeros(gen_len // block_len, np.int32)
+        margin = np.zeros(B, np.float64)
+        steps = self.lib.oracle_decode_loop(B, gen_len, block_len, V, int(mode), float(param),
+                                            int(seed), float(peak_max), int(max_steps),
+                                            _ptr(seq), _ptr(nfe), _ptr(margin), int(nthreads))
+        return dict(seq=seq, nfe=nfe, margin=margin, steps=int(steps))
 
     def select_from_conf(self, conf: np.ndarray, tok: np.ndarray, mask: np.ndarray, mode: int,
                          param: float, out_tokens: np.ndarray | None = None):

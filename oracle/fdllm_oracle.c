@@ -390,3 +390,111 @@ int64_t oracle_select(const void *logits, int dtype, int64_t B, int64_t L, int64
     return oracle_select_from_conf(conf, tok, B, L, mask, mode, param, out_tokens, out_commit,
                                    out_n, margin);
 }
+
+/* ---- synthetic forward pass and the decode loop (test infrastructure) ---- */
+
+static uint64_t splitmix_mix(uint64_t z)
+{
+    z ^= z >> 30;
+    z *= 0xBF58476D1CE4E5B9ull;
+    z ^= z >> 27;
+    z *= 0x94D049BB133111EBull;
+    z ^= z >> 31;
+    return z;
+}
+
+/* fp32 -> bf16 bits, round to nearest even (finite inputs). */
+static uint16_t bf16_round(float f)
+{
+    uint32_t u;
+    memcpy(&u, &f, sizeof u);
+    const uint32_t lsb = (u >> 16) & 1u;
+    return (uint16_t)((u + 0x7FFFu + lsb) >> 16);
+}
+
+void oracle_synth_block_logits(uint16_t *out, const uint8_t *mask, int64_t B, int64_t L,
+                               int64_t V, uint64_t seed, uint64_t step, double peak_max)
+{
+    const uint64_t G = 0x9E3779B97F4A7C15ull;
+    const float noise_scale = (float)(sqrt(3.0) / 131072.0);
+    const float peak_scale = (float)(peak_max / 16777216.0);
+    for (int64_t b = 0; b < B; ++b)
+        for (int64_t l = 0; l < L; ++l) {
+            const int64_t row = b * L + l;
+            if (mask && !mask[row])
+                continue;
+            const uint64_t k = splitmix_mix(
+                seed ^ splitmix_mix(step * G ^ splitmix_mix(((uint64_t)b << 32) | (uint64_t)l)));
+            const uint64_t p = splitmix_mix(k ^ 0xD1B54A32D192ED03ull);
+            const int64_t pidx = (int64_t)(p % (uint64_t)V);
+            const float height = (float)(p >> 40) * peak_scale;
+            for (int64_t v = 0; v < V; ++v) {
+                const uint64_t h = splitmix_mix(k + (uint64_t)(v + 1) * G);
+                const int32_t s = (int32_t)(2 * (h & 0xFFFF) + 2 * ((h >> 16) & 0xFFFF) +
+                                            2 * ((h >> 32) & 0xFFFF) + 2 * ((h >> 48) & 0xFFFF) +
+                                            4) -
+                                  262144;
+                float x = (float)s * noise_scale;
+                if (v == pidx)
+                    x = x + height;
+                out[row * V + v] = bf16_round(x);
+            }
+        }
+}
+
+int64_t oracle_decode_loop(int64_t B, int64_t gen_len, int64_t block_len, int64_t V, int mode,
+                           double param, uint64_t seed, double peak_max, int64_t max_steps,
+                           int32_t *out_seq, int32_t *out_nfe, double *out_margin,
+                           int nthreads)
+{
+    const int64_t nblocks = gen_len / block_len, Lb = block_len;
+    uint16_t *logits = (uint16_t *)malloc((size_t)(B * Lb * V) * sizeof(uint16_t));
+    uint8_t *mask = (uint8_t *)malloc((size_t)(B * Lb));
+    int32_t *tokens = (int32_t *)malloc((size_t)(B * Lb) * sizeof(int32_t));
+    uint8_t *commit = (uint8_t *)malloc((size_t)(B * Lb));
+    int32_t *n = (int32_t *)malloc((size_t)B * sizeof(int32_t));
+    double *margin = (double *)malloc((size_t)B * sizeof(double));
+    double *conf = (double *)malloc((size_t)(B * Lb) * sizeof(double));
+    int32_t *tok = (int32_t *)malloc((size_t)(B * Lb) * sizeof(int32_t));
+    for (int64_t i = 0; i < B * gen_len; ++i)
+        out_seq[i] = -1;
+    for (int64_t b = 0; b < B; ++b)
+        out_margin[b] = INFINITY;
+    int64_t step = 0;
+    for (int64_t blk = 0; blk < nblocks; ++blk) {
+        int64_t nfe = 0;
+        for (int64_t i = 0; i < B * Lb; ++i)
+            mask[i] = 1;
+        for (;;) { /* while the block contains masked positions (Alg. 1) */
+            int any = 0;
+            for (int64_t i = 0; i < B * Lb; ++i)
+                any |= mask[i];
+            if (!any || step >= max_steps)
+                break;
+            oracle_synth_block_logits(logits, mask, B, Lb, V, seed, (uint64_t)step, peak_max);
+            for (int64_t i = 0; i < B * Lb; ++i)
+                tokens[i] = -1;
+            oracle_select(logits, ORACLE_BF16, B, Lb, V, mask, mode, param, tokens, commit, n,
+                          margin, conf, tok, nthreads);
+            for (int64_t b = 0; b < B; ++b) {
+                if (margin[b] < out_margin[b])
+                    out_margin[b] = margin[b];
+                for (int64_t l = 0; l < Lb; ++l)
+                    if (commit[b * Lb + l])
+                        out_seq[b * gen_len + blk * Lb + l] = tokens[b * Lb + l];
+            }
+            ++step;
+            ++nfe;
+        }
+        out_nfe[blk] = (int32_t)nfe;
+    }
+    free(logits);
+    free(mask);
+    free(tokens);
+    free(commit);
+    free(n);
+    free(margin);
+    free(conf);
+    free(tok);
+    return step;
+}

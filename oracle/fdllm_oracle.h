@@ -83,6 +83,29 @@ void oracle_bonus_terms(const double *c_sorted, int64_t m, double *Fn, double *B
 void oracle_profile_terms(const double *conf, const uint8_t *mask, int64_t B, int64_t L,
                           double *G, double *F, double *Bn, int32_t *order);
 
+/* Counter-based synthetic logits (the stand-in forward pass of the decode loop), bf16 bits
+ * [B, L, V] for the rows with mask != 0 (mask NULL: all rows), defined for seed s, step t,
+ * row (b, l) and index v by SplitMix64's finaliser mix (Steele, Lea, Flood 2014),
+ * G = 0x9E3779B97F4A7C15, k = mix(s ^ mix(t*G ^ mix(b << 32 | l))):
+ *   noise x_v = float(sum_j (2 u_j + 1) - 262144) * fl32(sqrt(3)/131072), u_j the four
+ *               16-bit fields of mix(k + (v+1) G)   (Irwin-Hall, unit variance)
+ *   peak       p = mix(k ^ 0xD1B54A32D192ED03): x_{p mod V} += float(p >> 40) * fl32(peak/2^24)
+ *   rounded to bf16 (nearest even). */
+void oracle_synth_block_logits(uint16_t *out, const uint8_t *mask, int64_t B, int64_t L,
+                               int64_t V, uint64_t seed, uint64_t step, double peak_max);
+
+/* Algorithm 1's outer loop on the synthetic forward pass: for each of gen_len / block_len
+ * blocks, start with the block fully masked and repeat {logits of the block's masked rows at
+ * the global step; selection (mode, param); reveal} until no position of the block is
+ * masked, or max_steps global steps were taken.  out_seq [B, gen_len] receives the
+ * committed tokens (-1 where none), out_nfe [n_blocks] the steps per block, out_margin [B]
+ * the smallest decision margin each row saw (see oracle_select_from_conf).  Returns the
+ * total number of steps. */
+int64_t oracle_decode_loop(int64_t B, int64_t gen_len, int64_t block_len, int64_t V, int mode,
+                           double param, uint64_t seed, double peak_max, int64_t max_steps,
+                           int32_t *out_seq, int32_t *out_nfe, double *out_margin,
+                           int nthreads);
+
 /* oracle_confidence followed by oracle_select_from_conf.  conf/tok are caller scratch of
  * B*L entries; they come back holding the per-position confidences and argmax tokens. */
 int64_t oracle_select(const void *logits, int dtype, int64_t B, int64_t L, int64_t V,

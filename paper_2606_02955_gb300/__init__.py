@@ -21,15 +21,20 @@ __all__ = [
     "fdllm_confidence", "fdllm_select_from_conf", "fdllm_device_status",
     "fdllm_workspace_status", "fdllm_release_workspace", "fdllm_status_string",
     "fdllm_version", "library_path", "fdllm_select_static", "fdllm_select_robust",
-    "fdllm_profile_terms", "fdllm_check_bounded_wait",
+    "fdllm_profile_terms", "fdllm_check_bounded_wait", "fdllm_decode_loop", "FORWARD_FN",
 ]
 
 BF16, FP32 = 0, 1
 PROFILE, FACTOR, THRESHOLD = 0, 1, 2
 ROW_NONFINITE, ROW_DEVICE_ERROR = -1, -2
+OK, ERR_ARG, ERR_ALIGN, ERR_NONFINITE, ERR_CUDA, ERR_WORKSPACE, ERR_DEVICE = range(7)
 MODES = {"profile": PROFILE, "factor": FACTOR, "threshold": THRESHOLD}
 
 _lib = None
+
+# fdllm_forward_fn: (user, loop_state, block_mask, logits, stream) -> int
+FORWARD_FN = ctypes.CFUNCTYPE(ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+                              ctypes.c_void_p, ctypes.c_void_p)
 
 
 def _load():
@@ -59,6 +64,9 @@ def _load():
     lib.fdllm_select_from_conf.restype = i
     lib.fdllm_profile_terms.argtypes = [p, p, i, i, p, p, p, p, p]
     lib.fdllm_profile_terms.restype = i
+    lib.fdllm_decode_loop.argtypes = [i, i, i, i, i, d, i, FORWARD_FN, p, p, p, p, i,
+                                      ctypes.POINTER(ctypes.c_int), p]
+    lib.fdllm_decode_loop.restype = i
     lib.fdllm_check_bounded_wait.argtypes = [d, p]
     lib.fdllm_check_bounded_wait.restype = i
     lib.fdllm_device_status.argtypes = [p]
@@ -289,6 +297,37 @@ def fdllm_profile_terms(conf: torch.Tensor, mask: torch.Tensor, stream=None):
                                      order.data_ptr(), _stream(stream))
     _check(st, "fdllm_profile_terms")
     return dict(G=G, F=F, B=Bn, order=order)
+
+
+def fdllm_decode_loop(forward, logits: torch.Tensor, gen_len: int, param: float, mode=PROFILE,
+                      max_steps: int | None = None, stream=None):
+    """Algorithm 1's outer loop on the GPU (fdllm_decode_loop).  ``logits`` is the
+    [B, block_len, V] buffer the forward pass fills; ``forward(loop_state_ptr,
+    block_mask_ptr, logits_ptr, stream_ptr)`` receives raw device pointers and the capture
+    stream and must only enqueue stream-ordered GPU work.  Returns (seq_tokens [B, gen_len]
+    int32, nfe_per_block int32, total steps); synchronous."""
+    B, Lb, V = logits.shape
+    nblocks = gen_len // Lb
+    dev = logits.device
+    seq = torch.empty((B, gen_len), dtype=torch.int32, device=dev)
+    nfe = torch.empty((nblocks,), dtype=torch.int32, device=dev)
+    steps = ctypes.c_int(0)
+
+    def trampoline(user, state, mask, out, strm):
+        try:
+            r = forward(state, mask, out, strm)
+            return 0 if r is None else int(r)
+        except Exception:  # reported as an argument error by the library
+            return 1
+
+    cb = FORWARD_FN(trampoline)
+    st = _load().fdllm_decode_loop(B, gen_len, Lb, V, _dtype_code(logits), float(param),
+                                   _mode(mode), cb, None, _dev(logits, "logits"),
+                                   seq.data_ptr(), nfe.data_ptr(),
+                                   int(max_steps if max_steps is not None else gen_len + 1),
+                                   ctypes.byref(steps), _stream(stream))
+    _check(st, "fdllm_decode_loop")
+    return seq, nfe, steps.value
 
 
 def fdllm_check_bounded_wait(seconds: float = 0.01, stream=None) -> int:

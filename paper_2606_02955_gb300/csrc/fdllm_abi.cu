@@ -125,9 +125,10 @@ VocabReduceArgs reduce_args(const void *logits, int dtype, int B, int L, int V,
 fdllm_status run_select(const void *logits, int dtype, int B, int L, int V, uint8_t *mask,
                         double param, int mode, int32_t *out_tokens, uint8_t *out_commit,
                         int32_t *out_n, uint8_t *ws, const Layout &lay, cudaStream_t stream,
-                        double eta = 0.0, const float *eta_pos = nullptr)
+                        double eta = 0.0, const float *eta_pos = nullptr, bool pdl = true)
 {
     VocabReduceArgs ra = reduce_args(logits, dtype, B, L, V, mask, ws, lay);
+    ra.pdl = pdl;
     if (launch_vocab_reduce(ra, esize_of(dtype), stream) != cudaSuccess)
         return FDLLM_ERR_CUDA;
     ProfileSelectArgs pa;
@@ -147,6 +148,7 @@ fdllm_status run_select(const void *logits, int dtype, int B, int L, int V, uint
     pa.out_commit = out_commit;
     pa.out_n = out_n;
     pa.status = ra.status;
+    pa.pdl = pdl;
     if (launch_profile_select(pa, stream) != cudaSuccess)
         return FDLLM_ERR_CUDA;
     return FDLLM_OK;
@@ -214,6 +216,24 @@ fdllm_status static_scratch_address(void **out)
 }
 
 }  // namespace
+
+fdllm_status select_owned(const void *logits, int dtype, int B, int L, int V, uint8_t *mask,
+                          double param, int mode, int32_t *out_tokens, uint8_t *out_commit,
+                          int32_t *out_n, cudaStream_t stream, bool pdl)
+{
+    fdllm_status st = check_select_args(logits, dtype, B, L, V, mask, param, mode, out_tokens,
+                                        out_commit, out_n);
+    if (st != FDLLM_OK)
+        return st;
+    const Layout lay = layout_for((int64_t)B * L, (int64_t)V * esize_of(dtype));
+    void *ws = nullptr;
+    st = owned_workspace(lay.total, stream, &ws);
+    if (st != FDLLM_OK)
+        return st;
+    return run_select(logits, dtype, B, L, V, mask, param, mode, out_tokens, out_commit, out_n,
+                      static_cast<uint8_t *>(ws), lay, stream, 0.0, nullptr, pdl);
+}
+
 }  // namespace fdllm
 
 using namespace fdllm;
@@ -249,18 +269,8 @@ fdllm_status fdllm_select(const void *logits, int dtype, int B, int L, int V, ui
                           double param, int mode, int32_t *out_tokens, uint8_t *out_commit,
                           int32_t *out_n, void *stream)
 {
-    fdllm_status st = check_select_args(logits, dtype, B, L, V, mask, param, mode, out_tokens,
-                                        out_commit, out_n);
-    if (st != FDLLM_OK)
-        return st;
-    const Layout lay = layout_for((int64_t)B * L, (int64_t)V * esize_of(dtype));
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
-    void *ws = nullptr;
-    st = owned_workspace(lay.total, s, &ws);
-    if (st != FDLLM_OK)
-        return st;
-    return run_select(logits, dtype, B, L, V, mask, param, mode, out_tokens, out_commit, out_n,
-                      static_cast<uint8_t *>(ws), lay, s);
+    return select_owned(logits, dtype, B, L, V, mask, param, mode, out_tokens, out_commit,
+                        out_n, static_cast<cudaStream_t>(stream), true);
 }
 
 fdllm_status fdllm_select_robust(const void *logits, int dtype, int B, int L, int V,

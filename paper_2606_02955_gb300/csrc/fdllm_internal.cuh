@@ -7,6 +7,8 @@
 #include <cstddef>
 #include <cstdint>
 
+#include "fdllm.h"
+
 namespace fdllm {
 
 // ------------------------------------------------------------------ vocab reduction (a1)
@@ -44,6 +46,7 @@ struct VocabReduceArgs {
     uint32_t *next_unit;     // work queue past the first gridDim.x units: zero on entry,
                              // reset by the consumer kernel
     uint32_t *status;        // sticky device error bits
+    bool pdl = true;         // launch as a programmatic dependent of the previous kernel
 };
 
 struct UnitPlan {
@@ -115,9 +118,17 @@ struct ProfileSelectArgs {
     uint8_t *out_commit;     // [B, L]
     int32_t *out_n;          // [B]
     const uint32_t *status;  // nullable: nonzero -> every row reports a device error
+    bool pdl = true;         // with partials: launch as a programmatic dependent
 };
 
 cudaError_t launch_profile_select(const ProfileSelectArgs &a, cudaStream_t stream);
+
+// fdllm_select on the library-owned workspace, with programmatic dependent launches
+// switched on or off (the decode loop's graph body falls back to plain stream order where
+// the driver does not accept programmatic edges inside a conditional node).
+fdllm_status select_owned(const void *logits, int dtype, int B, int L, int V, uint8_t *mask,
+                          double param, int mode, int32_t *out_tokens, uint8_t *out_commit,
+                          int32_t *out_n, cudaStream_t stream, bool pdl);
 
 struct ProfileTermsArgs {
     const float *conf;       // [B, L]

@@ -250,7 +250,7 @@ cudaError_t launch_t(const ProfileSelectArgs &a, cudaStream_t stream)
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = a.partials != nullptr ? 1 : 0;  // a dependent of the vocab reduction
+    cfg.numAttrs = a.partials != nullptr && a.pdl ? 1 : 0;  // a dependent of the reduction
     return cudaLaunchKernelEx(&cfg, profile_select_kernel<T>, a);
 }
 

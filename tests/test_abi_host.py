@@ -118,3 +118,26 @@ def test_select_robust_rejects(lib):
     assert f(float("inf")) == ERR_ARG
     assert f(0.1, B=0) == ERR_ARG
     assert f(0.1, logits=A2) == ERR_ALIGN
+
+
+def test_decode_loop_rejects_before_any_device_call(lib):
+    p, i, d = ctypes.c_void_p, ctypes.c_int, ctypes.c_double
+    fwd_t = ctypes.CFUNCTYPE(i, p, p, p, p, p)
+    calls = []
+    fwd = fwd_t(lambda *a: calls.append(a) or 0)
+    lib.fdllm_decode_loop.argtypes = [i, i, i, i, i, d, i, fwd_t, p, p, p, p, i,
+                                      ctypes.POINTER(i), p]
+    steps = ctypes.c_int(-5)
+
+    def f(B=2, gen=64, Lb=32, mode=0, forward=fwd, logits=A16, max_steps=100):
+        return lib.fdllm_decode_loop(B, gen, Lb, 1024, 0, 1.0, mode, forward, None, logits,
+                                     A16, A16, max_steps, ctypes.byref(steps), None)
+    assert f(gen=48) == ERR_ARG                   # gen_len not a multiple of block_len
+    assert f(gen=16) == ERR_ARG                   # gen_len < block_len
+    assert f(Lb=2048, gen=4096) == ERR_ARG        # block_len > 1024
+    assert f(B=0) == ERR_ARG
+    assert f(mode=3) == ERR_ARG                   # the robust rule is not a loop mode
+    assert f(max_steps=0) == ERR_ARG
+    assert f(forward=fwd_t()) == ERR_ARG          # null forward pass
+    assert f(logits=None) == ERR_ARG
+    assert not calls and steps.value == -5
