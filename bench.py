@@ -469,12 +469,133 @@ def run_decode_loop(args) -> dict:
         "B": B, "gen_len": gen, "block_len": Lb, "V": V, "dtype": "bf16",
         "mode": args.mode, "param": args.param, "peak": peak, "data": "synthetic",
         "steps": int(steps_d), "nfe_per_block": [int(x) for x in nfe_d.cpu().numpy()],
+        "tokens_per_step": gen / max(int(steps_d), 1),
         "device_loop": {"ms_per_generation": dms, "tokens_per_s": tokens / (dms * 1e-3),
                         "ms_per_step": dms / max(steps_d, 1)},
         "host_loop": {"ms_per_generation": hms, "tokens_per_s": tokens / (hms * 1e-3),
                       "ms_per_step": hms / max(steps_hh, 1)},
         "host_round_trip_us_per_step": 1e3 * (hms - dms) / max(steps_d, 1),
         "identical_decisions": identical, "repeats": args.repeats,
+    }
+
+
+def run_lmhead(args) -> dict:
+    """Step a1 fused into the LM head (fdllm_lmhead_select: a tcgen05 GEMM whose epilogue
+    reduces the logits) against two unfused paths on the same inputs: our GEMM storing fp32
+    logits then fdllm_select, and cuBLAS (torch.matmul, bf16 logits for all B*L rows) then
+    fdllm_select.  LLaDA-8B head shape (H = 4096, V = 126464), the serving batch's masks.
+    Each variant runs as CUDA-graph replays timed with events; the mask is restored from a
+    saved copy before each step.  W (1.04 GB) exceeds L2, so every step reads it from HBM."""
+    import numpy as np
+    import torch
+
+    import fdllm_synth as syn
+    import paper_2606_02955_gb300 as fd
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    wl = syn.WORKLOADS["serving_b64_l32_bf16"]
+    B, L, H, V = wl.B, wl.L, syn.LLADA_HIDDEN, syn.LLADA_VOCAB
+    hidden, w, _ = syn.make_lmhead_inputs(B, L, H, V, seed=1234, device=dev)
+    mask0_np = syn.make_mask(wl, seed=1234)
+    R = int(mask0_np.sum())
+    mask0 = torch.from_numpy(mask0_np).to(dev)
+    mask = mask0.clone()
+    mode = fd.MODES[args.mode]
+    tok = torch.full((B, L), -1, dtype=torch.int32, device=dev)
+    commit = torch.empty((B, L), dtype=torch.uint8, device=dev)
+    n_out = torch.empty((B,), dtype=torch.int32, device=dev)
+    logits32 = torch.empty((B, L, V), dtype=torch.float32, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def fused():
+        mask.copy_(mask0, non_blocking=True)
+        fd.fdllm_lmhead_select(hidden, w, mask, args.param, mode, tok, commit, n_out,
+                               stream=stream)
+
+    def ours_unfused():
+        mask.copy_(mask0, non_blocking=True)
+        fd.fdllm_lmhead_logits(hidden, w, mask, logits32, stream=stream)
+        fd.fdllm_select(logits32, mask, args.param, mode, tok, commit, n_out, stream=stream)
+
+    def cublas_unfused():
+        mask.copy_(mask0, non_blocking=True)
+        x = torch.matmul(hidden.view(B * L, H), w.t()).view(B, L, V)
+        fd.fdllm_select(x, mask, args.param, mode, tok, commit, n_out, stream=stream)
+
+    def gemm_only():
+        fd.fdllm_lmhead_confidence(hidden, w, mask0, stream=stream)
+
+    reps = max(3, args.lmhead_steps)
+
+    def time_variant(fn):
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                fn()
+        stream.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            fn()
+        for _ in range(max(3, args.warmup // 4)):
+            g.replay()
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        with torch.cuda.stream(stream):
+            for _ in range(reps):
+                g.replay()
+        e1.record(stream)
+        e1.synchronize()
+        return e0.elapsed_time(e1) / reps
+
+    sampler = ClockSampler(0).start()
+    tw0 = time.time()
+    t_fused = time_variant(fused)
+    t_gemm = time_variant(gemm_only)
+    t_ours = time_variant(ours_unfused)
+    t_cublas = time_variant(cublas_unfused)
+    tw1 = time.time()
+    time.sleep(0.12)
+    sampler.stop()
+
+    # the fused path and the unfused ones take the same decisions on these inputs
+    res = {}
+    for name, fn in (("fused", fused), ("ours_unfused", ours_unfused)):
+        with torch.cuda.stream(stream):
+            fn()
+        stream.synchronize()
+        res[name] = (n_out.clone(), commit.clone())
+    same = bool(torch.equal(res["fused"][0], res["ours_unfused"][0]) and
+                torch.equal(res["fused"][1], res["ours_unfused"][1]))
+
+    flops = 2.0 * R * H * V
+    peaks = {}
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            peaks = json.load(f)
+    except OSError:
+        pass
+    peak = float(peaks.get("bf16_tflops", 1900.0))
+    achieved = flops / (t_gemm * 1e-3) / 1e12
+    return {
+        "metric": "LM head + commit-set selection: ms per step and GEMM TFLOP/s",
+        "workload": "lmhead_b%d_l%d_h%d_v%d_bf16" % (B, L, H, V),
+        "B": B, "L": L, "H": H, "V": V, "masked_rows": R, "mode": args.mode,
+        "param": args.param, "data": "synthetic",
+        "ms_per_step": {"fused": t_fused, "ours_gemm_store_then_select": t_ours,
+                        "cublas_bf16_logits_then_select": t_cublas,
+                        "fused_confidence_only": t_gemm},
+        "selections_per_s_fused": B / (t_fused * 1e-3),
+        "speedup_vs_cublas_unfused": t_cublas / t_fused,
+        "identical_decisions_fused_vs_unfused": same,
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak, "kernel": "fdllm_lmhead_confidence (compaction, "
+                     "gather, GEMM with reducing epilogue, combine)",
+                     "algorithmic_flops_per_launch": flops,
+                     "peak_source": "measured" if "bf16_tflops" in peaks else "fallback"},
+        "clocks": sampler.summary(tw0, tw1),
+        "steps": reps,
     }
 
 
@@ -590,7 +711,14 @@ def main(argv=None):
                     help="decode loop: largest planted logit height of the synthetic forward")
     ap.add_argument("--repeats", type=int, default=5)
     ap.add_argument("--warmup-loops", type=int, default=2)
+    ap.add_argument("--lmhead", action="store_true",
+                    help="time the LM-head-fused selection against unfused paths, instead of "
+                         "the throughput line")
+    ap.add_argument("--lmhead-steps", type=int, default=50)
     args = ap.parse_args(argv)
+    if args.lmhead:
+        print(json.dumps(run_lmhead(args)), flush=True)
+        return
     if args.decode_loop:
         print(json.dumps(run_decode_loop(args)), flush=True)
         return

@@ -192,6 +192,31 @@ def host_bits(logits: torch.Tensor) -> np.ndarray:
     raise TypeError(t.dtype)
 
 
+# ----------------------------------------------------------------------------- LM head
+LLADA_HIDDEN = 4096
+
+
+def make_lmhead_inputs(B: int, L: int, H: int, V: int, seed: int, beta_lo: float = 0.0,
+                       beta_hi: float = 20.0, device="cpu"):
+    """Seeded LM-head inputs (bf16): W [V, H] with N(0, 1/H) entries (rows of norm ~1), and
+    per position a target token t ~ U{0..V-1}, a height beta ~ U[beta_lo, beta_hi] and
+    hidden h = z + beta w_t / |w_t|^2 with z ~ N(0, I_H).  Then w_t . h ~ beta + N(0, 1) and
+    w_v . h ~ N(0, 1 + beta^2 / H) for v != t (N(0, ~1) at H = 4096): a planted peak of height
+    beta in logit space, as in the logits recipes.  Returns (hidden [B, L, H], w [V, H], targets [B, L])."""
+    dev = torch.device(device)
+    g = torch.Generator(device=dev)
+    g.manual_seed(int(seed) * 7919 + 17)
+    w = torch.randn((V, H), generator=g, device=dev, dtype=torch.float32)
+    w.mul_(1.0 / math.sqrt(H))
+    t = torch.randint(0, V, (B, L), generator=g, device=dev)
+    beta = torch.rand((B, L), generator=g, device=dev, dtype=torch.float32)
+    beta = beta * (beta_hi - beta_lo) + beta_lo
+    h = torch.randn((B, L, H), generator=g, device=dev, dtype=torch.float32)
+    wt = w[t]
+    h += beta[..., None] * wt / (wt * wt).sum(-1, keepdim=True)
+    return h.to(torch.bfloat16), w.to(torch.bfloat16), t
+
+
 # ----------------------------------------------------------------------------- GPU stand-in
 # Counter-based synthetic logits on the GPU (fdllm_synth_cuda.cu): the forward pass of the
 # decode-loop tests and benchmarks.  The CPU oracle implements the same generator itself.

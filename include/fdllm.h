@@ -176,6 +176,39 @@ fdllm_status fdllm_select_from_conf(const float *conf, const int32_t *argmax, in
                                     int32_t *out_tokens, uint8_t *out_commit, int32_t *out_n,
                                     void *stream);
 
+/* Step a1 fused with the LM head (the projection that produces the logits, Sec. 3
+ * "Notation": p_i = softmax of the logits of position i), then steps a2-a5 as in
+ * fdllm_select.  For every masked position the logits x = W h are computed on the tensor
+ * cores (bf16 inputs, fp32 accumulation) and reduced to (c, x_hat) in the GEMM's epilogue:
+ * the B*L*V logits are never written to memory.
+ *   hidden   [B, L, H] bf16 device, the final hidden state of each position (read at masked
+ *            positions only); 16-byte aligned.
+ *   w_vocab  [V, H] bf16 device, the vocabulary projection, row v = the weights of token v;
+ *            16-byte aligned.
+ *   H        hidden size, a multiple of 8 (16-byte rows); V >= 1, any value.
+ * mask, param, mode and the outputs as in fdllm_select (B*L <= FDLLM_MAX_ROWS, L <=
+ * FDLLM_MAX_L).  Uses the library-owned workspace (B*L*(2H + 16*ceil(V/256) + 12) bytes
+ * and a header), allocated outside the step as for fdllm_select.  Asynchronous on `stream`.
+ * Results agree with fdllm_select applied to the fp32 logits fdllm_lmhead_logits writes
+ * (the same tensor-core accumulation): tokens bit-exact, confidences within 1e-5. */
+fdllm_status fdllm_lmhead_select(const void *hidden, const void *w_vocab, int B, int L, int H,
+                                 int V, uint8_t *mask, double param, int mode,
+                                 int32_t *out_tokens, uint8_t *out_commit, int32_t *out_n,
+                                 void *stream);
+
+/* Step a1 alone on the LM head: out_conf (fp32) and out_argmax (int32), [B, L] device, written
+ * at masked positions (NaN and -1 for a row whose logits hold a NaN or an infinite maximum).
+ * Arguments as fdllm_lmhead_select. */
+fdllm_status fdllm_lmhead_confidence(const void *hidden, const void *w_vocab, int B, int L,
+                                     int H, int V, const uint8_t *mask, float *out_conf,
+                                     int32_t *out_argmax, void *stream);
+
+/* The same tensor-core GEMM with its accumulators stored instead of reduced: out_logits
+ * [B, L, V] fp32 device, written at the masked positions' rows only (the unfused path, and
+ * the exact inputs against which the fused reduction is checked). */
+fdllm_status fdllm_lmhead_logits(const void *hidden, const void *w_vocab, int B, int L, int H,
+                                 int V, const uint8_t *mask, float *out_logits, void *stream);
+
 /* Model forward pass used by fdllm_decode_loop.  It must only enqueue stream-ordered GPU
  * work on `stream`: it is called while the loop body is being captured into a CUDA graph
  * (once, or twice when the driver rejects the first capture and the body is captured again

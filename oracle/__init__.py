@@ -23,7 +23,7 @@ import threading
 import numpy as np
 
 PROFILE, FACTOR, THRESHOLD = 0, 1, 2
-BF16, FP32 = 0, 1
+BF16, FP32, F64 = 0, 1, 2
 
 HERE = os.path.dirname(os.path.abspath(__file__))
 SOURCE = os.path.join(HERE, "fdllm_oracle.c")
@@ -63,13 +63,16 @@ def _ptr(a: np.ndarray) -> int:
 
 
 def _logits_view(logits: np.ndarray):
-    """Accept fp32 arrays or bf16 given as raw uint16 bits; return (array, dtype code)."""
+    """Accept fp32 or fp64 arrays, or bf16 given as raw uint16 bits; return (array, code)."""
     a = np.ascontiguousarray(logits)
     if a.dtype == np.uint16:
         return a, BF16
     if a.dtype == np.float32:
         return a, FP32
-    raise TypeError("oracle logits must be float32 or uint16 (bf16 bits), got %s" % a.dtype)
+    if a.dtype == np.float64:
+        return a, F64
+    raise TypeError("oracle logits must be float32, float64 or uint16 (bf16 bits), got %s"
+                    % a.dtype)
 
 
 class Oracle:
@@ -95,6 +98,8 @@ class Oracle:
         lib.oracle_synth_block_logits.restype = None
         lib.oracle_decode_loop.argtypes = [i64, i64, i64, i64, i32, d, u64, d, i64, p, p, p, i32]
         lib.oracle_decode_loop.restype = i64
+        lib.oracle_lmhead_logits.argtypes = [p, p, i64, i64, i64, p, p, p, i32]
+        lib.oracle_lmhead_logits.restype = None
         self.lib = lib
         self.path = lib_path
 
@@ -137,6 +142,24 @@ class Oracle:
         self.lib.oracle_profile_terms(_ptr(c), _ptr(m), B, L, _ptr(G), _ptr(F), _ptr(Bn),
                                       _ptr(order))
         return dict(G=G, F=F, B=Bn, order=order)
+
+    def lmhead_logits(self, hidden_bits: np.ndarray, w_bits: np.ndarray, mask=None,
+                      with_abs: bool = False, nthreads: int = 1):
+        """Exact (fp64) logits of the LM head at masked rows: hidden [B, L, H] and w [V, H]
+        as bf16 bits (uint16).  Returns logits [B, L, V] (zero at unmasked rows) and, with
+        with_abs, the magnitudes sum_k |h_k w_vk| of the same shape."""
+        h = np.ascontiguousarray(hidden_bits, np.uint16)
+        w = np.ascontiguousarray(w_bits, np.uint16)
+        B, L, H = h.shape
+        V = w.shape[0]
+        assert w.shape == (V, H)
+        m = None if mask is None else np.ascontiguousarray(mask, np.uint8).reshape(B, L)
+        out = np.zeros((B, L, V), np.float64)
+        mag = np.zeros((B, L, V), np.float64) if with_abs else None
+        self.lib.oracle_lmhead_logits(_ptr(h), _ptr(w), B * L, H, V,
+                                      None if m is None else _ptr(m), _ptr(out),
+                                      None if mag is None else _ptr(mag), int(nthreads))
+        return (out, mag) if with_abs else out
 
     def synth_block_logits(self, B, L, V, seed, step, peak_max, mask=None):
         """Counter-based synthetic bf16 logits (uint16 bits [B, L, V]); unmasked rows zero."""

@@ -19,16 +19,26 @@
 #endif
 
 /* One logit widened to double.  bf16 is the upper half of an IEEE fp32 word, so the
- * widening is exact. */
+ * widening is exact; fp64 logits (the LM head's exact products) are taken as they are. */
 static double logit_at(const void *logits, int dtype, int64_t i)
 {
     float f;
+    if (dtype == ORACLE_F64)
+        return ((const double *)logits)[i];
     if (dtype == ORACLE_BF16) {
         uint32_t u = (uint32_t)((const uint16_t *)logits)[i] << 16;
         memcpy(&f, &u, sizeof f);
     } else {
         f = ((const float *)logits)[i];
     }
+    return (double)f;
+}
+
+static double bf16_to_double(uint16_t b)
+{
+    float f;
+    uint32_t u = (uint32_t)b << 16;
+    memcpy(&f, &u, sizeof f);
     return (double)f;
 }
 
@@ -497,4 +507,33 @@ int64_t oracle_decode_loop(int64_t B, int64_t gen_len, int64_t block_len, int64_
     free(conf);
     free(tok);
     return step;
+}
+
+void oracle_lmhead_logits(const uint16_t *hidden, const uint16_t *w, int64_t rows, int64_t H,
+                          int64_t V, const uint8_t *mask, double *out, double *out_abs,
+                          int nthreads)
+{
+    int64_t r;
+#ifdef _OPENMP
+#pragma omp parallel for schedule(dynamic, 1) num_threads(nthreads > 1 ? nthreads : 1)
+#endif
+    for (r = 0; r < rows; ++r) {
+        if (mask && !mask[r])
+            continue;
+        double *h = (double *)malloc((size_t)H * sizeof(double));
+        for (int64_t k = 0; k < H; ++k)
+            h[k] = bf16_to_double(hidden[r * H + k]);
+        for (int64_t v = 0; v < V; ++v) {
+            double sum = 0.0, mag = 0.0;
+            for (int64_t k = 0; k < H; ++k) {
+                const double t = h[k] * bf16_to_double(w[v * H + k]);
+                sum += t;
+                mag += fabs(t);
+            }
+            out[r * V + v] = sum;
+            if (out_abs)
+                out_abs[r * V + v] = mag;
+        }
+        free(h);
+    }
 }

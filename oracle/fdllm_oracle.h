@@ -26,7 +26,7 @@
 extern "C" {
 #endif
 
-enum { ORACLE_BF16 = 0, ORACLE_FP32 = 1 };
+enum { ORACLE_BF16 = 0, ORACLE_FP32 = 1, ORACLE_F64 = 2 };
 enum { ORACLE_PROFILE = 0, ORACLE_FACTOR = 1, ORACLE_THRESHOLD = 2 };
 
 /* Per masked position (b,l): x_hat = lowest v attaining max_v logit, c = max_v softmax(v)
@@ -112,6 +112,16 @@ int64_t oracle_select(const void *logits, int dtype, int64_t B, int64_t L, int64
                       uint8_t *mask, int mode, double param, int32_t *out_tokens,
                       uint8_t *out_commit, int32_t *out_n, double *margin, double *conf,
                       int32_t *tok, int nthreads);
+
+/* The LM head that produces the logits (Sec. 3 "Notation": p_i is the softmax of the logits
+ * of position i): for every masked row r, out[r][v] = sum_k hidden[r][k] * w[v][k], summed in
+ * k order in double precision from the bf16 inputs (raw uint16 bits, widened exactly), and,
+ * when out_abs is not NULL, out_abs[r][v] = sum_k |hidden[r][k] * w[v][k]| (the scale of the
+ * rounding error of any fp32 evaluation of the same sum).  Unmasked rows are not written.
+ * hidden [rows][H], w [V][H], out and out_abs [rows][V]. */
+void oracle_lmhead_logits(const uint16_t *hidden, const uint16_t *w, int64_t rows, int64_t H,
+                          int64_t V, const uint8_t *mask, double *out, double *out_abs,
+                          int nthreads);
 
 #ifdef __cplusplus
 }

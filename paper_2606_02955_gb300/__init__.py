@@ -22,6 +22,7 @@ __all__ = [
     "fdllm_workspace_status", "fdllm_release_workspace", "fdllm_status_string",
     "fdllm_version", "library_path", "fdllm_select_static", "fdllm_select_robust",
     "fdllm_profile_terms", "fdllm_check_bounded_wait", "fdllm_decode_loop", "FORWARD_FN",
+    "fdllm_lmhead_select", "fdllm_lmhead_confidence", "fdllm_lmhead_logits",
 ]
 
 BF16, FP32 = 0, 1
@@ -58,6 +59,12 @@ def _load():
     lib.fdllm_select_static.restype = i
     lib.fdllm_workspace_bytes.argtypes = [i, i, i, i]
     lib.fdllm_workspace_bytes.restype = sz
+    lib.fdllm_lmhead_select.argtypes = [p, p, i, i, i, i, p, d, i, p, p, p, p]
+    lib.fdllm_lmhead_select.restype = i
+    lib.fdllm_lmhead_confidence.argtypes = [p, p, i, i, i, i, p, p, p, p]
+    lib.fdllm_lmhead_confidence.restype = i
+    lib.fdllm_lmhead_logits.argtypes = [p, p, i, i, i, i, p, p, p]
+    lib.fdllm_lmhead_logits.restype = i
     lib.fdllm_confidence.argtypes = [p, i, i, i, i, p, p, p, p]
     lib.fdllm_confidence.restype = i
     lib.fdllm_select_from_conf.argtypes = [p, p, i, i, p, d, i, p, p, p, p]
@@ -265,6 +272,65 @@ def fdllm_confidence(logits: torch.Tensor, mask: torch.Tensor, out_conf=None, ou
                                _stream(stream))
     _check(st, "fdllm_confidence")
     return out_conf, out_argmax
+
+
+def _lmhead_shapes(hidden: torch.Tensor, w_vocab: torch.Tensor):
+    B, L, H = hidden.shape
+    V, H2 = w_vocab.shape
+    if H2 != H:
+        raise ValueError("w_vocab must be [V, %d], got %s" % (H, tuple(w_vocab.shape)))
+    hp = _dev(hidden, "hidden", torch.bfloat16)
+    wp = _dev(w_vocab, "w_vocab", torch.bfloat16)
+    return B, L, H, V, hp, wp
+
+
+def fdllm_lmhead_select(hidden: torch.Tensor, w_vocab: torch.Tensor, mask: torch.Tensor,
+                        param: float, mode=PROFILE, out_tokens=None, out_commit=None, out_n=None,
+                        stream=None):
+    """One selection step with the logits computed and reduced inside the LM-head GEMM
+    (fdllm_lmhead_select): ``hidden`` [B, L, H] bf16, ``w_vocab`` [V, H] bf16, ``mask``
+    [B, L] uint8 (updated in place).  Returns (out_tokens, out_commit, out_n)."""
+    B, L, H, V, hp, wp = _lmhead_shapes(hidden, w_vocab)
+    out_tokens, out_commit, out_n = _outputs(B, L, hidden.device, out_tokens, out_commit, out_n)
+    st = _load().fdllm_lmhead_select(hp, wp, B, L, H, V, _dev(mask, "mask", torch.uint8, (B, L)),
+                                     float(param), _mode(mode),
+                                     _dev(out_tokens, "out_tokens", torch.int32, (B, L)),
+                                     _dev(out_commit, "out_commit", torch.uint8, (B, L)),
+                                     _dev(out_n, "out_n", torch.int32, (B,)), _stream(stream))
+    _check(st, "fdllm_lmhead_select")
+    return out_tokens, out_commit, out_n
+
+
+def fdllm_lmhead_confidence(hidden: torch.Tensor, w_vocab: torch.Tensor, mask: torch.Tensor,
+                            out_conf=None, out_argmax=None, stream=None):
+    """Step a1 on the LM head: (conf fp32 [B, L], argmax int32 [B, L]) at masked positions."""
+    B, L, H, V, hp, wp = _lmhead_shapes(hidden, w_vocab)
+    if out_conf is None:
+        out_conf = torch.full((B, L), float("nan"), dtype=torch.float32, device=hidden.device)
+    if out_argmax is None:
+        out_argmax = torch.full((B, L), -1, dtype=torch.int32, device=hidden.device)
+    st = _load().fdllm_lmhead_confidence(hp, wp, B, L, H, V,
+                                         _dev(mask, "mask", torch.uint8, (B, L)),
+                                         _dev(out_conf, "out_conf", torch.float32, (B, L)),
+                                         _dev(out_argmax, "out_argmax", torch.int32, (B, L)),
+                                         _stream(stream))
+    _check(st, "fdllm_lmhead_confidence")
+    return out_conf, out_argmax
+
+
+def fdllm_lmhead_logits(hidden: torch.Tensor, w_vocab: torch.Tensor, mask: torch.Tensor,
+                        out_logits=None, stream=None):
+    """The LM-head GEMM's fp32 logits [B, L, V] at masked rows (other rows untouched; a
+    freshly allocated output holds NaN there)."""
+    B, L, H, V, hp, wp = _lmhead_shapes(hidden, w_vocab)
+    if out_logits is None:
+        out_logits = torch.full((B, L, V), float("nan"), dtype=torch.float32,
+                                device=hidden.device)
+    st = _load().fdllm_lmhead_logits(hp, wp, B, L, H, V, _dev(mask, "mask", torch.uint8, (B, L)),
+                                     _dev(out_logits, "out_logits", torch.float32, (B, L, V)),
+                                     _stream(stream))
+    _check(st, "fdllm_lmhead_logits")
+    return out_logits
 
 
 def fdllm_select_from_conf(conf: torch.Tensor, argmax: torch.Tensor, mask: torch.Tensor,

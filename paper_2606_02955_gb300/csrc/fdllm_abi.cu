@@ -76,6 +76,8 @@ constexpr int kMaxDevices = 64;
 OwnedWorkspace g_ws[kMaxDevices];
 std::mutex g_ws_mutex;
 
+}  // namespace
+
 fdllm_status owned_workspace(size_t need, cudaStream_t stream, void **out)
 {
     int dev = 0;
@@ -104,6 +106,8 @@ fdllm_status owned_workspace(size_t need, cudaStream_t stream, void **out)
     *out = w.ptr;
     return FDLLM_OK;
 }
+
+namespace {
 
 VocabReduceArgs reduce_args(const void *logits, int dtype, int B, int L, int V,
                             const uint8_t *mask, uint8_t *ws, const Layout &lay)

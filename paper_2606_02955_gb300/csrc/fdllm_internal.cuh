@@ -123,6 +123,12 @@ struct ProfileSelectArgs {
 
 cudaError_t launch_profile_select(const ProfileSelectArgs &a, cudaStream_t stream);
 
+// The library-owned workspace of the current device, grown on demand and zero-filled when
+// allocated.  Every user shares its 256-byte header: the sticky status word at offset 0 and
+// the vocab reduction's work counter at 4 (zero between calls); the LM-head path keeps its
+// compact row count at 8.
+fdllm_status owned_workspace(size_t need, cudaStream_t stream, void **out);
+
 // fdllm_select on the library-owned workspace, with programmatic dependent launches
 // switched on or off (the decode loop's graph body falls back to plain stream order where
 // the driver does not accept programmatic edges inside a conditional node).

@@ -1,0 +1,660 @@
+// lmhead.cu -- step a1 fused with the LM head that produces the logits.  The logits of a
+// masked position are x = W h (h its final hidden state [H], W the vocabulary projection
+// [V, H]); instead of writing B*L*V logits and reading them back, a tcgen05 GEMM reduces
+// each 128 x 256 accumulator tile in its epilogue to one (max, sum of exp, first argmax)
+// partial per row, straight from tensor memory.
+//
+// Launch sequence on one stream (all rows of one step):
+//   1. compact_rows_kernel   the masked rows' indices and their count (one CTA)
+//   2. gather_rows_kernel    the masked rows' hidden states, packed [R, H] (TMA-friendly)
+//   3. lmhead_gemm_kernel    persistent tcgen05 GEMM: warp 0 issues TMA loads into a 4-stage
+//                            ring, warp 1 issues tcgen05.mma into one of two TMEM
+//                            accumulators, warps 2-5 reduce (or store) the other one
+//   4. combine_rows_kernel   one warp per row folds its V/256 tile partials in a fixed order
+//   5. profile_select        steps a2-a5 on the confidences (profile_select.cu)
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+#include <mutex>
+
+#include "fdllm.h"
+#include "fdllm_internal.cuh"
+#include "ptx.cuh"
+#include "tcgen05.cuh"
+
+namespace fdllm {
+namespace {
+
+constexpr int BM = 128;  // rows per tile (TMEM lanes)
+constexpr int BN = 256;  // vocabulary entries per tile (fp32 TMEM columns per accumulator)
+constexpr int BK = 64;   // hidden elements per stage: one 128-byte swizzle row of bf16
+constexpr int kStages = 4;
+constexpr int kABytes = BM * BK * 2;
+constexpr int kBBytes = BN * BK * 2;
+constexpr int kStageBytes = kABytes + kBBytes;
+constexpr int kThreads = 192;           // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
+constexpr uint32_t kTmemCols = 2 * BN;  // two accumulators
+constexpr size_t kBarrierBytes = 256;
+constexpr size_t kSmemBytes = 1024 + (size_t)kStages * kStageBytes + kBarrierBytes;
+constexpr uint64_t kDrainLimitNs = 100000000ull;  // waits for own copies after an abort
+
+enum Epilogue { kReduce = 0, kStore = 1 };
+
+struct GemmArgs {
+    const int32_t *row_count;  // R, written by compact_rows_kernel
+    const int32_t *row_ids;    // [R] global row (b * L + l) of each packed row
+    int32_t V;
+    int32_t n_tiles;           // ceil(V / BN)
+    int32_t k_blocks;          // ceil(H / BK)
+    UnitPartial *partials;     // kReduce: [R][n_tiles]
+    float *logits;             // kStore: [B * L][V] fp32, written at masked rows
+    uint32_t *status;          // sticky device error bits
+};
+
+// A bounded wait that also gives up as soon as another role of the CTA has given up.
+__device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity, uint32_t *status,
+                                              volatile int *abort_flag)
+{
+    if (mbar_try_wait(bar, parity))
+        return true;
+    const uint64_t t0 = global_timer_ns();
+    for (uint32_t it = 1;; ++it) {
+        if (mbar_try_wait(bar, parity))
+            return true;
+        if ((it & 63u) == 0) {
+            if (*abort_flag)
+                return false;
+            if (global_timer_ns() - t0 > kWaitLimitNs) {
+                atomicOr(status, kDevStatTimeout);
+                *abort_flag = 1;
+                return false;
+            }
+        }
+    }
+}
+
+template <int EPI>
+__global__ void __launch_bounds__(kThreads, 1)
+    lmhead_gemm_kernel(const __grid_constant__ CUtensorMap map_h,
+                       const __grid_constant__ CUtensorMap map_w, const GemmArgs a)
+{
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *sA = smem;                     // kStages x [BM rows][128 B], 128-byte swizzled
+    uint8_t *sB = smem + kStages * kABytes; // kStages x [BN rows][128 B]
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sB + kStages * kBBytes);
+    uint64_t *full = bars;                  // TMA -> MMA, one per stage
+    uint64_t *empty = bars + kStages;       // MMA -> TMA, one per stage
+    uint64_t *tfull = bars + 2 * kStages;   // MMA -> epilogue, one per accumulator
+    uint64_t *tempty = tfull + 2;           // epilogue -> MMA, one per accumulator
+    uint64_t *done = tempty + 2;            // MMA thread: all its MMAs have completed
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 1);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&tfull[i], 1);
+            mbar_init(&tempty[i], 4);  // one arrival per epilogue warp
+        }
+        mbar_init(done, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+        tc::prefetch_tensormap(&map_h);
+        tc::prefetch_tensormap(&map_w);
+    }
+    if (warp == 1)
+        tc::tmem_alloc(tmem_slot, kTmemCols);
+    tc::fence_before_sync();
+    __syncthreads();
+    tc::fence_after_sync();
+    const uint32_t tmem_base = *tmem_slot;
+
+    const int R = *a.row_count;
+    const int num_m = (R + BM - 1) / BM;
+    const int64_t total = (int64_t)num_m * a.n_tiles;
+    // Tile t covers packed rows [m*BM, +BM) x vocabulary [n*BN, +BN) with m fastest, so the
+    // CTAs working at the same time share few W tiles (read from HBM once, then from L2).
+
+    if (warp == 0) {
+        if (lane == 0) {
+            int s = 0;
+            uint32_t ph = 0;
+            uint32_t last_ph[kStages];
+            bool used[kStages];
+            for (int i = 0; i < kStages; ++i)
+                used[i] = false;
+            bool ok = true;
+            for (int64_t t = blockIdx.x; ok && t < total; t += gridDim.x) {
+                const int m = (int)(t % num_m), n = (int)(t / num_m);
+                for (int kb = 0; kb < a.k_blocks; ++kb) {
+                    if (!wait_or_abort(&empty[s], ph ^ 1u, a.status, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(&full[s], kStageBytes);
+                    tc::tma_load_2d(sA + s * kABytes, &map_h, kb * BK, m * BM, &full[s]);
+                    tc::tma_load_2d(sB + s * kBBytes, &map_w, kb * BK, n * BN, &full[s]);
+                    used[s] = true;
+                    last_ph[s] = ph;
+                    if (++s == kStages) {
+                        s = 0;
+                        ph ^= 1u;
+                    }
+                }
+            }
+            // No copy of this CTA may still be in flight when it exits.
+            for (int i = 0; i < kStages; ++i)
+                if (used[i])
+                    mbar_wait(&full[i], last_ph[i], a.status, kDrainLimitNs);
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idesc = tc::idesc_bf16_f32(BM, BN);
+            int s = 0;
+            uint32_t ph = 0;
+            bool ok = true;
+            int i = 0;
+            for (int64_t t = blockIdx.x; ok && t < total; t += gridDim.x, ++i) {
+                const int acc = i & 1;
+                const uint32_t aph = (uint32_t)(i >> 1) & 1u;
+                if (!wait_or_abort(&tempty[acc], aph ^ 1u, a.status, abort_flag))
+                    break;
+                tc::fence_after_sync();
+                const uint32_t d = tmem_base + (uint32_t)(acc * BN);
+                for (int kb = 0; kb < a.k_blocks; ++kb) {
+                    if (!wait_or_abort(&full[s], ph, a.status, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    tc::fence_after_sync();
+                    const uint64_t ad = tc::sw128_kmajor_desc(sA + s * kABytes);
+                    const uint64_t bd = tc::sw128_kmajor_desc(sB + s * kBBytes);
+#pragma unroll
+                    for (int k = 0; k < BK / 16; ++k)  // K = 16 per MMA: +32 B in the row
+                        tc::mma_bf16(d, ad + 2u * k, bd + 2u * k, idesc, (kb | k) != 0);
+                    tc::commit(&empty[s]);  // the stage is free once these MMAs have read it
+                    if (++s == kStages) {
+                        s = 0;
+                        ph ^= 1u;
+                    }
+                }
+                if (ok)
+                    tc::commit(&tfull[acc]);
+            }
+            // Tensor memory is freed below only after every MMA issued here has completed.
+            tc::commit(done);
+            mbar_wait(done, 0, a.status, kDrainLimitNs);
+        }
+        __syncwarp();
+    } else {
+        // Epilogue: warp w reads TMEM lanes [32 (w % 4), +32): thread = one row of the tile.
+        const int quarter = warp & 3;
+        const int row_in_tile = quarter * 32 + lane;
+        int i = 0;
+        for (int64_t t = blockIdx.x; t < total; t += gridDim.x, ++i) {
+            const int acc = i & 1;
+            const uint32_t aph = (uint32_t)(i >> 1) & 1u;
+            const int m = (int)(t % num_m), n = (int)(t / num_m);
+            // Every lane waits; the warp leaves together if any lane gave up, so that the
+            // warp-collective tensor-memory loads below are always executed by all lanes.
+            const bool ok = wait_or_abort(&tfull[acc], aph, a.status, abort_flag);
+            if (!__all_sync(0xFFFFFFFFu, ok))
+                break;
+            tc::fence_after_sync();
+            const uint32_t taddr =
+                tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * BN);
+            const int r = m * BM + row_in_tile;
+            const int col0 = n * BN;
+            float v[32];
+            if (EPI == kReduce) {
+                // Pass 1: max and its first column; NaN is tracked apart (fmax would drop it).
+                float M = -__int_as_float(0x7F800000);
+                uint32_t idx = kNoIdx;
+                bool nan = false;
+#pragma unroll 1
+                for (int c = 0; c < BN / 32; ++c) {
+                    tc::tmem_ld_32cols(taddr + c * 32, v);
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        const int col = col0 + c * 32 + j;
+                        if (col < a.V) {
+                            nan |= v[j] != v[j];
+                            if (v[j] > M) {
+                                M = v[j];
+                                idx = (uint32_t)col;
+                            }
+                        }
+                    }
+                }
+                // Pass 2: sum of exp(x - M) = 2^(x log2e - M log2e), four partial sums.
+                const float M2 = M * kLog2e;
+                float S4[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll 1
+                for (int c = 0; c < BN / 32; ++c) {
+                    tc::tmem_ld_32cols(taddr + c * 32, v);
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        const int col = col0 + c * 32 + j;
+                        if (col < a.V)
+                            S4[j & 3] += ex2_mufu(fmaf(v[j], kLog2e, -M2));
+                    }
+                }
+                tc::fence_before_sync();
+                __syncwarp();
+                if (lane == 0)
+                    mbar_arrive(&tempty[acc]);
+                if (r < R) {
+                    UnitPartial p;
+                    p.M = nan ? __int_as_float(0x7FC00000) : M;
+                    p.S = (S4[0] + S4[1]) + (S4[2] + S4[3]);
+                    p.idx = idx;
+                    p.pad = 0;
+                    a.partials[(int64_t)r * a.n_tiles + n] = p;
+                }
+            } else {
+                const int64_t row = r < R ? a.row_ids[r] : -1;
+#pragma unroll 1
+                for (int c = 0; c < BN / 32; ++c) {
+                    tc::tmem_ld_32cols(taddr + c * 32, v);
+                    if (row >= 0) {
+                        float *dst = a.logits + row * a.V + col0 + c * 32;
+#pragma unroll
+                        for (int j = 0; j < 32; ++j)
+                            if (col0 + c * 32 + j < a.V)
+                                dst[j] = v[j];
+                    }
+                }
+                tc::fence_before_sync();
+                __syncwarp();
+                if (lane == 0)
+                    mbar_arrive(&tempty[acc]);
+            }
+        }
+    }
+    __syncthreads();
+    if (warp == 1) {
+        __syncwarp();
+        tc::fence_after_sync();
+        tc::tmem_dealloc(tmem_base, kTmemCols);
+    }
+}
+
+// One CTA: the packed list of masked rows (ascending) and its length.
+__global__ void __launch_bounds__(1024) compact_rows_kernel(const uint8_t *mask, int rows,
+                                                            int32_t *row_ids, int32_t *row_count)
+{
+    __shared__ int warp_sums[32];
+    const int per = (rows + blockDim.x - 1) / blockDim.x;
+    const int lo = threadIdx.x * per;
+    const int hi = lo + per < rows ? lo + per : rows;
+    int cnt = 0;
+    for (int i = lo; i < hi; ++i)
+        cnt += mask[i] != 0;
+    // Block exclusive scan of cnt.
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int incl = cnt;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+        if (lane >= o)
+            incl += y;
+    }
+    if (lane == 31)
+        warp_sums[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        const int nw = blockDim.x >> 5;
+        int w = lane < nw ? warp_sums[lane] : 0;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xFFFFFFFFu, w, o);
+            if (lane >= o)
+                w += y;
+        }
+        if (lane < nw)
+            warp_sums[lane] = w;  // inclusive over warps
+    }
+    __syncthreads();
+    int pos = incl - cnt + (warp > 0 ? warp_sums[warp - 1] : 0);
+    for (int i = lo; i < hi; ++i)
+        if (mask[i] != 0)
+            row_ids[pos++] = i;
+    if (threadIdx.x == blockDim.x - 1)
+        *row_count = pos;
+}
+
+// CTA k copies the hidden state of packed row k (16-byte vectors).
+__global__ void gather_rows_kernel(const int4 *hidden, int64_t vec_per_row, const int32_t *row_ids,
+                                   const int32_t *row_count, int4 *packed)
+{
+    const int k = blockIdx.x;
+    if (k >= *row_count)
+        return;
+    const int4 *src = hidden + (int64_t)row_ids[k] * vec_per_row;
+    int4 *dst = packed + (int64_t)k * vec_per_row;
+    for (int64_t i = threadIdx.x; i < vec_per_row; i += blockDim.x)
+        dst[i] = __ldg(src + i);
+}
+
+struct Part {
+    float M, S;
+    uint32_t idx;
+    bool nan;
+};
+
+// Fold of two partials: larger max, sums re-based to it, the lowest index attaining it.
+// Symmetric, so both lanes of a shuffle step obtain the same bits.
+__device__ __forceinline__ Part fold(const Part &x, const Part &y)
+{
+    Part r;
+    r.nan = x.nan || y.nan;
+    r.M = fmaxf(x.M, y.M);
+    const float M2 = r.M * kLog2e;
+    r.S = rebase(x.S, x.M * kLog2e, M2) + rebase(y.S, y.M * kLog2e, M2);
+    const uint32_t ix = x.M == r.M ? x.idx : kNoIdx;
+    const uint32_t iy = y.M == r.M ? y.idx : kNoIdx;
+    r.idx = ix < iy ? ix : iy;
+    return r;
+}
+
+// One warp per packed row: lane j folds tiles j, j + 32, ... in order, then the lanes fold
+// in a fixed butterfly.  Writes c = min(1/S, 1) and x_hat at the row's (b, l); a row with a
+// NaN logit or an infinite maximum gets c = NaN, x_hat = -1.
+__global__ void combine_rows_kernel(const UnitPartial *partials, int n_tiles,
+                                    const int32_t *row_ids, const int32_t *row_count,
+                                    float *conf, int32_t *tok)
+{
+    const int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (r >= *row_count)
+        return;
+    Part acc{-__int_as_float(0x7F800000), 0.0f, kNoIdx, false};
+    const UnitPartial *p = partials + (int64_t)r * n_tiles;
+    for (int j = lane; j < n_tiles; j += 32) {
+        const int4 q = __ldcg(reinterpret_cast<const int4 *>(p + j));
+        Part y{__int_as_float(q.x), __int_as_float(q.y), (uint32_t)q.z, false};
+        y.nan = y.M != y.M;
+        if (y.nan)
+            y.M = -__int_as_float(0x7F800000);
+        acc = fold(acc, y);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        Part y;
+        y.M = __shfl_xor_sync(0xFFFFFFFFu, acc.M, o);
+        y.S = __shfl_xor_sync(0xFFFFFFFFu, acc.S, o);
+        y.idx = __shfl_xor_sync(0xFFFFFFFFu, acc.idx, o);
+        y.nan = __shfl_xor_sync(0xFFFFFFFFu, (int)acc.nan, o) != 0;
+        acc = fold(acc, y);
+    }
+    if (lane == 0) {
+        const int row = row_ids[r];
+        const bool finite = fabsf(acc.M) <= 3.402823466e38f && fabsf(acc.S) <= 3.402823466e38f;
+        if (acc.nan || !finite || !(acc.S > 0.0f) || acc.idx == kNoIdx) {
+            conf[row] = __int_as_float(0x7FC00000);
+            tok[row] = -1;
+        } else {
+            conf[row] = fminf(1.0f / acc.S, 1.0f);
+            tok[row] = (int32_t)acc.idx;
+        }
+    }
+}
+
+// ----------------------------------------------------------------------------- host side
+// Workspace layout (offsets from the 256-byte aligned base; header shared with
+// fdllm_select's layout: status at 0, the vocab reduction's counter at 4 left untouched):
+//   row_count int32 at 8
+//   row_ids   int32 [rows]
+//   packed    bf16 [rows][H]            (1024-byte aligned: a TMA source)
+//   partials  UnitPartial [rows][n_tiles]
+//   conf      fp32 [rows], tok int32 [rows]
+struct LmLayout {
+    size_t row_count, row_ids, packed, partials, conf, tok, total;
+};
+
+size_t up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+LmLayout lm_layout(int64_t rows, int64_t H, int64_t n_tiles)
+{
+    LmLayout l;
+    l.row_count = 8;
+    l.row_ids = 256;
+    l.packed = up(l.row_ids + (size_t)rows * 4, 1024);
+    l.partials = up(l.packed + (size_t)rows * H * 2, 256);
+    l.conf = up(l.partials + (size_t)rows * n_tiles * sizeof(UnitPartial), 256);
+    l.tok = up(l.conf + (size_t)rows * 4, 256);
+    l.total = up(l.tok + (size_t)rows * 4, 256);
+    return l;
+}
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                   const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                   const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn()
+{
+    static EncodeTiledFn fn = [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                             cudaEnableDefault, &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess)
+            return (EncodeTiledFn) nullptr;
+        return reinterpret_cast<EncodeTiledFn>(p);
+    }();
+    return fn;
+}
+
+// bf16 matrix [outer][inner] (row stride inner * 2 bytes), loaded as boxes of
+// {BK, box_outer} with 128-byte swizzling; out-of-range elements read as zero.
+bool make_map(CUtensorMap *map, const void *base, int64_t inner, int64_t outer, int box_outer)
+{
+    EncodeTiledFn enc = encode_fn();
+    if (!enc)
+        return false;
+    const cuuint64_t dims[2] = {(cuuint64_t)inner, (cuuint64_t)outer};
+    const cuuint64_t strides[1] = {(cuuint64_t)inner * 2};
+    const cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)box_outer};
+    const cuuint32_t estr[2] = {1, 1};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides,
+               box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+           CUDA_SUCCESS;
+}
+
+fdllm_status check_lmhead(const void *hidden, const void *w, int B, int L, int H, int V,
+                          const uint8_t *mask)
+{
+    if (B < 1 || L < 1 || L > FDLLM_MAX_L || (int64_t)B * L > FDLLM_MAX_ROWS || V < 1 || H < 8)
+        return FDLLM_ERR_ARG;
+    if (!hidden || !w || !mask)
+        return FDLLM_ERR_ARG;
+    if ((reinterpret_cast<uintptr_t>(hidden) & 15u) || (reinterpret_cast<uintptr_t>(w) & 15u) ||
+        H % 8 != 0)
+        return FDLLM_ERR_ALIGN;
+    const int64_t n_tiles = (V + BN - 1) / BN;
+    if ((int64_t)B * L * n_tiles >= ((int64_t)1 << 31) || (int64_t)H * 2 >= ((int64_t)1 << 31))
+        return FDLLM_ERR_ARG;
+    return FDLLM_OK;
+}
+
+template <int EPI>
+cudaError_t launch_gemm(const CUtensorMap &mh, const CUtensorMap &mw, const GemmArgs &g,
+                        cudaStream_t stream)
+{
+    static std::once_flag once[64];
+    static int sms[64];
+    int dev = 0;
+    cudaError_t err = cudaGetDevice(&dev);
+    if (err != cudaSuccess)
+        return err;
+    if (dev < 0 || dev >= 64)
+        return cudaErrorInvalidDevice;
+    std::call_once(once[dev], [&] {
+        cudaFuncSetAttribute(lmhead_gemm_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)kSmemBytes);
+        cudaDeviceGetAttribute(&sms[dev], cudaDevAttrMultiProcessorCount, dev);
+    });
+    lmhead_gemm_kernel<EPI><<<sms[dev] > 0 ? sms[dev] : 1, kThreads, kSmemBytes, stream>>>(mh, mw,
+                                                                                          g);
+    return cudaGetLastError();
+}
+
+// Steps 1-3 (and 4 for the reduce epilogue) on the owned workspace.
+fdllm_status run_lmhead(const void *hidden, const void *w, int B, int L, int H, int V,
+                        const uint8_t *mask, int epi, float *out_logits, cudaStream_t s,
+                        uint8_t **ws_out, LmLayout *lay_out)
+{
+    const int64_t rows = (int64_t)B * L;
+    const int n_tiles = (V + BN - 1) / BN;
+    const LmLayout lay = lm_layout(rows, H, n_tiles);
+    void *wsv = nullptr;
+    fdllm_status st = owned_workspace(lay.total, s, &wsv);
+    if (st != FDLLM_OK)
+        return st;
+    uint8_t *ws = static_cast<uint8_t *>(wsv);
+    int32_t *row_count = reinterpret_cast<int32_t *>(ws + lay.row_count);
+    int32_t *row_ids = reinterpret_cast<int32_t *>(ws + lay.row_ids);
+    uint8_t *packed = ws + lay.packed;
+
+    CUtensorMap mh, mw;
+    if (!make_map(&mh, packed, H, rows, BM) || !make_map(&mw, w, H, V, BN))
+        return FDLLM_ERR_CUDA;
+
+    compact_rows_kernel<<<1, 1024, 0, s>>>(mask, (int)rows, row_ids, row_count);
+    gather_rows_kernel<<<(unsigned)rows, 128, 0, s>>>(static_cast<const int4 *>(hidden), H / 8,
+                                                      row_ids, row_count,
+                                                      reinterpret_cast<int4 *>(packed));
+    if (cudaGetLastError() != cudaSuccess)
+        return FDLLM_ERR_CUDA;
+    GemmArgs g;
+    g.row_count = row_count;
+    g.row_ids = row_ids;
+    g.V = V;
+    g.n_tiles = n_tiles;
+    g.k_blocks = (H + BK - 1) / BK;
+    g.partials = reinterpret_cast<UnitPartial *>(ws + lay.partials);
+    g.logits = out_logits;
+    g.status = reinterpret_cast<uint32_t *>(ws);
+    const cudaError_t e =
+        epi == kReduce ? launch_gemm<kReduce>(mh, mw, g, s) : launch_gemm<kStore>(mh, mw, g, s);
+    if (e != cudaSuccess)
+        return FDLLM_ERR_CUDA;
+    if (epi == kReduce) {
+        const int warps = 8;
+        combine_rows_kernel<<<(unsigned)((rows + warps - 1) / warps), warps * 32, 0, s>>>(
+            g.partials, n_tiles, row_ids, row_count,
+            reinterpret_cast<float *>(ws + lay.conf), reinterpret_cast<int32_t *>(ws + lay.tok));
+        if (cudaGetLastError() != cudaSuccess)
+            return FDLLM_ERR_CUDA;
+    }
+    *ws_out = ws;
+    *lay_out = lay;
+    return FDLLM_OK;
+}
+
+// Copy of the confidences and argmax of the masked rows to caller arrays.
+__global__ void scatter_conf_kernel(const float *conf, const int32_t *tok, const int32_t *row_ids,
+                                    const int32_t *row_count, float *out_conf, int32_t *out_tok)
+{
+    const int k = blockIdx.x * blockDim.x + threadIdx.x;
+    if (k >= *row_count)
+        return;
+    const int row = row_ids[k];
+    out_conf[row] = conf[row];
+    out_tok[row] = tok[row];
+}
+
+}  // namespace
+}  // namespace fdllm
+
+using namespace fdllm;
+
+extern "C" {
+
+fdllm_status fdllm_lmhead_select(const void *hidden, const void *w_vocab, int B, int L, int H,
+                                 int V, uint8_t *mask, double param, int mode,
+                                 int32_t *out_tokens, uint8_t *out_commit, int32_t *out_n,
+                                 void *stream)
+{
+    fdllm_status st = check_lmhead(hidden, w_vocab, B, L, H, V, mask);
+    if (st != FDLLM_OK)
+        return st;
+    if (!out_tokens || !out_commit || !out_n || !std::isfinite(param) ||
+        (mode != FDLLM_PROFILE && mode != FDLLM_FACTOR && mode != FDLLM_THRESHOLD))
+        return FDLLM_ERR_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    uint8_t *ws = nullptr;
+    LmLayout lay;
+    st = run_lmhead(hidden, w_vocab, B, L, H, V, mask, kReduce, nullptr, s, &ws, &lay);
+    if (st != FDLLM_OK)
+        return st;
+    ProfileSelectArgs pa;
+    pa.units_per_row = 0;
+    pa.partials = nullptr;
+    pa.next_unit = nullptr;
+    pa.conf = reinterpret_cast<const float *>(ws + lay.conf);
+    pa.tok = reinterpret_cast<const int32_t *>(ws + lay.tok);
+    pa.mask = mask;
+    pa.B = B;
+    pa.L = L;
+    pa.mode = mode;
+    pa.param = param;
+    pa.eta = 0.0;
+    pa.eta_pos = nullptr;
+    pa.out_tokens = out_tokens;
+    pa.out_commit = out_commit;
+    pa.out_n = out_n;
+    pa.status = reinterpret_cast<const uint32_t *>(ws);
+    pa.pdl = false;
+    return launch_profile_select(pa, s) == cudaSuccess ? FDLLM_OK : FDLLM_ERR_CUDA;
+}
+
+fdllm_status fdllm_lmhead_confidence(const void *hidden, const void *w_vocab, int B, int L,
+                                     int H, int V, const uint8_t *mask, float *out_conf,
+                                     int32_t *out_argmax, void *stream)
+{
+    fdllm_status st = check_lmhead(hidden, w_vocab, B, L, H, V, mask);
+    if (st != FDLLM_OK)
+        return st;
+    if (!out_conf || !out_argmax)
+        return FDLLM_ERR_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    uint8_t *ws = nullptr;
+    LmLayout lay;
+    st = run_lmhead(hidden, w_vocab, B, L, H, V, mask, kReduce, nullptr, s, &ws, &lay);
+    if (st != FDLLM_OK)
+        return st;
+    const int64_t rows = (int64_t)B * L;
+    scatter_conf_kernel<<<(unsigned)((rows + 255) / 256), 256, 0, s>>>(
+        reinterpret_cast<const float *>(ws + lay.conf),
+        reinterpret_cast<const int32_t *>(ws + lay.tok),
+        reinterpret_cast<const int32_t *>(ws + lay.row_ids),
+        reinterpret_cast<const int32_t *>(ws + lay.row_count), out_conf, out_argmax);
+    return cudaGetLastError() == cudaSuccess ? FDLLM_OK : FDLLM_ERR_CUDA;
+}
+
+fdllm_status fdllm_lmhead_logits(const void *hidden, const void *w_vocab, int B, int L, int H,
+                                 int V, const uint8_t *mask, float *out_logits, void *stream)
+{
+    fdllm_status st = check_lmhead(hidden, w_vocab, B, L, H, V, mask);
+    if (st != FDLLM_OK)
+        return st;
+    if (!out_logits)
+        return FDLLM_ERR_ARG;
+    uint8_t *ws = nullptr;
+    LmLayout lay;
+    return run_lmhead(hidden, w_vocab, B, L, H, V, mask, kStore, out_logits,
+                      static_cast<cudaStream_t>(stream), &ws, &lay);
+}
+
+}  // extern "C"

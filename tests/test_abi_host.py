@@ -141,3 +141,24 @@ def test_decode_loop_rejects_before_any_device_call(lib):
     assert f(forward=fwd_t()) == ERR_ARG          # null forward pass
     assert f(logits=None) == ERR_ARG
     assert not calls and steps.value == -5
+
+
+def test_lmhead_rejects_before_any_device_call(lib):
+    p, i, d = ctypes.c_void_p, ctypes.c_int, ctypes.c_double
+    lib.fdllm_lmhead_select.argtypes = [p, p, i, i, i, i, p, d, i, p, p, p, p]
+    lib.fdllm_lmhead_logits.argtypes = [p, p, i, i, i, i, p, p, p]
+
+    def f(hidden=A16, w=A16, B=2, L=32, H=4096, V=126464, mask=A16, mode=0, param=1.0):
+        return lib.fdllm_lmhead_select(hidden, w, B, L, H, V, mask, param, mode, A16, A16, A16,
+                                       None)
+    assert f(H=4100) == ERR_ALIGN          # rows of H bf16 not a multiple of 16 bytes
+    assert f(hidden=A2) == ERR_ALIGN
+    assert f(w=A2) == ERR_ALIGN
+    assert f(H=0) == ERR_ARG
+    assert f(V=0) == ERR_ARG
+    assert f(L=1025) == ERR_ARG
+    assert f(B=65, L=1024) == ERR_ARG      # B * L > 65536
+    assert f(mask=None) == ERR_ARG
+    assert f(mode=3) == ERR_ARG
+    assert f(param=float("nan")) == ERR_ARG
+    assert lib.fdllm_lmhead_logits(A16, A16, 2, 32, 64, 1000, A16, None, None) == ERR_ARG
