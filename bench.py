@@ -18,6 +18,7 @@ host cores, each step a bounded sample of the same workload.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import datetime
 import hashlib
 import json
@@ -495,7 +496,10 @@ def run_lmhead(args) -> dict:
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     wl = syn.WORKLOADS["serving_b64_l32_bf16"]
+    if args.lmhead_batch != wl.B:
+        wl = dataclasses.replace(wl, B=args.lmhead_batch)
     B, L, H, V = wl.B, wl.L, syn.LLADA_HIDDEN, syn.LLADA_VOCAB
+    variants = set(args.lmhead_variants.split(","))
     hidden, w, _ = syn.make_lmhead_inputs(B, L, H, V, seed=1234, device=dev)
     mask0_np = syn.make_mask(wl, seed=1234)
     R = int(mask0_np.sum())
@@ -505,7 +509,9 @@ def run_lmhead(args) -> dict:
     tok = torch.full((B, L), -1, dtype=torch.int32, device=dev)
     commit = torch.empty((B, L), dtype=torch.uint8, device=dev)
     n_out = torch.empty((B,), dtype=torch.int32, device=dev)
-    logits32 = torch.empty((B, L, V), dtype=torch.float32, device=dev)
+    logits32 = (torch.empty((B, L, V), dtype=torch.float32, device=dev)
+                if "ours" in variants else None)
+    rows_idx = torch.from_numpy(np.nonzero(mask0_np.reshape(-1))[0]).to(dev)
     stream = torch.cuda.Stream(device=dev)
 
     def fused():
@@ -522,6 +528,10 @@ def run_lmhead(args) -> dict:
         mask.copy_(mask0, non_blocking=True)
         x = torch.matmul(hidden.view(B * L, H), w.t()).view(B, L, V)
         fd.fdllm_select(x, mask, args.param, mode, tok, commit, n_out, stream=stream)
+
+    def cublas_masked_gemm():
+        # the same GEMM work as the fused path (masked rows only), logits in bf16, no selection
+        torch.matmul(hidden.view(B * L, H).index_select(0, rows_idx), w.t())
 
     def gemm_only():
         fd.fdllm_lmhead_confidence(hidden, w, mask0, stream=stream)
@@ -551,23 +561,32 @@ def run_lmhead(args) -> dict:
 
     sampler = ClockSampler(0).start()
     tw0 = time.time()
-    t_fused = time_variant(fused)
-    t_gemm = time_variant(gemm_only)
-    t_ours = time_variant(ours_unfused)
-    t_cublas = time_variant(cublas_unfused)
+    t = {}
+    for name, fn in (("fused", fused), ("fused_confidence_only", gemm_only),
+                     ("ours_gemm_store_then_select", ours_unfused),
+                     ("cublas_bf16_logits_then_select", cublas_unfused),
+                     ("cublas_gemm_masked_rows_only", cublas_masked_gemm)):
+        key = {"fused": "fused", "fused_confidence_only": "gemm",
+               "ours_gemm_store_then_select": "ours",
+               "cublas_bf16_logits_then_select": "cublas",
+               "cublas_gemm_masked_rows_only": "cublas_masked"}[name]
+        if key in variants:
+            t[name] = time_variant(fn)
     tw1 = time.time()
     time.sleep(0.12)
     sampler.stop()
 
     # the fused path and the unfused ones take the same decisions on these inputs
-    res = {}
-    for name, fn in (("fused", fused), ("ours_unfused", ours_unfused)):
-        with torch.cuda.stream(stream):
-            fn()
-        stream.synchronize()
-        res[name] = (n_out.clone(), commit.clone())
-    same = bool(torch.equal(res["fused"][0], res["ours_unfused"][0]) and
-                torch.equal(res["fused"][1], res["ours_unfused"][1]))
+    same = None
+    if "ours" in variants:
+        res = {}
+        for name, fn in (("fused", fused), ("ours_unfused", ours_unfused)):
+            with torch.cuda.stream(stream):
+                fn()
+            stream.synchronize()
+            res[name] = (n_out.clone(), commit.clone())
+        same = bool(torch.equal(res["fused"][0], res["ours_unfused"][0]) and
+                    torch.equal(res["fused"][1], res["ours_unfused"][1]))
 
     flops = 2.0 * R * H * V
     peaks = {}
@@ -577,17 +596,20 @@ def run_lmhead(args) -> dict:
     except OSError:
         pass
     peak = float(peaks.get("bf16_tflops", 1900.0))
+    t_gemm = t.get("fused_confidence_only", t.get("fused"))
     achieved = flops / (t_gemm * 1e-3) / 1e12
     return {
         "metric": "LM head + commit-set selection: ms per step and GEMM TFLOP/s",
         "workload": "lmhead_b%d_l%d_h%d_v%d_bf16" % (B, L, H, V),
         "B": B, "L": L, "H": H, "V": V, "masked_rows": R, "mode": args.mode,
         "param": args.param, "data": "synthetic",
-        "ms_per_step": {"fused": t_fused, "ours_gemm_store_then_select": t_ours,
-                        "cublas_bf16_logits_then_select": t_cublas,
-                        "fused_confidence_only": t_gemm},
-        "selections_per_s_fused": B / (t_fused * 1e-3),
-        "speedup_vs_cublas_unfused": t_cublas / t_fused,
+        "ms_per_step": t,
+        "selections_per_s_fused": B / (t["fused"] * 1e-3) if "fused" in t else None,
+        "speedup_vs_cublas_unfused": (t["cublas_bf16_logits_then_select"] / t["fused"]
+                                      if "fused" in t and "cublas_bf16_logits_then_select" in t
+                                      else None),
+        "cublas_masked_rows_tflops": (flops / (t["cublas_gemm_masked_rows_only"] * 1e-3) / 1e12
+                                      if "cublas_gemm_masked_rows_only" in t else None),
         "identical_decisions_fused_vs_unfused": same,
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak, "kernel": "fdllm_lmhead_confidence (compaction, "
@@ -715,6 +737,9 @@ def main(argv=None):
                     help="time the LM-head-fused selection against unfused paths, instead of "
                          "the throughput line")
     ap.add_argument("--lmhead-steps", type=int, default=50)
+    ap.add_argument("--lmhead-batch", type=int, default=64)
+    ap.add_argument("--lmhead-variants", default="fused,gemm,ours,cublas,cublas_masked",
+                    help="comma list of: fused, gemm, ours, cublas, cublas_masked")
     args = ap.parse_args(argv)
     if args.lmhead:
         print(json.dumps(run_lmhead(args)), flush=True)

@@ -206,15 +206,19 @@ def make_lmhead_inputs(B: int, L: int, H: int, V: int, seed: int, beta_lo: float
     dev = torch.device(device)
     g = torch.Generator(device=dev)
     g.manual_seed(int(seed) * 7919 + 17)
-    w = torch.randn((V, H), generator=g, device=dev, dtype=torch.float32)
-    w.mul_(1.0 / math.sqrt(H))
+    w = torch.empty((V, H), device=dev, dtype=torch.bfloat16)
+    chunk = 16384  # rows drawn in fp32 at a time (bounded temporary memory)
+    for v0 in range(0, V, chunk):
+        part = torch.randn((min(chunk, V - v0), H), generator=g, device=dev,
+                           dtype=torch.float32)
+        w[v0:v0 + part.shape[0]] = (part * (1.0 / math.sqrt(H))).to(torch.bfloat16)
     t = torch.randint(0, V, (B, L), generator=g, device=dev)
     beta = torch.rand((B, L), generator=g, device=dev, dtype=torch.float32)
     beta = beta * (beta_hi - beta_lo) + beta_lo
     h = torch.randn((B, L, H), generator=g, device=dev, dtype=torch.float32)
-    wt = w[t]
+    wt = w[t].float()
     h += beta[..., None] * wt / (wt * wt).sum(-1, keepdim=True)
-    return h.to(torch.bfloat16), w.to(torch.bfloat16), t
+    return h.to(torch.bfloat16), w, t
 
 
 # ----------------------------------------------------------------------------- GPU stand-in
