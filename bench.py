@@ -602,6 +602,8 @@ def run_lmhead(args) -> dict:
         "metric": "LM head + commit-set selection: ms per step and GEMM TFLOP/s",
         "workload": "lmhead_b%d_l%d_h%d_v%d_bf16" % (B, L, H, V),
         "B": B, "L": L, "H": H, "V": V, "masked_rows": R, "mode": args.mode,
+        "gemm_variant_env": {k: os.environ[k] for k in ("FDLLM_LMHEAD_CLUSTER", "FDLLM_LMHEAD_BN")
+                             if k in os.environ},
         "param": args.param, "data": "synthetic",
         "ms_per_step": t,
         "selections_per_s_fused": B / (t["fused"] * 1e-3) if "fused" in t else None,

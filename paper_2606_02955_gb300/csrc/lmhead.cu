@@ -17,6 +17,7 @@
 
 #include <cmath>
 #include <cstdint>
+#include <cstdlib>
 #include <mutex>
 
 #include "fdllm.h"
@@ -28,17 +29,29 @@ namespace fdllm {
 namespace {
 
 constexpr int BM = 128;  // rows per tile (TMEM lanes)
-constexpr int BN = 256;  // vocabulary entries per tile (fp32 TMEM columns per accumulator)
 constexpr int BK = 64;   // hidden elements per stage: one 128-byte swizzle row of bf16
-constexpr int kStages = 4;
 constexpr int kABytes = BM * BK * 2;
-constexpr int kBBytes = BN * BK * 2;
-constexpr int kStageBytes = kABytes + kBBytes;
-constexpr int kThreads = 192;           // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
-constexpr uint32_t kTmemCols = 2 * BN;  // two accumulators
+constexpr int kThreads = 192;         // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
+constexpr uint32_t kAccStride = 256;  // TMEM columns between the two accumulators
+constexpr uint32_t kTmemCols = 512;
 constexpr size_t kBarrierBytes = 256;
-constexpr size_t kSmemBytes = 1024 + (size_t)kStages * kStageBytes + kBarrierBytes;
+constexpr size_t kRingBudget = 220 * 1024;
 constexpr uint64_t kDrainLimitNs = 100000000ull;  // waits for own copies after an abort
+
+// Vocabulary entries per tile (the MMA's N and the fp32 accumulator's width): 256, or 208,
+// which splits LLaDA's V = 126464 into 608 = 4 x 152 tiles, one whole wave per SM count.
+// The stage count fills the ring budget: 4 x 48 KB at 256, 5 x 42 KB at 208.
+template <int BN_>
+struct TileCfg {
+    static constexpr int BN = BN_;
+    static constexpr int kBBytes = BN * BK * 2;
+    static constexpr int kStageBytes = kABytes + kBBytes;
+    static constexpr int kStages =
+        (int)(kRingBudget / kStageBytes) > 6 ? 6 : (int)(kRingBudget / kStageBytes);
+    static constexpr size_t kSmemBytes = 1024 + (size_t)kStages * kStageBytes + kBarrierBytes;
+    static_assert(BN % 16 == 0 && BN <= (int)kAccStride, "MMA N for M = 128");
+    static_assert((BN / 2) % 8 == 0, "halves of whole 8-row swizzle atoms");
+};
 
 enum Epilogue { kReduce = 0, kStore = 1 };
 
@@ -75,11 +88,18 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity, ui
     }
 }
 
-template <int EPI>
+// CL = 1: every CTA loads its own W tile.  CL = 2: the two CTAs of a cluster take row tiles
+// 2j and 2j + 1 of the same vocabulary tile; each loads half of the W tile and multicasts it
+// into both CTAs' shared memory (half the L2 -> SM traffic for W), and each MMA releases a
+// stage in both CTAs, since either producer overwrites it in both.
+template <int EPI, int CL, int BN_>
 __global__ void __launch_bounds__(kThreads, 1)
     lmhead_gemm_kernel(const __grid_constant__ CUtensorMap map_h,
                        const __grid_constant__ CUtensorMap map_w, const GemmArgs a)
 {
+    using Cfg = TileCfg<BN_>;
+    constexpr int BN = Cfg::BN, kStages = Cfg::kStages;
+    constexpr int kBBytes = Cfg::kBBytes, kStageBytes = Cfg::kStageBytes;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -98,7 +118,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             mbar_init(&full[s], 1);
-            mbar_init(&empty[s], 1);
+            mbar_init(&empty[s], CL);  // one release per consuming CTA
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&tfull[i], 1);
@@ -114,14 +134,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc::tmem_alloc(tmem_slot, kTmemCols);
     tc::fence_before_sync();
     __syncthreads();
+    if (CL > 1)
+        tc::cluster_sync();  // the peer's barriers are initialised before any multicast
     tc::fence_after_sync();
     const uint32_t tmem_base = *tmem_slot;
 
+    const int rank = CL > 1 ? (int)tc::cluster_ctarank() : 0;
+    const int64_t first = CL > 1 ? (int64_t)tc::cluster_id_x() : (int64_t)blockIdx.x;
+    const int64_t stride = CL > 1 ? (int64_t)tc::cluster_count_x() : (int64_t)gridDim.x;
     const int R = *a.row_count;
     const int num_m = (R + BM - 1) / BM;
-    const int64_t total = (int64_t)num_m * a.n_tiles;
-    // Tile t covers packed rows [m*BM, +BM) x vocabulary [n*BN, +BN) with m fastest, so the
-    // CTAs working at the same time share few W tiles (read from HBM once, then from L2).
+    const int num_mc = (num_m + CL - 1) / CL;  // row-tile groups, one per cluster
+    const int64_t total = (int64_t)num_mc * a.n_tiles;
+    // Work item t covers packed rows [m*BM, +BM) with m = (t % num_mc) * CL + rank, and
+    // vocabulary [n*BN, +BN) with n = t / num_mc: row tiles fastest, so the CTAs working at
+    // the same time share few W tiles (read from HBM once, then from L2).  With CL = 2 and
+    // an odd number of row tiles, the last rank-1 CTA computes a tile of rows >= R (zero or
+    // stale inputs) that its epilogue skips.
 
     if (warp == 0) {
         if (lane == 0) {
@@ -132,8 +161,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int i = 0; i < kStages; ++i)
                 used[i] = false;
             bool ok = true;
-            for (int64_t t = blockIdx.x; ok && t < total; t += gridDim.x) {
-                const int m = (int)(t % num_m), n = (int)(t / num_m);
+            for (int64_t t = first; ok && t < total; t += stride) {
+                const int m = (int)(t % num_mc) * CL + rank, n = (int)(t / num_mc);
                 for (int kb = 0; kb < a.k_blocks; ++kb) {
                     if (!wait_or_abort(&empty[s], ph ^ 1u, a.status, abort_flag)) {
                         ok = false;
@@ -141,7 +170,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     mbar_arrive_expect_tx(&full[s], kStageBytes);
                     tc::tma_load_2d(sA + s * kABytes, &map_h, kb * BK, m * BM, &full[s]);
-                    tc::tma_load_2d(sB + s * kBBytes, &map_w, kb * BK, n * BN, &full[s]);
+                    if (CL == 1)
+                        tc::tma_load_2d(sB + s * kBBytes, &map_w, kb * BK, n * BN, &full[s]);
+                    else
+                        tc::tma_load_2d_multicast(sB + s * kBBytes + rank * (kBBytes / CL), &map_w,
+                                                  kb * BK, n * BN + rank * (BN / CL), &full[s],
+                                                  (uint16_t)((1u << CL) - 1u));
                     used[s] = true;
                     last_ph[s] = ph;
                     if (++s == kStages) {
@@ -162,13 +196,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t ph = 0;
             bool ok = true;
             int i = 0;
-            for (int64_t t = blockIdx.x; ok && t < total; t += gridDim.x, ++i) {
+            for (int64_t t = first; ok && t < total; t += stride, ++i) {
                 const int acc = i & 1;
                 const uint32_t aph = (uint32_t)(i >> 1) & 1u;
                 if (!wait_or_abort(&tempty[acc], aph ^ 1u, a.status, abort_flag))
                     break;
                 tc::fence_after_sync();
-                const uint32_t d = tmem_base + (uint32_t)(acc * BN);
+                const uint32_t d = tmem_base + (uint32_t)acc * kAccStride;
                 for (int kb = 0; kb < a.k_blocks; ++kb) {
                     if (!wait_or_abort(&full[s], ph, a.status, abort_flag)) {
                         ok = false;
@@ -180,7 +214,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int k = 0; k < BK / 16; ++k)  // K = 16 per MMA: +32 B in the row
                         tc::mma_bf16(d, ad + 2u * k, bd + 2u * k, idesc, (kb | k) != 0);
-                    tc::commit(&empty[s]);  // the stage is free once these MMAs have read it
+                    // The stage is free once these MMAs have read it (in every CTA of the
+                    // cluster: either producer overwrites it in both).
+                    if (CL == 1)
+                        tc::commit(&empty[s]);
+                    else
+                        tc::commit_multicast(&empty[s], (uint16_t)((1u << CL) - 1u));
                     if (++s == kStages) {
                         s = 0;
                         ph ^= 1u;
@@ -199,10 +238,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int quarter = warp & 3;
         const int row_in_tile = quarter * 32 + lane;
         int i = 0;
-        for (int64_t t = blockIdx.x; t < total; t += gridDim.x, ++i) {
+        for (int64_t t = first; t < total; t += stride, ++i) {
             const int acc = i & 1;
             const uint32_t aph = (uint32_t)(i >> 1) & 1u;
-            const int m = (int)(t % num_m), n = (int)(t / num_m);
+            const int m = (int)(t % num_mc) * CL + rank, n = (int)(t / num_mc);
             // Every lane waits; the warp leaves together if any lane gave up, so that the
             // warp-collective tensor-memory loads below are always executed by all lanes.
             const bool ok = wait_or_abort(&tfull[acc], aph, a.status, abort_flag);
@@ -210,7 +249,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 break;
             tc::fence_after_sync();
             const uint32_t taddr =
-                tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * BN);
+                tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)acc * kAccStride;
             const int r = m * BM + row_in_tile;
             const int col0 = n * BN;
             float v[32];
@@ -220,12 +259,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 uint32_t idx = kNoIdx;
                 bool nan = false;
 #pragma unroll 1
-                for (int c = 0; c < BN / 32; ++c) {
-                    tc::tmem_ld_32cols(taddr + c * 32, v);
+                for (int c = 0; c < (BN + 31) / 32; ++c) {
+                    tc::tmem_ld_32cols(taddr + c * 32, v);  // columns >= BN: not this tile
 #pragma unroll
                     for (int j = 0; j < 32; ++j) {
                         const int col = col0 + c * 32 + j;
-                        if (col < a.V) {
+                        if (c * 32 + j < BN && col < a.V) {
                             nan |= v[j] != v[j];
                             if (v[j] > M) {
                                 M = v[j];
@@ -238,12 +277,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const float M2 = M * kLog2e;
                 float S4[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll 1
-                for (int c = 0; c < BN / 32; ++c) {
+                for (int c = 0; c < (BN + 31) / 32; ++c) {
                     tc::tmem_ld_32cols(taddr + c * 32, v);
 #pragma unroll
                     for (int j = 0; j < 32; ++j) {
                         const int col = col0 + c * 32 + j;
-                        if (col < a.V)
+                        if (c * 32 + j < BN && col < a.V)
                             S4[j & 3] += ex2_mufu(fmaf(v[j], kLog2e, -M2));
                     }
                 }
@@ -262,13 +301,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             } else {
                 const int64_t row = r < R ? a.row_ids[r] : -1;
 #pragma unroll 1
-                for (int c = 0; c < BN / 32; ++c) {
+                for (int c = 0; c < (BN + 31) / 32; ++c) {
                     tc::tmem_ld_32cols(taddr + c * 32, v);
                     if (row >= 0) {
                         float *dst = a.logits + row * a.V + col0 + c * 32;
 #pragma unroll
                         for (int j = 0; j < 32; ++j)
-                            if (col0 + c * 32 + j < a.V)
+                            if (c * 32 + j < BN && col0 + c * 32 + j < a.V)
                                 dst[j] = v[j];
                     }
                 }
@@ -285,6 +324,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc::fence_after_sync();
         tc::tmem_dealloc(tmem_base, kTmemCols);
     }
+    if (CL > 1)
+        tc::cluster_sync();  // no CTA leaves while its peer may still write into it
 }
 
 // One CTA: the packed list of masked rows (ascending) and its length.
@@ -378,13 +419,22 @@ __global__ void combine_rows_kernel(const UnitPartial *partials, int n_tiles,
         return;
     Part acc{-__int_as_float(0x7F800000), 0.0f, kNoIdx, false};
     const UnitPartial *p = partials + (int64_t)r * n_tiles;
-    for (int j = lane; j < n_tiles; j += 32) {
-        const int4 q = __ldcg(reinterpret_cast<const int4 *>(p + j));
-        Part y{__int_as_float(q.x), __int_as_float(q.y), (uint32_t)q.z, false};
-        y.nan = y.M != y.M;
-        if (y.nan)
-            y.M = -__int_as_float(0x7F800000);
-        acc = fold(acc, y);
+    constexpr int kBatch = 8;  // loads in flight per lane before the folds
+    for (int j0 = lane; j0 < n_tiles; j0 += 32 * kBatch) {
+        int4 q[kBatch];
+#pragma unroll
+        for (int b = 0; b < kBatch; ++b)
+            if (j0 + 32 * b < n_tiles)
+                q[b] = __ldcg(reinterpret_cast<const int4 *>(p + j0 + 32 * b));
+#pragma unroll
+        for (int b = 0; b < kBatch; ++b)
+            if (j0 + 32 * b < n_tiles) {
+                Part y{__int_as_float(q[b].x), __int_as_float(q[b].y), (uint32_t)q[b].z, false};
+                y.nan = y.M != y.M;
+                if (y.nan)
+                    y.M = -__int_as_float(0x7F800000);
+                acc = fold(acc, y);
+            }
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
@@ -481,32 +531,112 @@ fdllm_status check_lmhead(const void *hidden, const void *w, int B, int L, int H
     if ((reinterpret_cast<uintptr_t>(hidden) & 15u) || (reinterpret_cast<uintptr_t>(w) & 15u) ||
         H % 8 != 0)
         return FDLLM_ERR_ALIGN;
-    const int64_t n_tiles = (V + BN - 1) / BN;
+    const int64_t n_tiles = (V + 207) / 208;  // the narrowest tile
     if ((int64_t)B * L * n_tiles >= ((int64_t)1 << 31) || (int64_t)H * 2 >= ((int64_t)1 << 31))
         return FDLLM_ERR_ARG;
     return FDLLM_OK;
 }
 
-template <int EPI>
-cudaError_t launch_gemm(const CUtensorMap &mh, const CUtensorMap &mw, const GemmArgs &g,
-                        cudaStream_t stream)
+// CTAs sharing each W tile load: 2 (halves multicast) when at least 8 row tiles can share
+// every W tile, where halving the L2 -> SM traffic for W paid off on GB300 (B = 64, L = 32);
+// 1 below that, where the pairs' padding row tile costs more.  FDLLM_LMHEAD_CLUSTER = 1 or
+// 2 forces one.
+int cluster_size(int64_t rows)
+{
+    if (const char *e = std::getenv("FDLLM_LMHEAD_CLUSTER")) {
+        const int f = std::atoi(e);
+        if (f == 1 || f == 2)
+            return f;
+    }
+    return (rows + BM - 1) / BM >= 8 ? 2 : 1;
+}
+
+int sm_count()
+{
+    static int cache[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64)
+        return 152;
+    if (cache[dev] == 0) {
+        int n = 0;
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+        cache[dev] = n > 0 ? n : 152;
+    }
+    return cache[dev];
+}
+
+// The vocabulary tile width with the least estimated time: whole waves of tiles over the
+// SMs (row tiles estimated from B * L, the most the mask can hold) times the tile width;
+// ties go to the wider tile.  FDLLM_LMHEAD_BN = 256 or 208 forces one.
+int choose_bn(int64_t rows, int V)
+{
+    if (const char *e = std::getenv("FDLLM_LMHEAD_BN")) {
+        const int f = std::atoi(e);
+        if (f == 256 || f == 208)
+            return f;
+    }
+    const int64_t m_tiles = (rows + BM - 1) / BM, sms = sm_count();
+    int best = 256;
+    int64_t best_cost = -1;
+    for (int bn : {256, 208}) {
+        const int64_t tiles = (V + bn - 1) / bn * m_tiles;
+        const int64_t cost = (tiles + sms - 1) / sms * bn;
+        if (best_cost < 0 || cost < best_cost) {
+            best = bn;
+            best_cost = cost;
+        }
+    }
+    return best;
+}
+
+template <int EPI, int CL, int BN>
+cudaError_t launch_gemm_cfg(const CUtensorMap &mh, const CUtensorMap &mw, const GemmArgs &g,
+                            cudaStream_t stream)
 {
     static std::once_flag once[64];
-    static int sms[64];
+    static int grid[64];
     int dev = 0;
     cudaError_t err = cudaGetDevice(&dev);
     if (err != cudaSuccess)
         return err;
     if (dev < 0 || dev >= 64)
         return cudaErrorInvalidDevice;
+    auto kern = lmhead_gemm_kernel<EPI, CL, BN>;
+    constexpr size_t smem = TileCfg<BN>::kSmemBytes;
+    cudaLaunchConfig_t cfg = {};
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = CL;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
     std::call_once(once[dev], [&] {
-        cudaFuncSetAttribute(lmhead_gemm_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)kSmemBytes);
-        cudaDeviceGetAttribute(&sms[dev], cudaDevAttrMultiProcessorCount, dev);
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        const int sms = sm_count();
+        int clusters = 0;
+        cfg.gridDim = dim3((unsigned)(sms / CL * CL));
+        if (cudaOccupancyMaxActiveClusters(&clusters, kern, &cfg) != cudaSuccess || clusters < 1)
+            clusters = sms / CL;
+        (void)cudaGetLastError();
+        grid[dev] = clusters * CL;  // persistent: every cluster resident at once
     });
-    lmhead_gemm_kernel<EPI><<<sms[dev] > 0 ? sms[dev] : 1, kThreads, kSmemBytes, stream>>>(mh, mw,
-                                                                                          g);
-    return cudaGetLastError();
+    cfg.gridDim = dim3((unsigned)grid[dev]);
+    return cudaLaunchKernelEx(&cfg, kern, mh, mw, g);
+}
+
+template <int EPI>
+cudaError_t launch_gemm(const CUtensorMap &mh, const CUtensorMap &mw, const GemmArgs &g,
+                        int cl, int bn, cudaStream_t stream)
+{
+    if (bn == 208)
+        return cl == 1 ? launch_gemm_cfg<EPI, 1, 208>(mh, mw, g, stream)
+                       : launch_gemm_cfg<EPI, 2, 208>(mh, mw, g, stream);
+    return cl == 1 ? launch_gemm_cfg<EPI, 1, 256>(mh, mw, g, stream)
+                   : launch_gemm_cfg<EPI, 2, 256>(mh, mw, g, stream);
 }
 
 // Steps 1-3 (and 4 for the reduce epilogue) on the owned workspace.
@@ -515,7 +645,8 @@ fdllm_status run_lmhead(const void *hidden, const void *w, int B, int L, int H, 
                         uint8_t **ws_out, LmLayout *lay_out)
 {
     const int64_t rows = (int64_t)B * L;
-    const int n_tiles = (V + BN - 1) / BN;
+    const int bn = choose_bn(rows, V);
+    const int n_tiles = (V + bn - 1) / bn;
     const LmLayout lay = lm_layout(rows, H, n_tiles);
     void *wsv = nullptr;
     fdllm_status st = owned_workspace(lay.total, s, &wsv);
@@ -526,8 +657,9 @@ fdllm_status run_lmhead(const void *hidden, const void *w, int B, int L, int H, 
     int32_t *row_ids = reinterpret_cast<int32_t *>(ws + lay.row_ids);
     uint8_t *packed = ws + lay.packed;
 
+    const int cl = cluster_size(rows);
     CUtensorMap mh, mw;
-    if (!make_map(&mh, packed, H, rows, BM) || !make_map(&mw, w, H, V, BN))
+    if (!make_map(&mh, packed, H, rows, BM) || !make_map(&mw, w, H, V, bn / cl))
         return FDLLM_ERR_CUDA;
 
     compact_rows_kernel<<<1, 1024, 0, s>>>(mask, (int)rows, row_ids, row_count);
@@ -545,8 +677,8 @@ fdllm_status run_lmhead(const void *hidden, const void *w, int B, int L, int H, 
     g.partials = reinterpret_cast<UnitPartial *>(ws + lay.partials);
     g.logits = out_logits;
     g.status = reinterpret_cast<uint32_t *>(ws);
-    const cudaError_t e =
-        epi == kReduce ? launch_gemm<kReduce>(mh, mw, g, s) : launch_gemm<kStore>(mh, mw, g, s);
+    const cudaError_t e = epi == kReduce ? launch_gemm<kReduce>(mh, mw, g, cl, bn, s)
+                                         : launch_gemm<kStore>(mh, mw, g, cl, bn, s);
     if (e != cudaSuccess)
         return FDLLM_ERR_CUDA;
     if (epi == kReduce) {

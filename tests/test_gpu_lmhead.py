@@ -28,6 +28,17 @@ pytestmark = pytest.mark.gpu
 U = 2.0 ** -23
 
 
+@pytest.fixture(params=[(1, 256), (2, 256), (1, 208), (2, 208)],
+                ids=["cta1-n256", "cluster2-n256", "cta1-n208", "cluster2-n208"])
+def cluster(request, monkeypatch):
+    """Every GEMM variant: one CTA per W tile or W halves multicast across a 2-CTA cluster,
+    with vocabulary tiles of 256 or 208 entries."""
+    cl, bn = request.param
+    monkeypatch.setenv("FDLLM_LMHEAD_CLUSTER", str(cl))
+    monkeypatch.setenv("FDLLM_LMHEAD_BN", str(bn))
+    return request.param
+
+
 def bits(t: torch.Tensor) -> np.ndarray:
     return t.detach().cpu().contiguous().view(torch.int16).numpy().view(np.uint16)
 
@@ -51,11 +62,12 @@ SHAPES = [
     (4, 64, 512, 5000),
     (1, 3, 72, 40),
     (3, 100, 256, 2048),
+    (4, 100, 128, 1000),   # three row tiles: an odd count for the cluster pairs
 ]
 
 
 @pytest.mark.parametrize("B,L,H,V", SHAPES)
-def test_gemm_within_fp32_accumulation_bound(fd, orc, B, L, H, V):
+def test_gemm_within_fp32_accumulation_bound(fd, orc, cluster, B, L, H, V):
     h, w, mask_np = inputs(B, L, H, V, seed=B * 1000 + V)
     x = fd.fdllm_lmhead_logits(h, w, torch.from_numpy(mask_np).cuda())
     torch.cuda.synchronize()
@@ -75,7 +87,8 @@ def gpu_logits(fd, h, w, mask_np):
 
 
 @pytest.mark.parametrize("B,L,H,V", SHAPES)
-def test_fused_confidence_matches_oracle_on_the_same_accumulators(fd, orc, B, L, H, V):
+def test_fused_confidence_matches_oracle_on_the_same_accumulators(fd, orc, cluster, B, L, H,
+                                                                  V):
     h, w, mask_np = inputs(B, L, H, V, seed=7 + V)
     conf, tok = fd.fdllm_lmhead_confidence(h, w, torch.from_numpy(mask_np).cuda())
     torch.cuda.synchronize()
@@ -93,7 +106,7 @@ def test_fused_confidence_matches_oracle_on_the_same_accumulators(fd, orc, B, L,
 @pytest.mark.parametrize("mode,param", [(oracle.PROFILE, 1.0), (oracle.PROFILE, 0.75),
                                         (oracle.FACTOR, 1.0), (oracle.THRESHOLD, 0.9)])
 @pytest.mark.parametrize("B,L,H,V", [(4, 32, 512, 5000), (8, 64, 256, 3000)])
-def test_fused_select_matches_oracle(fd, orc, B, L, H, V, mode, param):
+def test_fused_select_matches_oracle(fd, orc, cluster, B, L, H, V, mode, param):
     h, w, mask_np = inputs(B, L, H, V, seed=11 + L)
     x32 = gpu_logits(fd, h, w, mask_np)
     mask = torch.from_numpy(mask_np.copy()).cuda()
@@ -111,7 +124,7 @@ def test_fused_select_matches_oracle(fd, orc, B, L, H, V, mode, param):
 
 
 @pytest.mark.parametrize("B,L,H,V", [(4, 64, 512, 5000), (2, 32, 4096, 8192)])
-def test_fused_confidence_against_exact_logits(fd, orc, B, L, H, V):
+def test_fused_confidence_against_exact_logits(fd, orc, cluster, B, L, H, V):
     h, w, mask_np = inputs(B, L, H, V, seed=21 + H)
     conf, tok = fd.fdllm_lmhead_confidence(h, w, torch.from_numpy(mask_np).cuda())
     torch.cuda.synchronize()
@@ -131,7 +144,7 @@ def test_fused_confidence_against_exact_logits(fd, orc, B, L, H, V):
     assert np.array_equal(g_tok[clear], rt[clear])
 
 
-def test_llada_shape_sampled_rows(fd, orc):
+def test_llada_shape_sampled_rows(fd, orc, cluster):
     # LLaDA-8B head: H = 4096, V = 126464; the serving batch B = 64, L = 32 with 75 % masked.
     B, L, H, V = 64, 32, syn.LLADA_HIDDEN, syn.LLADA_VOCAB
     h, w, mask_np = inputs(B, L, H, V, seed=99)
@@ -156,7 +169,7 @@ def test_llada_shape_sampled_rows(fd, orc):
     assert ((c > 0) & (c <= 1)).all() and ((t >= 0) & (t < V)).all()
 
 
-def test_empty_mask_and_repeat(fd):
+def test_empty_mask_and_repeat(fd, cluster):
     B, L, H, V = 2, 16, 128, 1000
     h, w, _ = inputs(B, L, H, V, seed=3)
     mask = torch.zeros((B, L), dtype=torch.uint8, device="cuda")
