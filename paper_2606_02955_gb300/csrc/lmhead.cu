@@ -139,6 +139,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::fence_after_sync();
     const uint32_t tmem_base = *tmem_slot;
 
+    // A programmatic dependent of the packing kernel: everything above overlapped its tail;
+    // the packed rows and their count are read only past this wait.
+    pdl_wait();
+
     const int rank = CL > 1 ? (int)tc::cluster_ctarank() : 0;
     const int64_t first = CL > 1 ? (int64_t)tc::cluster_id_x() : (int64_t)blockIdx.x;
     const int64_t stride = CL > 1 ? (int64_t)tc::cluster_count_x() : (int64_t)gridDim.x;
@@ -318,6 +322,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
     }
+    if (threadIdx.x == 0)
+        pdl_launch_dependents();  // the row combination may start launching
     __syncthreads();
     if (warp == 1) {
         __syncwarp();
@@ -333,6 +339,9 @@ __global__ void __launch_bounds__(1024) compact_rows_kernel(const uint8_t *mask,
                                                             int32_t *row_ids, int32_t *row_count)
 {
     __shared__ int warp_sums[32];
+    pdl_wait();  // the mask's writer has completed
+    if (threadIdx.x == 0)
+        pdl_launch_dependents();
     const int per = (rows + blockDim.x - 1) / blockDim.x;
     const int lo = threadIdx.x * per;
     const int hi = lo + per < rows ? lo + per : rows;
@@ -376,6 +385,9 @@ __global__ void __launch_bounds__(1024) compact_rows_kernel(const uint8_t *mask,
 __global__ void gather_rows_kernel(const int4 *hidden, int64_t vec_per_row, const int32_t *row_ids,
                                    const int32_t *row_count, int4 *packed)
 {
+    pdl_wait();  // the row list is complete
+    if (threadIdx.x == 0)
+        pdl_launch_dependents();  // the GEMM may start its prologue
     const int k = blockIdx.x;
     if (k >= *row_count)
         return;
@@ -413,6 +425,9 @@ __global__ void combine_rows_kernel(const UnitPartial *partials, int n_tiles,
                                     const int32_t *row_ids, const int32_t *row_count,
                                     float *conf, int32_t *tok)
 {
+    pdl_wait();  // every tile partial is written
+    if (threadIdx.x == 0)
+        pdl_launch_dependents();
     const int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
     if (r >= *row_count)
@@ -521,6 +536,23 @@ bool make_map(CUtensorMap *map, const void *base, int64_t inner, int64_t outer, 
            CUDA_SUCCESS;
 }
 
+// A launch as a programmatic dependent of the previous kernel on the stream.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), unsigned grid, unsigned block, cudaStream_t stream,
+                       Args... args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(block);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
 fdllm_status check_lmhead(const void *hidden, const void *w, int B, int L, int H, int V,
                           const uint8_t *mask)
 {
@@ -607,13 +639,15 @@ cudaError_t launch_gemm_cfg(const CUtensorMap &mh, const CUtensorMap &mw, const 
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = CL;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 1;  // the occupancy query below sees the cluster shape only
     std::call_once(once[dev], [&] {
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         const int sms = sm_count();
@@ -625,6 +659,7 @@ cudaError_t launch_gemm_cfg(const CUtensorMap &mh, const CUtensorMap &mw, const 
         grid[dev] = clusters * CL;  // persistent: every cluster resident at once
     });
     cfg.gridDim = dim3((unsigned)grid[dev]);
+    cfg.numAttrs = 2;
     return cudaLaunchKernelEx(&cfg, kern, mh, mw, g);
 }
 
@@ -662,11 +697,12 @@ fdllm_status run_lmhead(const void *hidden, const void *w, int B, int L, int H, 
     if (!make_map(&mh, packed, H, rows, BM) || !make_map(&mw, w, H, V, bn / cl))
         return FDLLM_ERR_CUDA;
 
-    compact_rows_kernel<<<1, 1024, 0, s>>>(mask, (int)rows, row_ids, row_count);
-    gather_rows_kernel<<<(unsigned)rows, 128, 0, s>>>(static_cast<const int4 *>(hidden), H / 8,
-                                                      row_ids, row_count,
-                                                      reinterpret_cast<int4 *>(packed));
-    if (cudaGetLastError() != cudaSuccess)
+    if (launch_pdl(compact_rows_kernel, 1, 1024, s, mask, (int)rows, row_ids, row_count) !=
+            cudaSuccess ||
+        launch_pdl(gather_rows_kernel, (unsigned)rows, 128, s,
+                   static_cast<const int4 *>(hidden), (int64_t)(H / 8),
+                   (const int32_t *)row_ids, (const int32_t *)row_count,
+                   reinterpret_cast<int4 *>(packed)) != cudaSuccess)
         return FDLLM_ERR_CUDA;
     GemmArgs g;
     g.row_count = row_count;
@@ -683,10 +719,10 @@ fdllm_status run_lmhead(const void *hidden, const void *w, int B, int L, int H, 
         return FDLLM_ERR_CUDA;
     if (epi == kReduce) {
         const int warps = 8;
-        combine_rows_kernel<<<(unsigned)((rows + warps - 1) / warps), warps * 32, 0, s>>>(
-            g.partials, n_tiles, row_ids, row_count,
-            reinterpret_cast<float *>(ws + lay.conf), reinterpret_cast<int32_t *>(ws + lay.tok));
-        if (cudaGetLastError() != cudaSuccess)
+        if (launch_pdl(combine_rows_kernel, (unsigned)((rows + warps - 1) / warps), warps * 32,
+                       s, (const UnitPartial *)g.partials, n_tiles, (const int32_t *)row_ids,
+                       (const int32_t *)row_count, reinterpret_cast<float *>(ws + lay.conf),
+                       reinterpret_cast<int32_t *>(ws + lay.tok)) != cudaSuccess)
             return FDLLM_ERR_CUDA;
     }
     *ws_out = ws;
@@ -698,6 +734,7 @@ fdllm_status run_lmhead(const void *hidden, const void *w, int B, int L, int H, 
 __global__ void scatter_conf_kernel(const float *conf, const int32_t *tok, const int32_t *row_ids,
                                     const int32_t *row_count, float *out_conf, int32_t *out_tok)
 {
+    pdl_wait();
     const int k = blockIdx.x * blockDim.x + threadIdx.x;
     if (k >= *row_count)
         return;
@@ -747,7 +784,7 @@ fdllm_status fdllm_lmhead_select(const void *hidden, const void *w_vocab, int B,
     pa.out_commit = out_commit;
     pa.out_n = out_n;
     pa.status = reinterpret_cast<const uint32_t *>(ws);
-    pa.pdl = false;
+    pa.pdl = true;
     return launch_profile_select(pa, s) == cudaSuccess ? FDLLM_OK : FDLLM_ERR_CUDA;
 }
 
@@ -767,12 +804,14 @@ fdllm_status fdllm_lmhead_confidence(const void *hidden, const void *w_vocab, in
     if (st != FDLLM_OK)
         return st;
     const int64_t rows = (int64_t)B * L;
-    scatter_conf_kernel<<<(unsigned)((rows + 255) / 256), 256, 0, s>>>(
-        reinterpret_cast<const float *>(ws + lay.conf),
-        reinterpret_cast<const int32_t *>(ws + lay.tok),
-        reinterpret_cast<const int32_t *>(ws + lay.row_ids),
-        reinterpret_cast<const int32_t *>(ws + lay.row_count), out_conf, out_argmax);
-    return cudaGetLastError() == cudaSuccess ? FDLLM_OK : FDLLM_ERR_CUDA;
+    return launch_pdl(scatter_conf_kernel, (unsigned)((rows + 255) / 256), 256, s,
+                      reinterpret_cast<const float *>(ws + lay.conf),
+                      reinterpret_cast<const int32_t *>(ws + lay.tok),
+                      reinterpret_cast<const int32_t *>(ws + lay.row_ids),
+                      reinterpret_cast<const int32_t *>(ws + lay.row_count), out_conf,
+                      out_argmax) == cudaSuccess
+               ? FDLLM_OK
+               : FDLLM_ERR_CUDA;
 }
 
 fdllm_status fdllm_lmhead_logits(const void *hidden, const void *w_vocab, int B, int L, int H,

@@ -123,8 +123,9 @@ __global__ void __launch_bounds__(T) profile_select_kernel(const ProfileSelectAr
 
     // (c, x_hat) of this thread's position: folded from the vocab reduction's unit
     // partials, or read from the given arrays.
-    if (a.partials != nullptr)
-        pdl_wait();  // the vocab reduction's partials are complete and visible
+    // Launched as a programmatic dependent: whatever produced the unit partials or the
+    // confidences (and the mask) has completed and its writes are visible past this wait.
+    pdl_wait();
     if (threadIdx.x == 0)
         pdl_launch_dependents();  // a following vocab reduction may start its prologue
     const bool masked = t < L && a.mask[base + t] != 0;
@@ -250,7 +251,7 @@ cudaError_t launch_t(const ProfileSelectArgs &a, cudaStream_t stream)
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = a.partials != nullptr && a.pdl ? 1 : 0;  // a dependent of the reduction
+    cfg.numAttrs = a.pdl ? 1 : 0;  // a programmatic dependent of the previous kernel
     return cudaLaunchKernelEx(&cfg, profile_select_kernel<T>, a);
 }
 
