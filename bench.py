@@ -288,8 +288,11 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
             fd.fdllm_select(h_logits, h_mask, args.param, mode, h_tok, h_commit, h_n)
         t_e2e = time.perf_counter() - t0
         e2e = {"value": w.B * e2e_steps / t_e2e, "unit": UNIT,
-               "h2d_bytes_per_step": h_logits.numel() * h_logits.element_size()
+               # only the masked rows cross the host link (read by the GPU from pinned memory)
+               "h2d_bytes_per_step": masked_rows * w.V * w.elem_bytes
                + h_mask.numel() + h_tok.numel() * 4,
+               "path": "pinned host logits; masked rows read over the host link by "
+                       "fdllm_gather_masked_rows, then fdllm_select; results copied back",
                "d2h_bytes_per_step": h_tok.numel() * 4 + h_commit.numel() + h_n.numel() * 4
                + h_mask.numel(),
                "steps": e2e_steps}

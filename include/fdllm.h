@@ -176,6 +176,17 @@ fdllm_status fdllm_select_from_conf(const float *conf, const int32_t *argmax, in
                                     int32_t *out_tokens, uint8_t *out_commit, int32_t *out_n,
                                     void *stream);
 
+/* Input movement for the end-to-end path (the paper has no counterpart: it moves data, it
+ * computes nothing): copies the rows of the masked positions of `src` [B, L, V] (dtype as
+ * given) to the same offsets of `dst`, a device buffer of the same shape; rows of unmasked
+ * positions of dst are not written.  src may be device memory or page-locked host memory
+ * (cudaHostAlloc / torch pin_memory), which the GPU reads directly over the host link, so
+ * that only the masked rows cross it.  mask [B, L] uint8 device.  Pageable host memory is
+ * rejected (FDLLM_ERR_ARG); src and dst 16-byte aligned, V * sizeof(dtype) a multiple of 16
+ * (FDLLM_ERR_ALIGN).  Asynchronous on `stream`. */
+fdllm_status fdllm_gather_masked_rows(const void *src, void *dst, int dtype, int B, int L, int V,
+                                      const uint8_t *mask, void *stream);
+
 /* Step a1 fused with the LM head (the projection that produces the logits, Sec. 3
  * "Notation": p_i = softmax of the logits of position i), then steps a2-a5 as in
  * fdllm_select.  For every masked position the logits x = W h are computed on the tensor

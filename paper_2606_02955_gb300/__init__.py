@@ -23,6 +23,7 @@ __all__ = [
     "fdllm_version", "library_path", "fdllm_select_static", "fdllm_select_robust",
     "fdllm_profile_terms", "fdllm_check_bounded_wait", "fdllm_decode_loop", "FORWARD_FN",
     "fdllm_lmhead_select", "fdllm_lmhead_confidence", "fdllm_lmhead_logits",
+    "fdllm_gather_masked_rows",
 ]
 
 BF16, FP32 = 0, 1
@@ -65,6 +66,8 @@ def _load():
     lib.fdllm_lmhead_confidence.restype = i
     lib.fdllm_lmhead_logits.argtypes = [p, p, i, i, i, i, p, p, p]
     lib.fdllm_lmhead_logits.restype = i
+    lib.fdllm_gather_masked_rows.argtypes = [p, p, i, i, i, i, p, p]
+    lib.fdllm_gather_masked_rows.restype = i
     lib.fdllm_confidence.argtypes = [p, i, i, i, i, p, p, p, p]
     lib.fdllm_confidence.restype = i
     lib.fdllm_select_from_conf.argtypes = [p, p, i, i, p, d, i, p, p, p, p]
@@ -178,8 +181,16 @@ def fdllm_select(logits: torch.Tensor, mask: torch.Tensor, param: float, mode=PR
 
 def _select_from_host(logits, mask, param, mode, out_tokens, out_commit, out_n):
     dev = torch.device("cuda", torch.cuda.current_device())
-    d_logits = logits.to(dev, non_blocking=True)
     d_mask = mask.to(dev, non_blocking=True)
+    if logits.is_pinned() and logits.is_contiguous():
+        # Page-locked logits: the GPU reads only the masked rows, straight from host memory.
+        B, L, V = logits.shape
+        d_logits = torch.empty(logits.shape, dtype=logits.dtype, device=dev)
+        _check(_load().fdllm_gather_masked_rows(logits.data_ptr(), d_logits.data_ptr(),
+                                                _dtype_code(logits), B, L, V, d_mask.data_ptr(),
+                                                _stream(None)), "fdllm_gather_masked_rows")
+    else:
+        d_logits = logits.to(dev, non_blocking=True)
     B, L, _ = logits.shape
     d_tok = (torch.full((B, L), -1, dtype=torch.int32, device=dev) if out_tokens is None
              else out_tokens.to(dev, non_blocking=True))
@@ -394,6 +405,25 @@ def fdllm_decode_loop(forward, logits: torch.Tensor, gen_len: int, param: float,
                                    ctypes.byref(steps), _stream(stream))
     _check(st, "fdllm_decode_loop")
     return seq, nfe, steps.value
+
+
+def fdllm_gather_masked_rows(src: torch.Tensor, mask: torch.Tensor, dst=None, stream=None):
+    """Copy the masked positions' rows of ``src`` [B, L, V] (a CUDA tensor or a pinned host
+    tensor, read by the GPU directly) into ``dst`` (a CUDA tensor of the same shape and
+    dtype; allocated when None).  Returns dst; its unmasked rows are not written."""
+    if not src.is_cuda and not src.is_pinned():
+        raise ValueError("src must be a CUDA tensor or a pinned host tensor")
+    if not src.is_contiguous():
+        raise ValueError("src must be contiguous")
+    B, L, V = src.shape
+    if dst is None:
+        dst = torch.empty(src.shape, dtype=src.dtype, device=mask.device)
+    _check(_load().fdllm_gather_masked_rows(src.data_ptr(),
+                                            _dev(dst, "dst", src.dtype, (B, L, V)),
+                                            _dtype_code(src), B, L, V,
+                                            _dev(mask, "mask", torch.uint8, (B, L)),
+                                            _stream(stream)), "fdllm_gather_masked_rows")
+    return dst
 
 
 def fdllm_check_bounded_wait(seconds: float = 0.01, stream=None) -> int:

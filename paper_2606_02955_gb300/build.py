@@ -17,7 +17,7 @@ INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 OBJ_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(HERE, "libfdllm.so")
 SOURCES = ["fdllm_abi.cu", "vocab_reduce.cu", "profile_select.cu", "decode_loop.cu",
-           "lmhead.cu"]
+           "lmhead.cu", "host_io.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC]
 

@@ -162,3 +162,17 @@ def test_lmhead_rejects_before_any_device_call(lib):
     assert f(mode=3) == ERR_ARG
     assert f(param=float("nan")) == ERR_ARG
     assert lib.fdllm_lmhead_logits(A16, A16, 2, 32, 64, 1000, A16, None, None) == ERR_ARG
+
+
+def test_gather_masked_rows_rejects(lib):
+    p, i = ctypes.c_void_p, ctypes.c_int
+    lib.fdllm_gather_masked_rows.argtypes = [p, p, i, i, i, i, p, p]
+    f = lambda src=A16, dst=A16, dtype=0, B=2, L=32, V=1024, mask=A16: \
+        lib.fdllm_gather_masked_rows(src, dst, dtype, B, L, V, mask, None)
+    assert f(src=None) == ERR_ARG
+    assert f(mask=None) == ERR_ARG
+    assert f(dtype=2) == ERR_ARG
+    assert f(L=1025) == ERR_ARG
+    assert f(V=1001) == ERR_ALIGN
+    assert f(src=A2) == ERR_ALIGN
+    assert f(dst=A2) == ERR_ALIGN
