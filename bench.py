@@ -600,12 +600,12 @@ def run_lmhead(args) -> dict:
         pass
     peak = float(peaks.get("bf16_tflops", 1900.0))
     t_gemm = t.get("fused_confidence_only", t.get("fused"))
-    achieved = flops / (t_gemm * 1e-3) / 1e12
+    achieved = flops / (t_gemm * 1e-3) / 1e12 if t_gemm else None
     return {
         "metric": "LM head + commit-set selection: ms per step and GEMM TFLOP/s",
         "workload": "lmhead_b%d_l%d_h%d_v%d_bf16" % (B, L, H, V),
         "B": B, "L": L, "H": H, "V": V, "masked_rows": R, "mode": args.mode,
-        "gemm_variant_env": {k: os.environ[k] for k in ("FDLLM_LMHEAD_CLUSTER", "FDLLM_LMHEAD_BN")
+        "gemm_variant_env": {k: os.environ[k] for k in ("FDLLM_LMHEAD_GEMM", "FDLLM_LMHEAD_BN")
                              if k in os.environ},
         "param": args.param, "data": "synthetic",
         "ms_per_step": t,
@@ -617,7 +617,8 @@ def run_lmhead(args) -> dict:
                                       if "cublas_gemm_masked_rows_only" in t else None),
         "identical_decisions_fused_vs_unfused": same,
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                     "frac": achieved / peak, "kernel": "fdllm_lmhead_confidence (compaction, "
+                     "frac": achieved / peak if achieved else None,
+                     "kernel": "fdllm_lmhead_confidence (compaction, "
                      "gather, GEMM with reducing epilogue, combine)",
                      "algorithmic_flops_per_launch": flops,
                      "peak_source": "measured" if "bf16_tflops" in peaks else "fallback"},

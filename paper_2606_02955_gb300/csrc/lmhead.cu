@@ -19,6 +19,7 @@
 #include <cstdint>
 #include <cstdlib>
 #include <mutex>
+#include <string>
 
 #include "fdllm.h"
 #include "fdllm_internal.cuh"
@@ -41,15 +42,25 @@ constexpr uint64_t kDrainLimitNs = 100000000ull;  // waits for own copies after 
 // Vocabulary entries per tile (the MMA's N and the fp32 accumulator's width): 256, or 208,
 // which splits LLaDA's V = 126464 into 608 = 4 x 152 tiles, one whole wave per SM count.
 // The stage count fills the ring budget: 4 x 48 KB at 256, 5 x 42 KB at 208.
-template <int BN_>
+// How the CTAs of a cluster share a W tile.
+enum Mode {
+    kSolo = 0,       // one CTA per work item; it loads the whole W tile
+    kMulticast = 1,  // 2-CTA cluster, two row tiles: each CTA loads half of the W tile and
+                     // multicasts it into both CTAs
+    kPair = 2,       // 2-CTA pair MMA (tcgen05 cta_group::2, M = 256): each CTA holds its 128
+                     // rows and half of the W tile; the even CTA issues the MMAs for both
+};
+
+template <int BN_, int MODE>
 struct TileCfg {
     static constexpr int BN = BN_;
-    static constexpr int kBBytes = BN * BK * 2;
+    static constexpr int kBRows = MODE == kPair ? BN / 2 : BN;  // W rows held per CTA
+    static constexpr int kBBytes = kBRows * BK * 2;
     static constexpr int kStageBytes = kABytes + kBBytes;
     static constexpr int kStages =
-        (int)(kRingBudget / kStageBytes) > 6 ? 6 : (int)(kRingBudget / kStageBytes);
+        (int)(kRingBudget / kStageBytes) > 8 ? 8 : (int)(kRingBudget / kStageBytes);
     static constexpr size_t kSmemBytes = 1024 + (size_t)kStages * kStageBytes + kBarrierBytes;
-    static_assert(BN % 16 == 0 && BN <= (int)kAccStride, "MMA N for M = 128");
+    static_assert(BN % 16 == 0 && BN <= (int)kAccStride, "MMA N");
     static_assert((BN / 2) % 8 == 0, "halves of whole 8-row swizzle atoms");
 };
 
@@ -88,23 +99,29 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity, ui
     }
 }
 
-// CL = 1: every CTA loads its own W tile.  CL = 2: the two CTAs of a cluster take row tiles
-// 2j and 2j + 1 of the same vocabulary tile; each loads half of the W tile and multicasts it
-// into both CTAs' shared memory (half the L2 -> SM traffic for W), and each MMA releases a
-// stage in both CTAs, since either producer overwrites it in both.
-template <int EPI, int CL, int BN_>
+// MODE kSolo: every CTA loads its own W tile.  kMulticast: the two CTAs of a cluster take
+// row tiles 2j and 2j + 1 of the same vocabulary tile; each loads half of the W tile and
+// multicasts it into both CTAs' shared memory (half the L2 -> SM traffic for W), and each
+// MMA releases a stage in both CTAs, since either producer overwrites it in both.  kPair:
+// the same two row tiles form one M = 256 MMA issued by the even CTA (tcgen05 cta_group::2):
+// each CTA loads its 128 rows and half of the W tile into its own shared memory and
+// signals the even CTA's stage barrier, so each CTA's shared memory supplies half the
+// operand bytes per MMA; the accumulators live in both CTAs' tensor memory.
+template <int EPI, int MODE, int BN_>
 __global__ void __launch_bounds__(kThreads, 1)
     lmhead_gemm_kernel(const __grid_constant__ CUtensorMap map_h,
                        const __grid_constant__ CUtensorMap map_w, const GemmArgs a)
 {
-    using Cfg = TileCfg<BN_>;
+    using Cfg = TileCfg<BN_, MODE>;
+    constexpr int CL = MODE == kSolo ? 1 : 2;
+    constexpr bool PAIR = MODE == kPair;
     constexpr int BN = Cfg::BN, kStages = Cfg::kStages;
     constexpr int kBBytes = Cfg::kBBytes, kStageBytes = Cfg::kStageBytes;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *sA = smem;                     // kStages x [BM rows][128 B], 128-byte swizzled
-    uint8_t *sB = smem + kStages * kABytes; // kStages x [BN rows][128 B]
+    uint8_t *sB = smem + kStages * kABytes; // kStages x [kBRows rows][128 B]
     uint64_t *bars = reinterpret_cast<uint64_t *>(sB + kStages * kBBytes);
     uint64_t *full = bars;                  // TMA -> MMA, one per stage
     uint64_t *empty = bars + kStages;       // MMA -> TMA, one per stage
@@ -118,11 +135,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             mbar_init(&full[s], 1);
-            mbar_init(&empty[s], CL);  // one release per consuming CTA
+            mbar_init(&empty[s], MODE == kMulticast ? 2 : 1);  // one release per MMA issuer
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&tfull[i], 1);
-            mbar_init(&tempty[i], 4);  // one arrival per epilogue warp
+            mbar_init(&tempty[i], PAIR ? 8 : 4);  // one arrival per epilogue warp (of the pair)
         }
         mbar_init(done, 1);
         *abort_flag = 0;
@@ -130,8 +147,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc::prefetch_tensormap(&map_h);
         tc::prefetch_tensormap(&map_w);
     }
-    if (warp == 1)
-        tc::tmem_alloc(tmem_slot, kTmemCols);
+    if (warp == 1) {
+        if (PAIR)
+            tc::tmem_alloc_pair(tmem_slot, kTmemCols);
+        else
+            tc::tmem_alloc(tmem_slot, kTmemCols);
+    }
     tc::fence_before_sync();
     __syncthreads();
     if (CL > 1)
@@ -146,6 +167,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int rank = CL > 1 ? (int)tc::cluster_ctarank() : 0;
     const int64_t first = CL > 1 ? (int64_t)tc::cluster_id_x() : (int64_t)blockIdx.x;
     const int64_t stride = CL > 1 ? (int64_t)tc::cluster_count_x() : (int64_t)gridDim.x;
+    // An epilogue warp hands an accumulator back to the MMA issuer (in a pair, the even
+    // CTA's barrier counts the warps of both CTAs).
+    auto release_acc = [](uint64_t *bar, int rk) {
+        if (PAIR && rk != 0)
+            tc::mbar_arrive_remote(tc::map_to_rank(bar, 0));
+        else
+            mbar_arrive(bar);
+    };
     const int R = *a.row_count;
     const int num_m = (R + BM - 1) / BM;
     const int num_mc = (num_m + CL - 1) / CL;  // row-tile groups, one per cluster
@@ -172,14 +201,24 @@ __global__ void __launch_bounds__(kThreads, 1)
                         ok = false;
                         break;
                     }
-                    mbar_arrive_expect_tx(&full[s], kStageBytes);
-                    tc::tma_load_2d(sA + s * kABytes, &map_h, kb * BK, m * BM, &full[s]);
-                    if (CL == 1)
-                        tc::tma_load_2d(sB + s * kBBytes, &map_w, kb * BK, n * BN, &full[s]);
-                    else
-                        tc::tma_load_2d_multicast(sB + s * kBBytes + rank * (kBBytes / CL), &map_w,
-                                                  kb * BK, n * BN + rank * (BN / CL), &full[s],
-                                                  (uint16_t)((1u << CL) - 1u));
+                    if constexpr (PAIR) {
+                        // Both CTAs' bytes complete on the even CTA's barrier, which it arms.
+                        if (rank == 0)
+                            mbar_arrive_expect_tx(&full[s], 2 * kStageBytes);
+                        const uint32_t bar0 = tc::map_to_rank(&full[s], 0);
+                        tc::tma_load_2d_pair(sA + s * kABytes, &map_h, kb * BK, m * BM, bar0);
+                        tc::tma_load_2d_pair(sB + s * kBBytes, &map_w, kb * BK,
+                                             n * BN + rank * (BN / 2), bar0);
+                    } else {
+                        mbar_arrive_expect_tx(&full[s], kStageBytes);
+                        tc::tma_load_2d(sA + s * kABytes, &map_h, kb * BK, m * BM, &full[s]);
+                        if (CL == 1)
+                            tc::tma_load_2d(sB + s * kBBytes, &map_w, kb * BK, n * BN, &full[s]);
+                        else
+                            tc::tma_load_2d_multicast(sB + s * kBBytes + rank * (kBBytes / CL),
+                                                      &map_w, kb * BK, n * BN + rank * (BN / CL),
+                                                      &full[s], (uint16_t)((1u << CL) - 1u));
+                    }
                     used[s] = true;
                     last_ph[s] = ph;
                     if (++s == kStages) {
@@ -188,14 +227,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
             }
-            // No copy of this CTA may still be in flight when it exits.
-            for (int i = 0; i < kStages; ++i)
-                if (used[i])
-                    mbar_wait(&full[i], last_ph[i], a.status, kDrainLimitNs);
+            // No copy of this CTA may still be in flight when it exits (in a pair, the even
+            // CTA's barriers count both CTAs' copies, and the odd CTA leaves only after it,
+            // at the final cluster barrier).
+            if (!PAIR || rank == 0)
+                for (int i = 0; i < kStages; ++i)
+                    if (used[i])
+                        mbar_wait(&full[i], last_ph[i], a.status, kDrainLimitNs);
         }
     } else if (warp == 1) {
-        if (lane == 0) {
-            constexpr uint32_t idesc = tc::idesc_bf16_f32(BM, BN);
+        if (lane == 0 && (!PAIR || rank == 0)) {
+            constexpr uint32_t idesc = tc::idesc_bf16_f32(PAIR ? 2 * BM : BM, BN);
             int s = 0;
             uint32_t ph = 0;
             bool ok = true;
@@ -216,11 +258,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const uint64_t ad = tc::sw128_kmajor_desc(sA + s * kABytes);
                     const uint64_t bd = tc::sw128_kmajor_desc(sB + s * kBBytes);
 #pragma unroll
-                    for (int k = 0; k < BK / 16; ++k)  // K = 16 per MMA: +32 B in the row
-                        tc::mma_bf16(d, ad + 2u * k, bd + 2u * k, idesc, (kb | k) != 0);
+                    for (int k = 0; k < BK / 16; ++k) {  // K = 16 per MMA: +32 B in the row
+                        if constexpr (PAIR)
+                            tc::mma_bf16_pair(d, ad + 2u * k, bd + 2u * k, idesc, (kb | k) != 0);
+                        else
+                            tc::mma_bf16(d, ad + 2u * k, bd + 2u * k, idesc, (kb | k) != 0);
+                    }
                     // The stage is free once these MMAs have read it (in every CTA of the
-                    // cluster: either producer overwrites it in both).
-                    if (CL == 1)
+                    // cluster: either producer overwrites it in both, or each refills its own
+                    // half of the pair's operands).
+                    if constexpr (PAIR)
+                        tc::commit_pair_multicast(&empty[s]);
+                    else if (CL == 1)
                         tc::commit(&empty[s]);
                     else
                         tc::commit_multicast(&empty[s], (uint16_t)((1u << CL) - 1u));
@@ -229,11 +278,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                         ph ^= 1u;
                     }
                 }
-                if (ok)
-                    tc::commit(&tfull[acc]);
+                if (ok) {
+                    if constexpr (PAIR)
+                        tc::commit_pair_multicast(&tfull[acc]);  // both CTAs' accumulators
+                    else
+                        tc::commit(&tfull[acc]);
+                }
             }
             // Tensor memory is freed below only after every MMA issued here has completed.
-            tc::commit(done);
+            if constexpr (PAIR)
+                tc::commit_pair_multicast(done);  // the odd CTA's copy is never waited on
+            else
+                tc::commit(done);
             mbar_wait(done, 0, a.status, kDrainLimitNs);
         }
         __syncwarp();
@@ -293,7 +349,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc::fence_before_sync();
                 __syncwarp();
                 if (lane == 0)
-                    mbar_arrive(&tempty[acc]);
+                    release_acc(&tempty[acc], rank);
                 if (r < R) {
                     UnitPartial p;
                     p.M = nan ? __int_as_float(0x7FC00000) : M;
@@ -318,17 +374,22 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc::fence_before_sync();
                 __syncwarp();
                 if (lane == 0)
-                    mbar_arrive(&tempty[acc]);
+                    release_acc(&tempty[acc], rank);
             }
         }
     }
     if (threadIdx.x == 0)
         pdl_launch_dependents();  // the row combination may start launching
     __syncthreads();
+    if (PAIR)
+        tc::cluster_sync();  // both CTAs are done with the pair's tensor memory
     if (warp == 1) {
         __syncwarp();
         tc::fence_after_sync();
-        tc::tmem_dealloc(tmem_base, kTmemCols);
+        if (PAIR)
+            tc::tmem_dealloc_pair(tmem_base, kTmemCols);
+        else
+            tc::tmem_dealloc(tmem_base, kTmemCols);
     }
     if (CL > 1)
         tc::cluster_sync();  // no CTA leaves while its peer may still write into it
@@ -569,18 +630,22 @@ fdllm_status check_lmhead(const void *hidden, const void *w, int B, int L, int H
     return FDLLM_OK;
 }
 
-// CTAs sharing each W tile load: 2 (halves multicast) when at least 8 row tiles can share
-// every W tile, where halving the L2 -> SM traffic for W paid off on GB300 (B = 64, L = 32);
-// 1 below that, where the pairs' padding row tile costs more.  FDLLM_LMHEAD_CLUSTER = 1 or
-// 2 forces one.
-int cluster_size(int64_t rows)
+// The GEMM variant: kPair (cta_group::2) when at least 8 row tiles can share every W tile,
+// kSolo below that (the pair pads to an even number of row tiles, and W streaming from HBM,
+// not shared-memory bandwidth, is the limit there).  FDLLM_LMHEAD_GEMM = solo, multicast or
+// pair forces one.
+int gemm_mode(int64_t rows)
 {
-    if (const char *e = std::getenv("FDLLM_LMHEAD_CLUSTER")) {
-        const int f = std::atoi(e);
-        if (f == 1 || f == 2)
-            return f;
+    if (const char *e = std::getenv("FDLLM_LMHEAD_GEMM")) {
+        const std::string v(e);
+        if (v == "solo")
+            return kSolo;
+        if (v == "multicast")
+            return kMulticast;
+        if (v == "pair")
+            return kPair;
     }
-    return (rows + BM - 1) / BM >= 8 ? 2 : 1;
+    return (rows + BM - 1) / BM >= 8 ? kPair : kSolo;
 }
 
 int sm_count()
@@ -621,10 +686,11 @@ int choose_bn(int64_t rows, int V)
     return best;
 }
 
-template <int EPI, int CL, int BN>
+template <int EPI, int MODE, int BN>
 cudaError_t launch_gemm_cfg(const CUtensorMap &mh, const CUtensorMap &mw, const GemmArgs &g,
                             cudaStream_t stream)
 {
+    constexpr int CL = MODE == kSolo ? 1 : 2;
     static std::once_flag once[64];
     static int grid[64];
     int dev = 0;
@@ -633,8 +699,8 @@ cudaError_t launch_gemm_cfg(const CUtensorMap &mh, const CUtensorMap &mw, const 
         return err;
     if (dev < 0 || dev >= 64)
         return cudaErrorInvalidDevice;
-    auto kern = lmhead_gemm_kernel<EPI, CL, BN>;
-    constexpr size_t smem = TileCfg<BN>::kSmemBytes;
+    auto kern = lmhead_gemm_kernel<EPI, MODE, BN>;
+    constexpr size_t smem = TileCfg<BN, MODE>::kSmemBytes;
     cudaLaunchConfig_t cfg = {};
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = smem;
@@ -663,15 +729,23 @@ cudaError_t launch_gemm_cfg(const CUtensorMap &mh, const CUtensorMap &mw, const 
     return cudaLaunchKernelEx(&cfg, kern, mh, mw, g);
 }
 
+template <int EPI, int MODE>
+cudaError_t launch_gemm_mode(const CUtensorMap &mh, const CUtensorMap &mw, const GemmArgs &g,
+                             int bn, cudaStream_t stream)
+{
+    return bn == 208 ? launch_gemm_cfg<EPI, MODE, 208>(mh, mw, g, stream)
+                     : launch_gemm_cfg<EPI, MODE, 256>(mh, mw, g, stream);
+}
+
 template <int EPI>
 cudaError_t launch_gemm(const CUtensorMap &mh, const CUtensorMap &mw, const GemmArgs &g,
-                        int cl, int bn, cudaStream_t stream)
+                        int mode, int bn, cudaStream_t stream)
 {
-    if (bn == 208)
-        return cl == 1 ? launch_gemm_cfg<EPI, 1, 208>(mh, mw, g, stream)
-                       : launch_gemm_cfg<EPI, 2, 208>(mh, mw, g, stream);
-    return cl == 1 ? launch_gemm_cfg<EPI, 1, 256>(mh, mw, g, stream)
-                   : launch_gemm_cfg<EPI, 2, 256>(mh, mw, g, stream);
+    switch (mode) {
+    case kPair: return launch_gemm_mode<EPI, kPair>(mh, mw, g, bn, stream);
+    case kMulticast: return launch_gemm_mode<EPI, kMulticast>(mh, mw, g, bn, stream);
+    default: return launch_gemm_mode<EPI, kSolo>(mh, mw, g, bn, stream);
+    }
 }
 
 // Steps 1-3 (and 4 for the reduce epilogue) on the owned workspace.
@@ -692,9 +766,10 @@ fdllm_status run_lmhead(const void *hidden, const void *w, int B, int L, int H, 
     int32_t *row_ids = reinterpret_cast<int32_t *>(ws + lay.row_ids);
     uint8_t *packed = ws + lay.packed;
 
-    const int cl = cluster_size(rows);
+    const int mode = gemm_mode(rows);
     CUtensorMap mh, mw;
-    if (!make_map(&mh, packed, H, rows, BM) || !make_map(&mw, w, H, V, bn / cl))
+    if (!make_map(&mh, packed, H, rows, BM) ||
+        !make_map(&mw, w, H, V, mode == kSolo ? bn : bn / 2))
         return FDLLM_ERR_CUDA;
 
     if (launch_pdl(compact_rows_kernel, 1, 1024, s, mask, (int)rows, row_ids, row_count) !=
@@ -713,8 +788,8 @@ fdllm_status run_lmhead(const void *hidden, const void *w, int B, int L, int H, 
     g.partials = reinterpret_cast<UnitPartial *>(ws + lay.partials);
     g.logits = out_logits;
     g.status = reinterpret_cast<uint32_t *>(ws);
-    const cudaError_t e = epi == kReduce ? launch_gemm<kReduce>(mh, mw, g, cl, bn, s)
-                                         : launch_gemm<kStore>(mh, mw, g, cl, bn, s);
+    const cudaError_t e = epi == kReduce ? launch_gemm<kReduce>(mh, mw, g, mode, bn, s)
+                                         : launch_gemm<kStore>(mh, mw, g, mode, bn, s);
     if (e != cudaSuccess)
         return FDLLM_ERR_CUDA;
     if (epi == kReduce) {

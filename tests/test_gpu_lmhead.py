@@ -28,13 +28,13 @@ pytestmark = pytest.mark.gpu
 U = 2.0 ** -23
 
 
-@pytest.fixture(params=[(1, 256), (2, 256), (1, 208), (2, 208)],
-                ids=["cta1-n256", "cluster2-n256", "cta1-n208", "cluster2-n208"])
+@pytest.fixture(params=[(g, bn) for bn in (256, 208) for g in ("solo", "multicast", "pair")],
+                ids=lambda p: "%s-n%d" % p)
 def cluster(request, monkeypatch):
-    """Every GEMM variant: one CTA per W tile or W halves multicast across a 2-CTA cluster,
-    with vocabulary tiles of 256 or 208 entries."""
-    cl, bn = request.param
-    monkeypatch.setenv("FDLLM_LMHEAD_CLUSTER", str(cl))
+    """Every GEMM variant: one CTA per W tile, W halves multicast across a 2-CTA cluster, or
+    a CTA-pair MMA (M = 256), with vocabulary tiles of 256 or 208 entries."""
+    mode, bn = request.param
+    monkeypatch.setenv("FDLLM_LMHEAD_GEMM", mode)
     monkeypatch.setenv("FDLLM_LMHEAD_BN", str(bn))
     return request.param
 
