@@ -39,7 +39,9 @@ METRIC = ("decode-step selections/sec and logits HBM GB/s (fraction of GB300 pea
 UNIT = "selections/s"
 FALLBACK_HBM_GBS = 6800.0
 PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "vocab_reduce_serving_b64_l32_bf16.md")
-KERNEL_SOURCE = os.path.join(ROOT, "paper_2606_02955_gb300", "csrc", "vocab_reduce.cu")
+# the vocab reduction's sources: the kernel and the unit plan it shares with the interface
+KERNEL_SOURCES = [os.path.join(ROOT, "paper_2606_02955_gb300", "csrc", f)
+                  for f in ("vocab_reduce.cu", "fdllm_internal.cuh")]
 
 
 # ----------------------------------------------------------------------------- host logic
@@ -76,10 +78,13 @@ def peak_hbm_gbs():
 
 def ncu_traffic():
     """DRAM traffic per vocab-reduction launch from the committed ncu summary, only while
-    the kernel source is the one the counters were taken on."""
+    the kernel's sources (hashed in order) are the ones the counters were taken on."""
     try:
         text = open(PROFILE_SUMMARY).read()
-        sha = hashlib.sha256(open(KERNEL_SOURCE, "rb").read()).hexdigest()
+        h = hashlib.sha256()
+        for f in KERNEL_SOURCES:
+            h.update(open(f, "rb").read())
+        sha = h.hexdigest()
     except OSError:
         return None
     m_sha = re.search(r"source_sha256:\s*([0-9a-f]{64})", text)

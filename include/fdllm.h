@@ -141,9 +141,9 @@ fdllm_status fdllm_select_robust(const void *logits, int dtype, int B, int L, in
  * array of FDLLM_STATIC_SCRATCH_BYTES bytes compiled into the library; every GPU that loads
  * the library holds it until the process exits.  A shape whose scratch need,
  * fdllm_workspace_bytes(B, L, V, dtype), exceeds that size is rejected with
- * FDLLM_ERR_WORKSPACE before anything is enqueued.  8 MiB covers, for example, every bf16
- * shape with V <= 126464 (up to B * L = 65536 rows) and fp32 V = 126464 up to
- * B * L = 32768 rows.
+ * FDLLM_ERR_WORKSPACE before anything is enqueued.  8 MiB covers, for example, every shape
+ * with V <= 126464 in bf16 or fp32 (up to B * L = 65536 rows), and fp32 V = 2^20 up to
+ * B * L = 16383 rows.
  * The call allocates nothing: no cudaMalloc, no cudaFree, no allocating library routine.
  *
  * The first call on a device looks up the array's device address (cudaGetSymbolAddress)

@@ -17,7 +17,7 @@ namespace fdllm {
 // reduced by one CTA in a fixed order, so a row's result depends only on its bytes.  The
 // CTA streams a unit through a ring of shared-memory chunk buffers.
 constexpr int kSegQueue = 8;  // unit results queued from math warps to the epilogue warp
-constexpr int64_t kUnitTargetBytes = 65536;
+constexpr int64_t kUnitTargetBytes = 131072;
 constexpr int kMaxGrid = 1024;
 constexpr int kMaxRows = 65536;
 constexpr int kMaskWords = kMaxRows / 32;

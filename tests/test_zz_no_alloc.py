@@ -67,7 +67,7 @@ def test_static_scratch_matches_select_on_two_calls(fd, name, mode, param):
 def test_static_scratch_rejects_shapes_beyond_its_size(cuda_lib_path):
     """Checked on the host before any device work: fake, never-dereferenced addresses."""
     lib = _c_entry(cuda_lib_path)
-    B, L, V, dtype = 64, 1024, 126464, 1  # fp32: 8 MiB of unit partials + header
+    B, L, V, dtype = 64, 1024, 1 << 20, 1  # fp32 rows of 4 MiB: 32 MiB of unit partials
     assert lib.fdllm_workspace_bytes(B, L, V, dtype) > STATIC_BYTES
     a16 = 0x10000
     st = lib.fdllm_select_static(a16, dtype, B, L, V, a16, 1.0, 0, a16, a16, a16, None)
