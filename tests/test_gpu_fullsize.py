@@ -97,24 +97,34 @@ def test_full_sequence_first_step_full_size(fd, orc):
 @pytest.mark.parametrize("mode", [PROFILE, FACTOR])
 def test_full_sequence_loop_until_done(fd, orc, mode):
     """Selection + commit until no mask remains (B = 16, L = 1024, fp32, logits regenerated
-    from (seed, step) every step).  Every step commits >= 1 position per unmasked-remaining
-    row and only masked ones; all rows finish within L steps; sampled steps match the
-    oracle on one row."""
+    from (seed, step) every step), checked three ways:
+      * every step, every row: >= 1 commit per row with masked positions left, commits only
+        at masked positions, the mask updated by exactly the commits; all rows finish
+        within L steps;
+      * every step, two complete row trajectories: the GPU's decision equals the oracle's
+        rule applied to the GPU's confidences on the GPU's mask state;
+      * every 64th step, all rows: the confidences and argmax of 8 sampled masked positions
+        per row against the oracle on the same logits; and one row's whole decision
+        against the oracle from the logits."""
     w = syn.WORKLOADS["full_seq_b16_l1024_fp32"]
     B, L = w.B, w.L
+    traj = (3, 11)
+    rng = np.random.default_rng(7)
     mask = torch.ones((B, L), dtype=torch.uint8, device="cuda")
     tokens = torch.full((B, L), -1, dtype=torch.int32, device="cuda")
     commit = torch.empty((B, L), dtype=torch.uint8, device="cuda")
     n = torch.empty((B,), dtype=torch.int32, device="cuda")
+    conf = torch.empty((B, L), dtype=torch.float32, device="cuda")
+    amax = torch.empty((B, L), dtype=torch.int32, device="cuda")
     committed_total = np.zeros(B, np.int64)
     step = 0
-    check_steps = {0, 1, 7, 100, 511}
     while True:
         before = mask.cpu().numpy()
         if before.sum() == 0:
             break
         assert step < L, "loop did not finish within L steps"
         logits = syn.make_logits(w, seed=99, device="cuda", step=step)
+        fd.fdllm_confidence(logits, mask, conf, amax)
         fd.fdllm_select(logits, mask, 1.0, mode, tokens, commit, n)
         after, c, nn = mask.cpu().numpy(), commit.cpu().numpy(), n.cpu().numpy()
         live = before.sum(1) > 0
@@ -122,8 +132,34 @@ def test_full_sequence_loop_until_done(fd, orc, mode):
         assert np.array_equal(c.sum(1), nn)
         assert np.all(before[c == 1] == 1) and np.array_equal(after, before & (1 - c))
         committed_total += nn
-        if step in check_steps:
-            b = step % B
+        # two trajectories: the rule on the GPU's own confidences, every step
+        g_conf = conf.cpu().numpy().astype(np.float64)
+        g_amax = amax.cpu().numpy()
+        rows = list(traj)
+        rg = orc.select_from_conf(g_conf[rows], g_amax[rows], before[rows], mode, 1.0)
+        for k, b in enumerate(rows):
+            if rg["margin"][k] >= 1e-12:
+                assert nn[b] == rg["n"][k], "step %d row %d" % (step, b)
+                assert np.array_equal(c[b], rg["commit"][k]), "step %d row %d" % (step, b)
+        if step % 64 == 0:
+            # sampled confidences of every row against the oracle on the same bytes
+            picks = []
+            for b in range(B):
+                pos = np.nonzero(before[b])[0]
+                if pos.size:
+                    for l in rng.choice(pos, size=min(8, pos.size), replace=False):
+                        picks.append((b, int(l)))
+            bi = torch.tensor([p[0] for p in picks], device="cuda")
+            li = torch.tensor([p[1] for p in picks], device="cuda")
+            sample = logits[bi, li][None]  # [1, k, V]
+            rc, rt, _ = orc.confidence(syn.host_bits(sample), np.ones((1, len(picks)), np.uint8),
+                                       nthreads=oracle_threads())
+            gc = np.array([g_conf[b, l] for b, l in picks])
+            gt = np.array([g_amax[b, l] for b, l in picks])
+            assert np.array_equal(gt, rt[0])
+            assert (np.abs(gc - rc[0]) / rc[0]).max() <= CONF_RTOL
+            # one row's whole decision from the logits
+            b = (step // 64) % B
             ref = orc.select(syn.host_bits(logits[b:b + 1]), before[b:b + 1], mode, 1.0,
                              nthreads=oracle_threads())
             if ref["margin"][0] >= MARGIN:
