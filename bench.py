@@ -265,6 +265,17 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
     t_step, tw0, tw1 = timed(step_run, replays)
     k1_run = make_runner(k1_only, per_replay)
     t_k1, _, _ = timed(k1_run, replays)
+    # distribution of the step time: replays timed one by one (outside the timed region)
+    per_step_us = []
+    for r in range(min(200, replays)):
+        a0 = torch.cuda.Event(enable_timing=True)
+        a1 = torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        with torch.cuda.stream(stream):
+            step_run(r)
+        a1.record(stream)
+        a1.synchronize()
+        per_step_us.append(a0.elapsed_time(a1) * 1e3 / per_replay)
     if sampler is not None:
         time.sleep(0.12)
         sampler.stop()
@@ -321,6 +332,11 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
                 "masked_rows_per_step": masked_rows,
                 "logits_bytes_per_step": alg_bytes,
                 "logits_gbs_per_step": alg_bytes / (ms_per_step * 1e-3) / 1e9,
+                "positions_per_s": masked_rows * world / (ms_per_step * 1e-3),
+                "step_us_distribution": {
+                    "median": float(np.median(per_step_us)), "min": float(min(per_step_us)),
+                    "max": float(max(per_step_us)), "replays": len(per_step_us),
+                    "steps_per_replay": per_replay},
                 "l2_policy": "inputs larger than L2: %d rotating logits buffers of %.0f MB "
                              "(%.2f GB > 129 MB L2)" % (n_buf, bufs[0].numel() *
                                                         bufs[0].element_size() / 1e6,
@@ -332,6 +348,7 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
             "roofline": {
                 "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak, "traffic": traffic,
+                "frac_of_nominal_7900_gbs": achieved / 7900.0,
                 "kernel": "vocab_reduce (a1), timed with its finalize pass",
                 "kernel_us": k1_s * 1e6, "peak_source": peak_kind,
                 "algorithmic_bytes_per_launch": alg_bytes,
@@ -675,6 +692,13 @@ def run_oracle_timed(args, steps: int, warmup: int, budget_s: float | None):
         if budget_s is None and done >= steps:
             break
     t = time.perf_counter() - t0
+    # the same oracle on one thread, one step
+    t1 = time.perf_counter()
+    if args.mode == "robust":
+        orc.select_robust(host, mask, args.param, args.eta, None, nthreads=1)
+    else:
+        orc.select(host, mask, mode, args.param, nthreads=1)
+    t_single = time.perf_counter() - t1
     cpu = "unknown"
     try:
         for line in open("/proc/cpuinfo"):
@@ -683,12 +707,23 @@ def run_oracle_timed(args, steps: int, warmup: int, budget_s: float | None):
                 break
     except OSError:
         pass
+    if cpu == "unknown":
+        try:
+            out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+            for line in out.splitlines():
+                if line.strip().lower().startswith(("model name", "vendor id")):
+                    cpu = line.split(":", 1)[1].strip()
+                    if line.strip().lower().startswith("model name"):
+                        break
+        except (OSError, subprocess.SubprocessError):
+            pass
     return {
         "value": rows * done / t, "unit": UNIT, "cores": threads, "kind": "oracle",
         "sample": "%d batch rows of %s drawn by its recipe (%d masked positions of V=%d) "
                   "per step, %d steps, fp64 C oracle with OpenMP over positions"
                   % (rows, w.name, int(mask.sum()), w.V, done),
         "seconds": t, "steps": done, "cpu": cpu,
+        "single_thread_value": rows / t_single,
     }
 
 
@@ -738,7 +773,7 @@ def main(argv=None):
                     help="time a whole generation through the device-resident decode loop "
                          "and through a host-driven loop, instead of the throughput line")
     ap.add_argument("--loop-batch", type=int, default=8)
-    ap.add_argument("--gen-len", type=int, default=256)
+    ap.add_argument("--gen-len", type=int, nargs="+", default=[256, 512, 1024])
     ap.add_argument("--block-len", type=int, default=32)
     ap.add_argument("--peak", type=float, default=20.0,
                     help="decode loop: largest planted logit height of the synthetic forward")
@@ -756,7 +791,15 @@ def main(argv=None):
         print(json.dumps(run_lmhead(args)), flush=True)
         return
     if args.decode_loop:
-        print(json.dumps(run_decode_loop(args)), flush=True)
+        lengths = list(args.gen_len)
+        runs = []
+        for g in lengths:
+            args.gen_len = g
+            runs.append(run_decode_loop(args))
+        out = runs[0] if len(runs) == 1 else {
+            "metric": runs[0]["metric"], "data": "synthetic",
+            "workloads": runs}
+        print(json.dumps(out), flush=True)
         return
     if args.loop:
         if args.workload == "serving_b64_l32_bf16":
