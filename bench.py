@@ -434,17 +434,46 @@ def run_decode_loop(args) -> dict:
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     B, gen, Lb, V = args.loop_batch, args.gen_len, args.block_len, syn.LLADA_VOCAB
+    H = syn.LLADA_HIDDEN
     seed, peak = 2024, args.peak
     mode = fd.MODES[args.mode]
-    logits = torch.empty((B, Lb, V), dtype=torch.bfloat16, device=dev)
+    lm = args.loop_lmhead
     stream = torch.cuda.current_stream()
+    if lm:
+        # the forward pass writes hidden states; the LM head (tcgen05) runs in the loop body
+        _, w_vocab, _ = syn.make_lmhead_inputs(1, 1, H, V, seed=7, device=dev)
+        logits = torch.empty((B, Lb, H), dtype=torch.bfloat16, device=dev)
 
-    def forward(state, mask, out, strm):
-        syn.synth_block_logits_gpu(out, mask, B, Lb, V, seed, step_ptr=state, peak_max=peak,
-                                   stream_ptr=strm)
+        def forward(state, mask, out, strm):
+            syn.synth_block_hidden_gpu(out, mask, B, Lb, H, V, w_vocab.data_ptr(), seed,
+                                       step_ptr=state, beta_max=peak, stream_ptr=strm)
 
-    def device_loop():
-        return fd.fdllm_decode_loop(forward, logits, gen, args.param, mode)
+        def forward_step(step):
+            syn.synth_block_hidden_gpu(logits.data_ptr(), mask.data_ptr(), B, Lb, H, V,
+                                       w_vocab.data_ptr(), seed, step=step, beta_max=peak,
+                                       stream_ptr=stream.cuda_stream)
+
+        def select_step():
+            fd.fdllm_lmhead_select(logits, w_vocab, mask, args.param, mode, tok, commit, n)
+
+        def device_loop():
+            return fd.fdllm_decode_loop_lmhead(forward, logits, w_vocab, gen, args.param, mode)
+    else:
+        logits = torch.empty((B, Lb, V), dtype=torch.bfloat16, device=dev)
+
+        def forward(state, mask, out, strm):
+            syn.synth_block_logits_gpu(out, mask, B, Lb, V, seed, step_ptr=state,
+                                       peak_max=peak, stream_ptr=strm)
+
+        def forward_step(step):
+            syn.synth_block_logits_gpu(logits.data_ptr(), mask.data_ptr(), B, Lb, V, seed,
+                                       step=step, peak_max=peak, stream_ptr=stream.cuda_stream)
+
+        def select_step():
+            fd.fdllm_select(logits, mask, args.param, mode, tok, commit, n)
+
+        def device_loop():
+            return fd.fdllm_decode_loop(forward, logits, gen, args.param, mode)
 
     seq_h = torch.empty((B, gen), dtype=torch.int32, device=dev)
     mask = torch.empty((B, Lb), dtype=torch.uint8, device=dev)
@@ -459,10 +488,8 @@ def run_decode_loop(args) -> dict:
             mask.fill_(1)
             k = 0
             while bool(mask.any().item()):
-                syn.synth_block_logits_gpu(logits.data_ptr(), mask.data_ptr(), B, Lb, V, seed,
-                                           step=step, peak_max=peak,
-                                           stream_ptr=stream.cuda_stream)
-                fd.fdllm_select(logits, mask, args.param, mode, tok, commit, n)
+                forward_step(step)
+                select_step()
                 view = seq_h[:, blk * Lb:(blk + 1) * Lb]
                 view.copy_(torch.where(commit.bool(), tok, view))
                 step += 1
@@ -491,8 +518,11 @@ def run_decode_loop(args) -> dict:
     tokens = B * gen
     return {
         "metric": "decode loop: generated tokens/s on a synthetic forward pass",
-        "workload": "decode_loop_b%d_gen%d_block%d_bf16" % (B, gen, Lb),
+        "workload": "decode_loop%s_b%d_gen%d_block%d_bf16" % ("_lmhead_h%d" % H if lm else "",
+                                                              B, gen, Lb),
         "B": B, "gen_len": gen, "block_len": Lb, "V": V, "dtype": "bf16",
+        "forward": ("hidden states [B, 32, 4096] + the LM head fused with the selection"
+                    if lm else "logits [B, 32, V]"),
         "mode": args.mode, "param": args.param, "peak": peak, "data": "synthetic",
         "steps": int(steps_d), "nfe_per_block": [int(x) for x in nfe_d.cpu().numpy()],
         "tokens_per_step": gen / max(int(steps_d), 1),
@@ -778,6 +808,9 @@ def main(argv=None):
     ap.add_argument("--peak", type=float, default=20.0,
                     help="decode loop: largest planted logit height of the synthetic forward")
     ap.add_argument("--repeats", type=int, default=5)
+    ap.add_argument("--loop-lmhead", action="store_true",
+                    help="decode loop: the forward pass writes hidden states and the LM head "
+                         "(H = 4096) runs fused with the selection inside the loop")
     ap.add_argument("--warmup-loops", type=int, default=2)
     ap.add_argument("--lmhead", action="store_true",
                     help="time the LM-head-fused selection against unfused paths, instead of "

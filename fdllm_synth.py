@@ -251,6 +251,9 @@ def _synth_lib():
         lib.fdllm_synth_block_logits.argtypes = [p, p, i, i, i, ctypes.c_ulonglong, p,
                                                  ctypes.c_longlong, ctypes.c_double, p]
         lib.fdllm_synth_block_logits.restype = i
+        lib.fdllm_synth_block_hidden.argtypes = [p, p, i, i, i, i, p, ctypes.c_ulonglong, p,
+                                                 ctypes.c_longlong, ctypes.c_double, p]
+        lib.fdllm_synth_block_hidden.restype = i
         _synth = lib
     return _synth
 
@@ -263,3 +266,14 @@ def synth_block_logits_gpu(out_ptr, mask_ptr, B, L, V, seed, step_ptr=None, step
                                                 int(step), float(peak_max), stream_ptr)
     if err != 0:
         raise RuntimeError("synthetic logits launch failed: %d" % err)
+
+
+def synth_block_hidden_gpu(out_ptr, mask_ptr, B, L, H, V, w_ptr, seed, step_ptr=None, step=0,
+                           beta_max=16.0, stream_ptr=None):
+    """Enqueue counter-based bf16 hidden states [B, L, H] against the bf16 head w [V, H]
+    (raw device pointers; rows whose mask byte is 0 are skipped; the step is read from
+    step_ptr on the device when given)."""
+    err = _synth_lib().fdllm_synth_block_hidden(out_ptr, mask_ptr, B, L, H, V, w_ptr, int(seed),
+                                                step_ptr, int(step), float(beta_max), stream_ptr)
+    if err != 0:
+        raise RuntimeError("synthetic hidden-state launch failed: %d" % err)

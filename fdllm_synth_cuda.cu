@@ -65,9 +65,72 @@ __global__ void synth_block_logits(__nv_bfloat16 *out, const uint8_t *mask, int 
     }
 }
 
+// Hidden states with a planted target (the LM-head counterpart of synth_block_logits).
+// For row (b, l): k as above, p = mix(k ^ 0xD1B54A32D192ED03), target t = p % V, height
+// beta = float(p >> 40) * fl32(beta_max / 2^24); noise z_j as the logits noise at index j;
+// n2 = |w_t|^2 in fp32, lane i of 32 summing w_tj^2 for j = i, i + 32, ... in order, then an
+// xor butterfly over offsets 16, 8, 4, 2, 1; scale = beta / n2 (IEEE division);
+// h_j = z_j + scale * w_tj (each operation rounded to fp32), stored as bf16 (nearest even).
+// Then w_t . h ~ beta + N(0, 1): a planted peak at t in the logits x = W h.
+__global__ void synth_block_hidden(__nv_bfloat16 *out, const uint8_t *mask, int B, int L, int H,
+                                   int V, const __nv_bfloat16 *w, uint64_t seed,
+                                   const int32_t *step_ptr, int64_t step_const,
+                                   float noise_scale, float beta_scale)
+{
+    __shared__ float s_scale;
+    const int row = blockIdx.x;
+    if (row >= B * L || (mask != nullptr && mask[row] == 0))
+        return;
+    const int b = row / L, l = row % L;
+    const uint64_t step = step_ptr != nullptr ? (uint64_t)step_ptr[0] : (uint64_t)step_const;
+    const uint64_t k = row_key(seed, step, (uint32_t)b, (uint32_t)l);
+    const uint64_t p = mix64(k ^ 0xD1B54A32D192ED03ull);
+    const int64_t t = (int64_t)(p % (uint64_t)V);
+    const float beta = __fmul_rn((float)(p >> 40), beta_scale);
+    const __nv_bfloat16 *wt = w + t * H;
+    if (threadIdx.x < 32) {
+        float acc = 0.0f;
+        for (int j = threadIdx.x; j < H; j += 32) {
+            const float x = __bfloat162float(wt[j]);
+            acc = __fadd_rn(acc, __fmul_rn(x, x));
+        }
+        for (int o = 16; o > 0; o >>= 1)
+            acc = __fadd_rn(acc, __shfl_xor_sync(0xFFFFFFFFu, acc, o));
+        if (threadIdx.x == 0)
+            s_scale = __fdiv_rn(beta, acc);
+    }
+    __syncthreads();
+    const float scale = s_scale;
+    __nv_bfloat16 *o = out + (int64_t)row * H;
+    for (int j = threadIdx.x; j < H; j += blockDim.x) {
+        const uint64_t h = mix64(k + (uint64_t)(j + 1) * kGolden);
+        const int32_t sv = (int32_t)(2 * (h & 0xFFFF) + 2 * ((h >> 16) & 0xFFFF) +
+                                     2 * ((h >> 32) & 0xFFFF) + 2 * ((h >> 48) & 0xFFFF) + 4) -
+                           262144;
+        const float z = __fmul_rn((float)sv, noise_scale);
+        o[j] = __float2bfloat16_rn(__fadd_rn(z, __fmul_rn(scale, __bfloat162float(wt[j]))));
+    }
+}
+
 }  // namespace
 
 extern "C" {
+
+// Enqueue synthetic bf16 hidden states [B, L, H] for the masked rows against the bf16 head
+// w [V, H]; the step as for fdllm_synth_block_logits.
+int fdllm_synth_block_hidden(void *out, const uint8_t *mask, int B, int L, int H, int V,
+                             const void *w, unsigned long long seed, const int32_t *step_ptr,
+                             long long step_const, double beta_max, void *stream)
+{
+    const float noise_scale = (float)(1.7320508075688772 / 131072.0);
+    const float beta_scale = (float)(beta_max / 16777216.0);
+    synth_block_hidden<<<B * L, 128, 0, static_cast<cudaStream_t>(stream)>>>(
+        static_cast<__nv_bfloat16 *>(out), mask, B, L, H, V,
+        static_cast<const __nv_bfloat16 *>(w), seed, step_ptr, step_const, noise_scale,
+        beta_scale);
+    return (int)cudaGetLastError();
+}
+
 
 // Enqueue synthetic bf16 logits [B, L, V] for the masked rows (mask may be NULL: all rows).
 // The step comes from device memory (step_ptr, read when the kernel runs, so a captured

@@ -257,6 +257,17 @@ fdllm_status fdllm_decode_loop(int B, int gen_len, int block_len, int V, int dty
                                void *logits, int32_t *seq_tokens, int32_t *nfe_per_block,
                                int max_steps, int *out_steps, void *stream);
 
+/* fdllm_decode_loop with the LM head inside the loop body: the forward pass writes the final
+ * hidden states [B, block_len, H] bf16 into `hidden` (rows with block_mask != 0), and each
+ * step's selection is fdllm_lmhead_select against w_vocab [V, H] bf16 (the logits never
+ * reach memory).  Arguments, limits and errors otherwise as fdllm_decode_loop and
+ * fdllm_lmhead_select (H a multiple of 8; w_vocab NULL: FDLLM_ERR_ARG). */
+fdllm_status fdllm_decode_loop_lmhead(int B, int gen_len, int block_len, int H, int V,
+                                      const void *w_vocab, double param, int mode,
+                                      fdllm_forward_fn forward, void *user, void *hidden,
+                                      int32_t *seq_tokens, int32_t *nfe_per_block, int max_steps,
+                                      int *out_steps, void *stream);
+
 /* Heterogeneity-bonus diagnostics (Prop. heterogeneity-bonus, Eq. heterogeneity_decomp,
  * Remark adaptive-factor).  For each batch row, the masked confidences are sorted as the
  * selection sorts them (descending, ties: lower position first); at rank n = 1..m_b:

@@ -98,6 +98,8 @@ class Oracle:
         lib.oracle_synth_block_logits.restype = None
         lib.oracle_decode_loop.argtypes = [i64, i64, i64, i64, i32, d, u64, d, i64, p, p, p, i32]
         lib.oracle_decode_loop.restype = i64
+        lib.oracle_synth_block_hidden.argtypes = [p, p, i64, i64, i64, i64, p, u64, u64, d]
+        lib.oracle_synth_block_hidden.restype = None
         lib.oracle_lmhead_logits.argtypes = [p, p, i64, i64, i64, p, p, p, i32]
         lib.oracle_lmhead_logits.restype = None
         self.lib = lib
@@ -160,6 +162,17 @@ class Oracle:
                                       None if m is None else _ptr(m), _ptr(out),
                                       None if mag is None else _ptr(mag), int(nthreads))
         return (out, mag) if with_abs else out
+
+    def synth_block_hidden(self, w_bits, B, L, seed, step, beta_max, mask=None):
+        """Counter-based synthetic bf16 hidden states (uint16 bits [B, L, H]) against the
+        bf16 head w (uint16 bits [V, H]); unmasked rows zero."""
+        w = np.ascontiguousarray(w_bits, np.uint16)
+        V, H = w.shape
+        out = np.zeros((B, L, H), np.uint16)
+        m = None if mask is None else np.ascontiguousarray(mask, np.uint8).reshape(B, L)
+        self.lib.oracle_synth_block_hidden(_ptr(out), None if m is None else _ptr(m), B, L, H,
+                                           V, _ptr(w), int(seed), int(step), float(beta_max))
+        return out
 
     def synth_block_logits(self, B, L, V, seed, step, peak_max, mask=None):
         """Counter-based synthetic bf16 logits (uint16 bits [B, L, V]); unmasked rows zero."""

@@ -537,3 +537,53 @@ void oracle_lmhead_logits(const uint16_t *hidden, const uint16_t *w, int64_t row
         free(h);
     }
 }
+
+void oracle_synth_block_hidden(uint16_t *out, const uint8_t *mask, int64_t B, int64_t L,
+                               int64_t H, int64_t V, const uint16_t *w, uint64_t seed,
+                               uint64_t step, double beta_max)
+{
+    const uint64_t G = 0x9E3779B97F4A7C15ull;
+    const float noise_scale = (float)(sqrt(3.0) / 131072.0);
+    const float beta_scale = (float)(beta_max / 16777216.0);
+    for (int64_t b = 0; b < B; ++b)
+        for (int64_t l = 0; l < L; ++l) {
+            const int64_t row = b * L + l;
+            if (mask && !mask[row])
+                continue;
+            const uint64_t k = splitmix_mix(
+                seed ^ splitmix_mix(step * G ^ splitmix_mix(((uint64_t)b << 32) | (uint64_t)l)));
+            const uint64_t p = splitmix_mix(k ^ 0xD1B54A32D192ED03ull);
+            const int64_t t = (int64_t)(p % (uint64_t)V);
+            const float beta = (float)(p >> 40) * beta_scale;
+            const uint16_t *wt = w + t * H;
+            float lane[32];
+            for (int i = 0; i < 32; ++i) {
+                float acc = 0.0f;
+                for (int64_t j = i; j < H; j += 32) {
+                    const float x = (float)bf16_to_double(wt[j]);
+                    const float sq = x * x;
+                    acc = acc + sq;
+                }
+                lane[i] = acc;
+            }
+            for (int o = 16; o > 0; o >>= 1) {
+                float next[32];
+                for (int i = 0; i < 32; ++i)
+                    next[i] = lane[i] + lane[i ^ o];
+                for (int i = 0; i < 32; ++i)
+                    lane[i] = next[i];
+            }
+            const float scale = beta / lane[0];
+            for (int64_t j = 0; j < H; ++j) {
+                const uint64_t h = splitmix_mix(k + (uint64_t)(j + 1) * G);
+                const int32_t sv = (int32_t)(2 * (h & 0xFFFF) + 2 * ((h >> 16) & 0xFFFF) +
+                                             2 * ((h >> 32) & 0xFFFF) + 2 * ((h >> 48) & 0xFFFF) +
+                                             4) -
+                                   262144;
+                const float z = (float)sv * noise_scale;
+                const float prod = scale * (float)bf16_to_double(wt[j]);
+                const float hj = z + prod;
+                out[row * H + j] = bf16_round(hj);
+            }
+        }
+}

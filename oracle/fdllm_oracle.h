@@ -123,6 +123,18 @@ void oracle_lmhead_logits(const uint16_t *hidden, const uint16_t *w, int64_t row
                           int64_t V, const uint8_t *mask, double *out, double *out_abs,
                           int nthreads);
 
+/* Counter-based synthetic hidden states [B, L, H] (bf16 bits) against the bf16 head w [V, H]:
+ * the LM-head counterpart of oracle_synth_block_logits, an input generator (test
+ * infrastructure, no selection arithmetic).  For row (b, l) with row key k: p = mix(k ^
+ * 0xD1B54A32D192ED03), target t = p % V, beta = fl32(float(p >> 40) * fl32(beta_max / 2^24));
+ * z_j the Irwin-Hall noise at index j; n2 = |w_t|^2 in fp32 as 32 lane sums (lane i: j = i,
+ * i + 32, ... in order) folded by an xor butterfly over offsets 16, 8, 4, 2, 1; scale =
+ * beta / n2; h_j = fl32(z_j + fl32(scale * w_tj)), rounded to bf16.  Unmasked rows are left
+ * as they are. */
+void oracle_synth_block_hidden(uint16_t *out, const uint8_t *mask, int64_t B, int64_t L,
+                               int64_t H, int64_t V, const uint16_t *w, uint64_t seed,
+                               uint64_t step, double beta_max);
+
 #ifdef __cplusplus
 }
 #endif

@@ -23,7 +23,7 @@ __all__ = [
     "fdllm_version", "library_path", "fdllm_select_static", "fdllm_select_robust",
     "fdllm_profile_terms", "fdllm_check_bounded_wait", "fdllm_decode_loop", "FORWARD_FN",
     "fdllm_lmhead_select", "fdllm_lmhead_confidence", "fdllm_lmhead_logits",
-    "fdllm_gather_masked_rows",
+    "fdllm_gather_masked_rows", "fdllm_decode_loop_lmhead",
 ]
 
 BF16, FP32 = 0, 1
@@ -77,6 +77,9 @@ def _load():
     lib.fdllm_decode_loop.argtypes = [i, i, i, i, i, d, i, FORWARD_FN, p, p, p, p, i,
                                       ctypes.POINTER(ctypes.c_int), p]
     lib.fdllm_decode_loop.restype = i
+    lib.fdllm_decode_loop_lmhead.argtypes = [i, i, i, i, i, p, d, i, FORWARD_FN, p, p, p, p, i,
+                                             ctypes.POINTER(ctypes.c_int), p]
+    lib.fdllm_decode_loop_lmhead.restype = i
     lib.fdllm_check_bounded_wait.argtypes = [d, p]
     lib.fdllm_check_bounded_wait.restype = i
     lib.fdllm_device_status.argtypes = [p]
@@ -424,6 +427,39 @@ def fdllm_gather_masked_rows(src: torch.Tensor, mask: torch.Tensor, dst=None, st
                                             _dev(mask, "mask", torch.uint8, (B, L)),
                                             _stream(stream)), "fdllm_gather_masked_rows")
     return dst
+
+
+def fdllm_decode_loop_lmhead(forward, hidden: torch.Tensor, w_vocab: torch.Tensor, gen_len: int,
+                             param: float, mode=PROFILE, max_steps: int | None = None,
+                             stream=None):
+    """fdllm_decode_loop with the LM head in the loop: ``hidden`` is the [B, block_len, H]
+    bf16 buffer the forward pass fills, ``w_vocab`` the [V, H] bf16 head.  Returns
+    (seq_tokens [B, gen_len] int32, nfe_per_block int32, total steps); synchronous."""
+    B, Lb, H = hidden.shape
+    V, H2 = w_vocab.shape
+    if H2 != H:
+        raise ValueError("w_vocab must be [V, %d]" % H)
+    nblocks = gen_len // Lb
+    dev = hidden.device
+    seq = torch.empty((B, gen_len), dtype=torch.int32, device=dev)
+    nfe = torch.empty((nblocks,), dtype=torch.int32, device=dev)
+    steps = ctypes.c_int(0)
+
+    def trampoline(user, state, mask, out, strm):
+        try:
+            r = forward(state, mask, out, strm)
+            return 0 if r is None else int(r)
+        except Exception:  # reported as an argument error by the library
+            return 1
+
+    cb = FORWARD_FN(trampoline)
+    st = _load().fdllm_decode_loop_lmhead(
+        B, gen_len, Lb, H, V, _dev(w_vocab, "w_vocab", torch.bfloat16), float(param),
+        _mode(mode), cb, None, _dev(hidden, "hidden", torch.bfloat16), seq.data_ptr(),
+        nfe.data_ptr(), int(max_steps if max_steps is not None else gen_len + 1),
+        ctypes.byref(steps), _stream(stream))
+    _check(st, "fdllm_decode_loop_lmhead")
+    return seq, nfe, steps.value
 
 
 def fdllm_check_bounded_wait(seconds: float = 0.01, stream=None) -> int:

@@ -109,13 +109,26 @@ struct LoopArgs {
     double param;
     fdllm_forward_fn forward;
     void *user;
-    void *logits;
+    void *logits;           // what the forward pass writes: logits, or hidden states with w_vocab
+    const void *w_vocab;    // non-null: the selection runs on the LM head (hidden size H)
+    int H;
     int32_t *seq;
     int32_t *nfe;
     LoopState *st;
     uint8_t *block_mask, *commit;
     int32_t *block_tokens, *block_n;
 };
+
+// One step's selection on the block buffer: from logits, or from hidden states through the
+// LM head.
+fdllm_status run_step_select(const LoopArgs &a, cudaStream_t s, bool pdl)
+{
+    if (a.w_vocab)
+        return lmhead_select_owned(a.logits, a.w_vocab, a.B, a.Lb, a.H, a.V, a.block_mask,
+                                   a.param, a.mode, a.block_tokens, a.commit, a.block_n, s, pdl);
+    return select_owned(a.logits, a.dtype, a.B, a.Lb, a.V, a.block_mask, a.param, a.mode,
+                        a.block_tokens, a.commit, a.block_n, s, pdl);
+}
 
 fdllm_status build_loop_graph(const LoopArgs &a, cudaStream_t cs, bool pdl, LoopGraph &g)
 {
@@ -140,8 +153,7 @@ fdllm_status build_loop_graph(const LoopArgs &a, cudaStream_t cs, bool pdl, Loop
     if (a.forward(a.user, &a.st->step, a.block_mask, a.logits, cs) != 0)
         st = FDLLM_ERR_ARG;
     if (st == FDLLM_OK)
-        st = select_owned(a.logits, a.dtype, a.B, a.Lb, a.V, a.block_mask, a.param, a.mode,
-                          a.block_tokens, a.commit, a.block_n, cs, pdl);
+        st = run_step_select(a, cs, pdl);
     if (st == FDLLM_OK) {
         loop_control_kernel<<<1, 256, 0, cs>>>(a.st, a.block_mask, a.commit, a.block_tokens,
                                                a.seq, a.nfe, a.B, a.Lb, a.gen_len, a.nblocks,
@@ -164,38 +176,21 @@ fdllm_status build_loop_graph(const LoopArgs &a, cudaStream_t cs, bool pdl, Loop
 
 using namespace fdllm;
 
-extern "C" fdllm_status fdllm_decode_loop(int B, int gen_len, int block_len, int V, int dtype,
-                                          double param, int mode, fdllm_forward_fn forward,
-                                          void *user, void *logits, int32_t *seq_tokens,
-                                          int32_t *nfe_per_block, int max_steps, int *out_steps,
-                                          void *stream)
+namespace fdllm {
+namespace {
+
+fdllm_status run_decode_loop(LoopArgs a, int *out_steps, cudaStream_t s)
 {
-    if (B < 1 || block_len < 1 || block_len > FDLLM_MAX_L || gen_len < block_len ||
-        gen_len % block_len != 0 || (int64_t)B * block_len > FDLLM_MAX_ROWS || max_steps < 1 ||
-        !forward || !logits || !seq_tokens || !nfe_per_block || !out_steps)
+    if (a.B < 1 || a.Lb < 1 || a.Lb > FDLLM_MAX_L || a.gen_len < a.Lb ||
+        a.gen_len % a.Lb != 0 || (int64_t)a.B * a.Lb > FDLLM_MAX_ROWS || a.max_steps < 1 ||
+        !a.forward || !a.logits || !a.seq || !a.nfe || !out_steps)
         return FDLLM_ERR_ARG;
-    if (mode != FDLLM_PROFILE && mode != FDLLM_FACTOR && mode != FDLLM_THRESHOLD)
+    if (a.mode != FDLLM_PROFILE && a.mode != FDLLM_FACTOR && a.mode != FDLLM_THRESHOLD)
         return FDLLM_ERR_ARG;
     *out_steps = 0;
-    const int Lb = block_len, nblocks = gen_len / block_len;
+    const int B = a.B, Lb = a.Lb, gen_len = a.gen_len;
+    a.nblocks = gen_len / Lb;
     const int64_t rows = (int64_t)B * Lb;
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
-
-    LoopArgs a = {};
-    a.B = B;
-    a.Lb = Lb;
-    a.V = V;
-    a.dtype = dtype;
-    a.mode = mode;
-    a.gen_len = gen_len;
-    a.nblocks = nblocks;
-    a.max_steps = max_steps;
-    a.param = param;
-    a.forward = forward;
-    a.user = user;
-    a.logits = logits;
-    a.seq = seq_tokens;
-    a.nfe = nfe_per_block;
     cudaStream_t cs = nullptr;
     fdllm_status result = FDLLM_ERR_CUDA;
 
@@ -210,8 +205,7 @@ extern "C" fdllm_status fdllm_decode_loop(int B, int gen_len, int block_len, int
         // and sizes the library workspace (nothing may be allocated inside the captured body).
         if (cudaMemsetAsync(a.block_mask, 0, rows, s) != cudaSuccess)
             break;
-        fdllm_status pre = select_owned(logits, dtype, B, Lb, V, a.block_mask, param, mode,
-                                        a.block_tokens, a.commit, a.block_n, s, true);
+        fdllm_status pre = run_step_select(a, s, true);
         if (pre != FDLLM_OK) {
             result = pre;
             break;
@@ -236,9 +230,8 @@ extern "C" fdllm_status fdllm_decode_loop(int B, int gen_len, int block_len, int
         const int64_t total = rows > (int64_t)B * gen_len ? rows : (int64_t)B * gen_len;
         const int threads = 256;
         const int blocks = (int)((total + threads - 1) / threads);
-        loop_init_kernel<<<blocks, threads, 0, s>>>(a.st, a.block_mask, rows, seq_tokens,
-                                                     (int64_t)B * gen_len, nfe_per_block,
-                                                     nblocks);
+        loop_init_kernel<<<blocks, threads, 0, s>>>(a.st, a.block_mask, rows, a.seq,
+                                                     (int64_t)B * gen_len, a.nfe, a.nblocks);
         if (cudaGetLastError() != cudaSuccess || cudaGraphLaunch(g->exec, s) != cudaSuccess)
             break;
         LoopState host;
@@ -259,4 +252,58 @@ extern "C" fdllm_status fdllm_decode_loop(int B, int gen_len, int block_len, int
     cudaFree(a.block_tokens);
     cudaFree(a.block_n);
     return result;
+}
+
+}  // namespace
+}  // namespace fdllm
+
+extern "C" fdllm_status fdllm_decode_loop(int B, int gen_len, int block_len, int V, int dtype,
+                                          double param, int mode, fdllm_forward_fn forward,
+                                          void *user, void *logits, int32_t *seq_tokens,
+                                          int32_t *nfe_per_block, int max_steps, int *out_steps,
+                                          void *stream)
+{
+    LoopArgs a = {};
+    a.B = B;
+    a.Lb = block_len;
+    a.V = V;
+    a.dtype = dtype;
+    a.mode = mode;
+    a.gen_len = gen_len;
+    a.max_steps = max_steps;
+    a.param = param;
+    a.forward = forward;
+    a.user = user;
+    a.logits = logits;
+    a.seq = seq_tokens;
+    a.nfe = nfe_per_block;
+    return run_decode_loop(a, out_steps, static_cast<cudaStream_t>(stream));
+}
+
+extern "C" fdllm_status fdllm_decode_loop_lmhead(int B, int gen_len, int block_len, int H, int V,
+                                                 const void *w_vocab, double param, int mode,
+                                                 fdllm_forward_fn forward, void *user,
+                                                 void *hidden, int32_t *seq_tokens,
+                                                 int32_t *nfe_per_block, int max_steps,
+                                                 int *out_steps, void *stream)
+{
+    if (!w_vocab)
+        return FDLLM_ERR_ARG;
+    LoopArgs a = {};
+    a.B = B;
+    a.Lb = block_len;
+    a.V = V;
+    a.dtype = FDLLM_BF16;
+    a.mode = mode;
+    a.gen_len = gen_len;
+    a.max_steps = max_steps;
+    a.param = param;
+    a.forward = forward;
+    a.user = user;
+    a.logits = hidden;
+    a.w_vocab = w_vocab;
+    a.H = H;
+    a.seq = seq_tokens;
+    a.nfe = nfe_per_block;
+    return run_decode_loop(a, out_steps, static_cast<cudaStream_t>(stream));
 }

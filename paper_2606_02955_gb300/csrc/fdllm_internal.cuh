@@ -123,6 +123,13 @@ struct ProfileSelectArgs {
 
 cudaError_t launch_profile_select(const ProfileSelectArgs &a, cudaStream_t stream);
 
+// fdllm_lmhead_select on the library-owned workspace, with programmatic dependent launches
+// switched on or off (as select_owned).
+fdllm_status lmhead_select_owned(const void *hidden, const void *w_vocab, int B, int L, int H,
+                                 int V, uint8_t *mask, double param, int mode,
+                                 int32_t *out_tokens, uint8_t *out_commit, int32_t *out_n,
+                                 cudaStream_t stream, bool pdl);
+
 // The library-owned workspace of the current device, grown on demand and zero-filled when
 // allocated.  Every user shares its 256-byte header: the sticky status word at offset 0 and
 // the vocab reduction's work counter at 4 (zero between calls); the LM-head path keeps its

@@ -75,6 +75,7 @@ struct GemmArgs {
     UnitPartial *partials;     // kReduce: [R][n_tiles]
     float *logits;             // kStore: [B * L][V] fp32, written at masked rows
     uint32_t *status;          // sticky device error bits
+    bool pdl;                  // host side: launch as a programmatic dependent
 };
 
 // A bounded wait that also gives up as soon as another role of the CTA has given up.
@@ -597,10 +598,11 @@ bool make_map(CUtensorMap *map, const void *base, int64_t inner, int64_t outer, 
            CUDA_SUCCESS;
 }
 
-// A launch as a programmatic dependent of the previous kernel on the stream.
+// A launch as a programmatic dependent of the previous kernel on the stream (in plain
+// stream order when pdl is false).
 template <typename... KArgs, typename... Args>
-cudaError_t launch_pdl(void (*kern)(KArgs...), unsigned grid, unsigned block, cudaStream_t stream,
-                       Args... args)
+cudaError_t launch_pdl(bool pdl, void (*kern)(KArgs...), unsigned grid, unsigned block,
+                       cudaStream_t stream, Args... args)
 {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
@@ -610,7 +612,7 @@ cudaError_t launch_pdl(void (*kern)(KArgs...), unsigned grid, unsigned block, cu
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = pdl ? 1 : 0;
     return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
 }
 
@@ -725,7 +727,7 @@ cudaError_t launch_gemm_cfg(const CUtensorMap &mh, const CUtensorMap &mw, const 
         grid[dev] = clusters * CL;  // persistent: every cluster resident at once
     });
     cfg.gridDim = dim3((unsigned)grid[dev]);
-    cfg.numAttrs = 2;
+    cfg.numAttrs = g.pdl ? 2 : 1;
     return cudaLaunchKernelEx(&cfg, kern, mh, mw, g);
 }
 
@@ -751,7 +753,7 @@ cudaError_t launch_gemm(const CUtensorMap &mh, const CUtensorMap &mw, const Gemm
 // Steps 1-3 (and 4 for the reduce epilogue) on the owned workspace.
 fdllm_status run_lmhead(const void *hidden, const void *w, int B, int L, int H, int V,
                         const uint8_t *mask, int epi, float *out_logits, cudaStream_t s,
-                        uint8_t **ws_out, LmLayout *lay_out)
+                        uint8_t **ws_out, LmLayout *lay_out, bool pdl = true)
 {
     const int64_t rows = (int64_t)B * L;
     const int bn = choose_bn(rows, V);
@@ -772,9 +774,9 @@ fdllm_status run_lmhead(const void *hidden, const void *w, int B, int L, int H, 
         !make_map(&mw, w, H, V, mode == kSolo ? bn : bn / 2))
         return FDLLM_ERR_CUDA;
 
-    if (launch_pdl(compact_rows_kernel, 1, 1024, s, mask, (int)rows, row_ids, row_count) !=
+    if (launch_pdl(pdl, compact_rows_kernel, 1, 1024, s, mask, (int)rows, row_ids, row_count) !=
             cudaSuccess ||
-        launch_pdl(gather_rows_kernel, (unsigned)rows, 128, s,
+        launch_pdl(pdl, gather_rows_kernel, (unsigned)rows, 128, s,
                    static_cast<const int4 *>(hidden), (int64_t)(H / 8),
                    (const int32_t *)row_ids, (const int32_t *)row_count,
                    reinterpret_cast<int4 *>(packed)) != cudaSuccess)
@@ -788,13 +790,14 @@ fdllm_status run_lmhead(const void *hidden, const void *w, int B, int L, int H, 
     g.partials = reinterpret_cast<UnitPartial *>(ws + lay.partials);
     g.logits = out_logits;
     g.status = reinterpret_cast<uint32_t *>(ws);
+    g.pdl = pdl;
     const cudaError_t e = epi == kReduce ? launch_gemm<kReduce>(mh, mw, g, mode, bn, s)
                                          : launch_gemm<kStore>(mh, mw, g, mode, bn, s);
     if (e != cudaSuccess)
         return FDLLM_ERR_CUDA;
     if (epi == kReduce) {
         const int warps = 8;
-        if (launch_pdl(combine_rows_kernel, (unsigned)((rows + warps - 1) / warps), warps * 32,
+        if (launch_pdl(pdl, combine_rows_kernel, (unsigned)((rows + warps - 1) / warps), warps * 32,
                        s, (const UnitPartial *)g.partials, n_tiles, (const int32_t *)row_ids,
                        (const int32_t *)row_count, reinterpret_cast<float *>(ws + lay.conf),
                        reinterpret_cast<int32_t *>(ws + lay.tok)) != cudaSuccess)
@@ -823,12 +826,12 @@ __global__ void scatter_conf_kernel(const float *conf, const int32_t *tok, const
 
 using namespace fdllm;
 
-extern "C" {
+namespace fdllm {
 
-fdllm_status fdllm_lmhead_select(const void *hidden, const void *w_vocab, int B, int L, int H,
+fdllm_status lmhead_select_owned(const void *hidden, const void *w_vocab, int B, int L, int H,
                                  int V, uint8_t *mask, double param, int mode,
                                  int32_t *out_tokens, uint8_t *out_commit, int32_t *out_n,
-                                 void *stream)
+                                 cudaStream_t s, bool pdl)
 {
     fdllm_status st = check_lmhead(hidden, w_vocab, B, L, H, V, mask);
     if (st != FDLLM_OK)
@@ -836,10 +839,9 @@ fdllm_status fdllm_lmhead_select(const void *hidden, const void *w_vocab, int B,
     if (!out_tokens || !out_commit || !out_n || !std::isfinite(param) ||
         (mode != FDLLM_PROFILE && mode != FDLLM_FACTOR && mode != FDLLM_THRESHOLD))
         return FDLLM_ERR_ARG;
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
     uint8_t *ws = nullptr;
     LmLayout lay;
-    st = run_lmhead(hidden, w_vocab, B, L, H, V, mask, kReduce, nullptr, s, &ws, &lay);
+    st = run_lmhead(hidden, w_vocab, B, L, H, V, mask, kReduce, nullptr, s, &ws, &lay, pdl);
     if (st != FDLLM_OK)
         return st;
     ProfileSelectArgs pa;
@@ -859,8 +861,21 @@ fdllm_status fdllm_lmhead_select(const void *hidden, const void *w_vocab, int B,
     pa.out_commit = out_commit;
     pa.out_n = out_n;
     pa.status = reinterpret_cast<const uint32_t *>(ws);
-    pa.pdl = true;
+    pa.pdl = pdl;
     return launch_profile_select(pa, s) == cudaSuccess ? FDLLM_OK : FDLLM_ERR_CUDA;
+}
+
+}  // namespace fdllm
+
+extern "C" {
+
+fdllm_status fdllm_lmhead_select(const void *hidden, const void *w_vocab, int B, int L, int H,
+                                 int V, uint8_t *mask, double param, int mode,
+                                 int32_t *out_tokens, uint8_t *out_commit, int32_t *out_n,
+                                 void *stream)
+{
+    return lmhead_select_owned(hidden, w_vocab, B, L, H, V, mask, param, mode, out_tokens,
+                               out_commit, out_n, static_cast<cudaStream_t>(stream), true);
 }
 
 fdllm_status fdllm_lmhead_confidence(const void *hidden, const void *w_vocab, int B, int L,
@@ -879,7 +894,7 @@ fdllm_status fdllm_lmhead_confidence(const void *hidden, const void *w_vocab, in
     if (st != FDLLM_OK)
         return st;
     const int64_t rows = (int64_t)B * L;
-    return launch_pdl(scatter_conf_kernel, (unsigned)((rows + 255) / 256), 256, s,
+    return launch_pdl(true, scatter_conf_kernel, (unsigned)((rows + 255) / 256), 256, s,
                       reinterpret_cast<const float *>(ws + lay.conf),
                       reinterpret_cast<const int32_t *>(ws + lay.tok),
                       reinterpret_cast<const int32_t *>(ws + lay.row_ids),

@@ -134,3 +134,81 @@ def test_decode_loop_forward_failure_is_reported(fd):
     seq, nfe, steps = fd.fdllm_decode_loop(forward_for(B, Lb, V, 3, 16.0), logits, gen, 1.5,
                                            oracle.THRESHOLD)
     assert steps == gen
+
+
+# ----------------------------------------------------------------------------- LM head loop
+def lm_inputs(H, V):
+    _, w, _ = syn.make_lmhead_inputs(1, 1, H, V, seed=V, device="cuda")
+    return w
+
+
+@pytest.mark.parametrize("B,L,H,V", [(2, 8, 256, 3000), (3, 5, 72, 1000)])
+def test_synth_hidden_gpu_bytes_match_oracle(fd, orc, B, L, H, V):
+    w = lm_inputs(H, V)
+    mask_np = (np.arange(B * L).reshape(B, L) % 4 != 2).astype(np.uint8)
+    mask = torch.from_numpy(mask_np).cuda()
+    out = torch.full((B, L, H), 5.0, dtype=torch.bfloat16, device="cuda")
+    st = torch.tensor([9], dtype=torch.int32, device="cuda")
+    syn.synth_block_hidden_gpu(out.data_ptr(), mask.data_ptr(), B, L, H, V, w.data_ptr(), 77,
+                               step_ptr=st.data_ptr(), beta_max=18.0,
+                               stream_ptr=torch.cuda.current_stream().cuda_stream)
+    torch.cuda.synchronize()
+    got = syn.host_bits(out)
+    ref = orc.synth_block_hidden(syn.host_bits(w), B, L, 77, 9, 18.0, mask=mask_np)
+    mk = mask_np.astype(bool)
+    assert np.array_equal(got[mk], ref[mk])
+
+
+def hidden_forward(B, Lb, H, V, w, seed, beta):
+    def forward(state, mask, out, stream):
+        syn.synth_block_hidden_gpu(out, mask, B, Lb, H, V, w.data_ptr(), seed, step_ptr=state,
+                                   beta_max=beta, stream_ptr=stream)
+    return forward
+
+
+@pytest.mark.parametrize("mode,param", [(oracle.PROFILE, 1.0), (oracle.PROFILE, 0.75),
+                                        (oracle.FACTOR, 1.0)])
+def test_decode_loop_lmhead_against_host_loop_and_oracle(fd, orc, mode, param):
+    """The device-resident loop with the LM head equals a host-driven loop of
+    fdllm_lmhead_select calls (same kernels: bit-exact), and every step of the host loop
+    matches the oracle run on that step's tensor-core accumulators (margin >= 1e-5)."""
+    B, gen, Lb, H, V, seed, beta = 2, 32, 16, 256, 3000, 5, 20.0
+    w = lm_inputs(H, V)
+    hidden = torch.empty((B, Lb, H), dtype=torch.bfloat16, device="cuda")
+    seq_d, nfe_d, steps_d = fd.fdllm_decode_loop_lmhead(
+        hidden_forward(B, Lb, H, V, w, seed, beta), hidden, w, gen, param, mode)
+    torch.cuda.synchronize()
+
+    stream = torch.cuda.current_stream().cuda_stream
+    seq = np.full((B, gen), -1, np.int32)
+    nfe, step, checked = [], 0, 0
+    tok = torch.empty((B, Lb), dtype=torch.int32, device="cuda")
+    commit = torch.empty((B, Lb), dtype=torch.uint8, device="cuda")
+    n = torch.empty((B,), dtype=torch.int32, device="cuda")
+    for blk in range(gen // Lb):
+        mask = torch.ones((B, Lb), dtype=torch.uint8, device="cuda")
+        k = 0
+        while bool(mask.any().item()):
+            syn.synth_block_hidden_gpu(hidden.data_ptr(), mask.data_ptr(), B, Lb, H, V,
+                                       w.data_ptr(), seed, step=step, beta_max=beta,
+                                       stream_ptr=stream)
+            before = mask.cpu().numpy()
+            x32 = fd.fdllm_lmhead_logits(hidden, w, mask)
+            fd.fdllm_lmhead_select(hidden, w, mask, param, mode, tok, commit, n)
+            torch.cuda.synchronize()
+            x32 = np.nan_to_num(x32.cpu().numpy(), nan=0.0).astype(np.float32)
+            ref = orc.select(x32, before, mode, param, nthreads=oracle_threads())
+            c = commit.cpu().numpy()
+            for b in range(B):
+                if ref["margin"][b] >= MARGIN:
+                    assert n[b].item() == ref["n"][b] and np.array_equal(c[b], ref["commit"][b])
+                    checked += 1
+            t = tok.cpu().numpy()
+            seq[:, blk * Lb:(blk + 1) * Lb][c == 1] = t[c == 1]
+            step += 1
+            k += 1
+        nfe.append(k)
+    assert checked > 0
+    assert steps_d == step
+    assert list(nfe_d.cpu().numpy()) == nfe
+    assert np.array_equal(seq_d.cpu().numpy(), seq)

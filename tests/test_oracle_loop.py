@@ -137,3 +137,63 @@ def test_loop_stops_at_max_steps(orc):
     filled = r["seq"] >= 0
     assert filled[:, :8].all() and (filled[:, 8:16].sum(axis=1) == 3).all()
     assert not filled[:, 16:].any()
+
+
+def py_synth_hidden(w_bits, B, L, seed, step, beta_max):
+    V, H = w_bits.shape
+    f32 = np.float32
+    out = np.zeros((B, L, H), np.uint16)
+    wf = bits_to_f32(w_bits)
+    scale_n = f32(np.sqrt(3.0) / 131072.0)
+    bscale = f32(beta_max / 16777216.0)
+    for b in range(B):
+        for l in range(L):
+            k = mix(seed ^ mix(((step * GOLD) & M64) ^ mix((b << 32) | l)))
+            p = mix(k ^ 0xD1B54A32D192ED03)
+            t = p % V
+            beta = f32(f32(p >> 40) * bscale)
+            lanes = []
+            for i in range(32):
+                acc = f32(0.0)
+                for j in range(i, H, 32):
+                    acc = f32(acc + f32(wf[t, j] * wf[t, j]))
+                lanes.append(acc)
+            o = 16
+            while o:
+                lanes = [f32(lanes[i] + lanes[i ^ o]) for i in range(32)]
+                o >>= 1
+            scale = f32(beta / lanes[0])
+            for j in range(H):
+                h = mix(k + (j + 1) * GOLD)
+                sv = sum(2 * ((h >> (16 * q)) & 0xFFFF) + 1 for q in range(4)) - 262144
+                z = f32(f32(sv) * scale_n)
+                out[b, l, j] = bf16_bits(f32(z + f32(scale * wf[t, j])))
+    return out
+
+
+def test_synth_hidden_matches_its_definition(orc):
+    import torch
+    g = torch.Generator().manual_seed(4)
+    w = (torch.randn((50, 40), generator=g) / 6).to(torch.bfloat16)
+    wb = w.view(torch.int16).numpy().view(np.uint16)
+    for seed, step in ((7, 0), (99, 5)):
+        got = orc.synth_block_hidden(wb, 2, 3, seed, step, 20.0)
+        assert np.array_equal(got, py_synth_hidden(wb, 2, 3, seed, step, 20.0))
+
+
+def test_synth_hidden_plants_the_target(orc):
+    import fdllm_synth as syn
+    _, w, _ = syn.make_lmhead_inputs(1, 1, 256, 2000, seed=1)
+    wb = w.view(torch_int16()).numpy().view(np.uint16)
+    h = orc.synth_block_hidden(wb, 2, 8, 11, 0, 16.0)
+    x = orc.lmhead_logits(h, wb)
+    # the planted index carries beta ~ U[0, 16) above N(0, ~1) noise: the argmax for tall peaks
+    k_hits = (x.max(-1) > 8.0).sum()
+    assert k_hits > 0
+    noise = np.sort(x, axis=-1)[..., :-1]
+    assert abs(noise.mean()) < 0.05 and abs(noise.std() - 1.0) < 0.15
+
+
+def torch_int16():
+    import torch
+    return torch.int16
