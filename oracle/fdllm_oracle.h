@@ -11,7 +11,8 @@
  *   confidence/argmax per masked position -> sort -> scan of L_n, U_n, G_n -> n* -> reveal.
  *
  * Conventions shared with the CUDA library's public interface (not its code):
- *   logits  [B, L, V] row-major, V contiguous; dtype 0 = bf16 (raw uint16 bits), 1 = fp32.
+ *   logits  [B, L, V] row-major, V contiguous; dtype 0 = bf16 (raw uint16 bits), 1 = fp32,
+ *           2 = fp64 (exact LM-head products).
  *   mask    uint8 [B, L], 1 = masked; updated in place by the reveal (committed -> 0).
  *   mode    0 = profile (Frechet), 1 = factor, 2 = threshold.
  *   param   profile: f, with margin delta = 1 - f (matched parameter, Cor. factor-reduction);
