@@ -397,7 +397,10 @@ def fdllm_decode_loop(forward, logits: torch.Tensor, gen_len: int, param: float,
         try:
             r = forward(state, mask, out, strm)
             return 0 if r is None else int(r)
-        except Exception:  # reported as an argument error by the library
+        except Exception:  # the library reports it as FDLLM_ERR_ARG; keep the cause visible
+            import traceback
+            import warnings
+            warnings.warn("forward pass raised during loop capture:\n" + traceback.format_exc())
             return 1
 
     cb = FORWARD_FN(trampoline)
@@ -449,7 +452,10 @@ def fdllm_decode_loop_lmhead(forward, hidden: torch.Tensor, w_vocab: torch.Tenso
         try:
             r = forward(state, mask, out, strm)
             return 0 if r is None else int(r)
-        except Exception:  # reported as an argument error by the library
+        except Exception:  # the library reports it as FDLLM_ERR_ARG; keep the cause visible
+            import traceback
+            import warnings
+            warnings.warn("forward pass raised during loop capture:\n" + traceback.format_exc())
             return 1
 
     cb = FORWARD_FN(trampoline)

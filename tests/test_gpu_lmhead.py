@@ -185,3 +185,21 @@ def test_empty_mask_and_repeat(fd, cluster):
         assert torch.equal(x, y)
     assert torch.equal(m1, m2)
     assert fd.fdllm_device_status() == 0
+
+
+@pytest.mark.parametrize("H", [8, 16, 40])
+def test_hidden_sizes_below_one_stage(fd, orc, H):
+    """H smaller than the 64-element stage: the TMA boxes reach past the rows' end and read
+    zeros there."""
+    B, L, V = 2, 8, 700
+    h, w, mask_np = inputs(B, L, H, V, seed=H)
+    x = fd.fdllm_lmhead_logits(h, w, torch.from_numpy(mask_np).cuda())
+    conf, tok = fd.fdllm_lmhead_confidence(h, w, torch.from_numpy(mask_np).cuda())
+    torch.cuda.synchronize()
+    ref, mag = orc.lmhead_logits(bits(h), bits(w), mask=mask_np, with_abs=True)
+    mk = mask_np.astype(bool)
+    xg = x.cpu().numpy().astype(np.float64)
+    assert (np.abs(xg[mk] - ref[mk]) <= gemm_bound(mag[mk], ref[mk], H)).all()
+    rc, rt, _ = orc.confidence(np.nan_to_num(x.cpu().numpy(), nan=0.0), mask_np)
+    assert np.array_equal(tok.cpu().numpy()[mk], rt[mk])
+    assert (np.abs(conf.cpu().numpy()[mk] - rc[mk]) / rc[mk]).max() <= CONF_RTOL
