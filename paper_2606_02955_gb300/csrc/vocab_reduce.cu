@@ -268,51 +268,121 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
     if (threadIdx.x == 0)
         pdl_launch_dependents();
 
-    // Mask -> bitmap (one ballot per 32 rows, four words in flight per warp) -> exclusive
-    // prefix count per word.
+    const uint32_t upr = (uint32_t)a.units_per_row;
     const int nwords = (int)((a.rows + 31) / 32);
-    for (int w0 = warp; w0 < nwords; w0 += 4 * kWarps) {
-        bool m[4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const int w = w0 + i * kWarps;
-            const int64_t r = (int64_t)w * 32 + lane;
-            m[i] = w < nwords && r < a.rows && a.mask[r] != 0;
+
+    // The producer's first unit (unit blockIdx.x: masked row blockIdx.x / upr) is located by
+    // the producer warp alone, with a ballot scan of the mask, and its copies are issued
+    // before the CTA-wide mask compaction below: the first data is in flight while the other
+    // warps build the bitmap.
+    uint32_t k = 0;  // producer: chunks issued so far
+    uint64_t policy = 0;
+    auto issue_unit = [&](uint32_t u, int64_t grow) -> bool {
+        const uint32_t j = u % upr;
+        const int64_t v0 = (int64_t)j * a.unit_vecs;
+        const int64_t v1 = min(v0 + (int64_t)a.unit_vecs, a.vec_per_row);
+        const uint8_t *rowp = a.logits + grow * a.row_bytes;
+        for (int64_t v = v0; v < v1; v += kChunkVecs) {
+            const uint32_t n = (uint32_t)min((int64_t)kChunkVecs, v1 - v);
+            const uint32_t s = k % kStages;
+            if (k >= kStages && !mbar_wait(&sm.empty[s], ((k / kStages) - 1) & 1, a.status))
+                return false;  // math warps stopped; issued copies complete on their own
+            ChunkMeta cm;
+            cm.n = n;
+            cm.vec_base = (uint32_t)v;
+            cm.last = (v + n == v1) ? 1u : 0u;
+            cm.pidx = (uint32_t)(grow * upr + j);
+            sm.meta[s] = cm;
+            mbar_arrive_expect_tx(&sm.full[s], n * 16u);
+            if (EVICT)
+                bulk_copy_g2s_hint(ring + (size_t)s * kChunkBytes, rowp + v * 16, n * 16u,
+                                   &sm.full[s], policy);
+            else
+                bulk_copy_g2s(ring + (size_t)s * kChunkBytes, rowp + v * 16, n * 16u,
+                              &sm.full[s]);
+            ++k;
         }
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const uint32_t b = __ballot_sync(0xFFFFFFFFu, m[i]);
-            if (lane == 0 && w0 + i * kWarps < nwords)
-                sm.bits[w0 + i * kWarps] = b;
-        }
-    }
-    __syncthreads();
+        return true;
+    };
+    bool first_issued = false;
+    uint32_t u_next = 0;
     if (warp == 0) {
-        const int per = (nwords + 31) / 32;
-        const int w0 = lane * per;
-        uint32_t local = 0;
-        for (int k = 0; k < per; ++k)
-            if (w0 + k < nwords)
-                local += __popc(sm.bits[w0 + k]);
-        uint32_t incl = local;
+        if (EVICT)
+            policy = make_evict_first_policy();
+        const uint32_t kth = blockIdx.x / upr;
+        uint32_t seen = 0;
+        int64_t grow = -1;
+        for (int64_t base = 0; base < a.rows && grow < 0; base += 8 * 32) {
+            uint32_t ball[8];
 #pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const uint32_t t = __shfl_up_sync(0xFFFFFFFFu, incl, o);
-            if (lane >= o)
-                incl += t;
-        }
-        uint32_t run = incl - local;
-        for (int k = 0; k < per; ++k)
-            if (w0 + k < nwords) {
-                sm.pref[w0 + k] = run;
-                run += __popc(sm.bits[w0 + k]);
+            for (int i = 0; i < 8; ++i) {
+                const int64_t r = base + i * 32 + lane;
+                ball[i] = __ballot_sync(0xFFFFFFFFu, r < a.rows && a.mask[r] != 0);
             }
-        if (lane == 31)
-            sm.pref[nwords] = incl;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const uint32_t c = (uint32_t)__popc(ball[i]);
+                if (grow < 0 && seen + c > kth)
+                    grow = base + i * 32 + (int64_t)__fns(ball[i], 0, (int)(kth - seen) + 1);
+                seen += c;
+            }
+        }
+        if (grow >= 0) {
+            first_issued = true;
+            if (lane == 0) {
+                // the next unit's request is in flight while the first one streams
+                u_next = gridDim.x + atomicAdd(a.next_unit, 1u);
+                if (!issue_unit(blockIdx.x, grow))
+                    first_issued = false;
+            }
+        }
+    } else {
+        // Mask -> bitmap (one ballot per 32 rows, four words in flight per warp) -> exclusive
+        // prefix count per word, by every warp but the producer's.
+        constexpr int kBuilders = kWarps - 1;
+        const int bw = warp - 1;
+        for (int w0 = bw; w0 < nwords; w0 += 4 * kBuilders) {
+            bool m[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int w = w0 + i * kBuilders;
+                const int64_t r = (int64_t)w * 32 + lane;
+                m[i] = w < nwords && r < a.rows && a.mask[r] != 0;
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const uint32_t b = __ballot_sync(0xFFFFFFFFu, m[i]);
+                if (lane == 0 && w0 + i * kBuilders < nwords)
+                    sm.bits[w0 + i * kBuilders] = b;
+            }
+        }
+        asm volatile("bar.sync 1, %0;" ::"r"(kBuilders * 32) : "memory");
+        if (warp == 1) {
+            const int per = (nwords + 31) / 32;
+            const int w0 = lane * per;
+            uint32_t local = 0;
+            for (int q = 0; q < per; ++q)
+                if (w0 + q < nwords)
+                    local += __popc(sm.bits[w0 + q]);
+            uint32_t incl = local;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const uint32_t t = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+                if (lane >= o)
+                    incl += t;
+            }
+            uint32_t run = incl - local;
+            for (int q = 0; q < per; ++q)
+                if (w0 + q < nwords) {
+                    sm.pref[w0 + q] = run;
+                    run += __popc(sm.bits[w0 + q]);
+                }
+            if (lane == 31)
+                sm.pref[nwords] = incl;
+        }
     }
     __syncthreads();
 
-    const uint32_t upr = (uint32_t)a.units_per_row;
     const uint32_t total = sm.pref[nwords] * upr;  // host checks rows * upr < 2^31
     if (total == 0)
         return;
@@ -321,42 +391,15 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
         // ------------------------------------------------------------ producer (one lane)
         if (lane != 0)
             return;
-        uint64_t policy = 0;
-        if (EVICT)
-            policy = make_evict_first_policy();
-        // Unit blockIdx.x first (no atomic before the first copy), then the work queue,
-        // which hands out units gridDim.x, gridDim.x + 1, ...
-        uint32_t k = 0;
-        uint32_t u = blockIdx.x;
-        while (u < total) {
-            // the next unit's request is in flight while u streams
-            const uint32_t u_next = gridDim.x + atomicAdd(a.next_unit, 1u);
-            const uint32_t r = u / upr, j = u - r * upr;
-            const int64_t grow = masked_row(r, sm.bits, sm.pref, nwords);
-            const int64_t v0 = (int64_t)j * a.unit_vecs;
-            const int64_t v1 = min(v0 + (int64_t)a.unit_vecs, a.vec_per_row);
-            const uint8_t *rowp = a.logits + grow * a.row_bytes;
-            for (int64_t v = v0; v < v1; v += kChunkVecs) {
-                const uint32_t n = (uint32_t)min((int64_t)kChunkVecs, v1 - v);
-                const uint32_t s = k % kStages;
-                if (k >= kStages && !mbar_wait(&sm.empty[s], ((k / kStages) - 1) & 1, a.status))
-                    return;  // math warps stopped; issued copies complete on their own
-                ChunkMeta cm;
-                cm.n = n;
-                cm.vec_base = (uint32_t)v;
-                cm.last = (v + n == v1) ? 1u : 0u;
-                cm.pidx = (uint32_t)(grow * upr + j);
-                sm.meta[s] = cm;
-                mbar_arrive_expect_tx(&sm.full[s], n * 16u);
-                if (EVICT)
-                    bulk_copy_g2s_hint(ring + (size_t)s * kChunkBytes, rowp + v * 16, n * 16u,
-                                       &sm.full[s], policy);
-                else
-                    bulk_copy_g2s(ring + (size_t)s * kChunkBytes, rowp + v * 16, n * 16u,
-                                  &sm.full[s]);
-                ++k;
+        if (first_issued) {
+            // Then the work queue, which hands out units gridDim.x, gridDim.x + 1, ...
+            uint32_t u = u_next;
+            while (u < total) {
+                const uint32_t un = gridDim.x + atomicAdd(a.next_unit, 1u);
+                if (!issue_unit(u, masked_row(u / upr, sm.bits, sm.pref, nwords)))
+                    return;
+                u = un;
             }
-            u = u_next;
         }
         const uint32_t s = k % kStages;
         if (k >= kStages && !mbar_wait(&sm.empty[s], ((k / kStages) - 1) & 1, a.status))
