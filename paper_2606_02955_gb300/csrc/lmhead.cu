@@ -1,16 +1,20 @@
 // lmhead.cu -- step a1 fused with the LM head that produces the logits.  The logits of a
 // masked position are x = W h (h its final hidden state [H], W the vocabulary projection
 // [V, H]); instead of writing B*L*V logits and reading them back, a tcgen05 GEMM reduces
-// each 128 x 256 accumulator tile in its epilogue to one (max, sum of exp, first argmax)
-// partial per row, straight from tensor memory.
+// each 128-row x BN-column accumulator tile (BN = 256 or 208 vocabulary entries) in its
+// epilogue to one (max, sum of exp, first argmax) partial per row, straight from tensor
+// memory.
 //
-// Launch sequence on one stream (all rows of one step):
+// Launch sequence on one stream (all rows of one step), chained by programmatic dependent
+// launches:
 //   1. compact_rows_kernel   the masked rows' indices and their count (one CTA)
 //   2. gather_rows_kernel    the masked rows' hidden states, packed [R, H] (TMA-friendly)
-//   3. lmhead_gemm_kernel    persistent tcgen05 GEMM: warp 0 issues TMA loads into a 4-stage
-//                            ring, warp 1 issues tcgen05.mma into one of two TMEM
-//                            accumulators, warps 2-5 reduce (or store) the other one
-//   4. combine_rows_kernel   one warp per row folds its V/256 tile partials in a fixed order
+//   3. lmhead_gemm_kernel    persistent tcgen05 GEMM: warp 0 issues TMA loads into a ring of
+//                            stages, warp 1 issues tcgen05.mma into one of two TMEM
+//                            accumulators, warps 2-5 reduce (or store) the other one; solo,
+//                            W-multicast or CTA-pair (cta_group::2) variants
+//   4. combine_rows_kernel   one warp per row folds its ceil(V / BN) tile partials in a fixed
+//                            order
 //   5. profile_select        steps a2-a5 on the confidences (profile_select.cu)
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -39,9 +43,6 @@ constexpr size_t kBarrierBytes = 256;
 constexpr size_t kRingBudget = 220 * 1024;
 constexpr uint64_t kDrainLimitNs = 100000000ull;  // waits for own copies after an abort
 
-// Vocabulary entries per tile (the MMA's N and the fp32 accumulator's width): 256, or 208,
-// which splits LLaDA's V = 126464 into 608 = 4 x 152 tiles, one whole wave per SM count.
-// The stage count fills the ring budget: 4 x 48 KB at 256, 5 x 42 KB at 208.
 // How the CTAs of a cluster share a W tile.
 enum Mode {
     kSolo = 0,       // one CTA per work item; it loads the whole W tile
@@ -51,6 +52,10 @@ enum Mode {
                      // rows and half of the W tile; the even CTA issues the MMAs for both
 };
 
+// Vocabulary entries per tile (the MMA's N and the fp32 accumulator's width): 256, or 208,
+// which splits LLaDA's V = 126464 into 608 = 4 x 152 tiles, whole waves over 152 SMs.  The
+// stage count fills the ring budget: solo 4 x 48 KB at 256, 5 x 42 KB at 208; pair 6 x 32 KB
+// at 256 (each CTA holds half the W tile).
 template <int BN_, int MODE>
 struct TileCfg {
     static constexpr int BN = BN_;
