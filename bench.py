@@ -594,6 +594,10 @@ def run_lmhead(args) -> dict:
     reps = max(3, args.lmhead_steps)
 
     def time_variant(fn):
+        # each variant starts from a rested GPU: a ~1 ms, 1.4 kW step drives the board into
+        # its power cap within tens of steps, which would penalise whichever runs later
+        torch.cuda.synchronize()
+        time.sleep(1.0)
         with torch.cuda.stream(stream):
             for _ in range(3):
                 fn()

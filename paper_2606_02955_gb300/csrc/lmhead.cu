@@ -13,8 +13,8 @@
 //                            stages, warp 1 issues tcgen05.mma into one of two TMEM
 //                            accumulators, warps 2-5 reduce (or store) the other one; solo,
 //                            W-multicast or CTA-pair (cta_group::2) variants
-//   4. combine_rows_kernel   one warp per row folds its ceil(V / BN) tile partials in a fixed
-//                            order
+//   4. combine_rows_kernel   four warps per row fold its ceil(V / BN) tile partials in a
+//                            fixed order
 //   5. profile_select        steps a2-a5 on the confidences (profile_select.cu)
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -485,33 +485,39 @@ __device__ __forceinline__ Part fold(const Part &x, const Part &y)
     return r;
 }
 
-// One warp per packed row: lane j folds tiles j, j + 32, ... in order, then the lanes fold
-// in a fixed butterfly.  Writes c = min(1/S, 1) and x_hat at the row's (b, l); a row with a
-// NaN logit or an infinite maximum gets c = NaN, x_hat = -1.
-__global__ void combine_rows_kernel(const UnitPartial *partials, int n_tiles,
-                                    const int32_t *row_ids, const int32_t *row_count,
-                                    float *conf, int32_t *tok)
+// One CTA of kCombineWarps warps per packed row: lane l of warp q folds tiles
+// q * 32 + l + 128 i (i = 0, 1, ...) in order, the lanes of each warp fold in a fixed
+// butterfly, and the warps' results fold in warp order.  A fixed tree, so the result does not
+// depend on timing.  Writes c = min(1/S, 1) and x_hat at the row's (b, l); a row with a NaN
+// logit or an infinite maximum gets c = NaN, x_hat = -1.
+constexpr int kCombineWarps = 4;
+
+__global__ void __launch_bounds__(kCombineWarps * 32)
+    combine_rows_kernel(const UnitPartial *partials, int n_tiles, const int32_t *row_ids,
+                        const int32_t *row_count, float *conf, int32_t *tok)
 {
+    __shared__ Part s_part[kCombineWarps];
     pdl_wait();  // every tile partial is written
     if (threadIdx.x == 0)
         pdl_launch_dependents();
-    const int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-    const int lane = threadIdx.x & 31;
+    const int r = blockIdx.x;
+    const int lane = threadIdx.x & 31, q = threadIdx.x >> 5;
     if (r >= *row_count)
         return;
     Part acc{-__int_as_float(0x7F800000), 0.0f, kNoIdx, false};
     const UnitPartial *p = partials + (int64_t)r * n_tiles;
+    constexpr int kStride = kCombineWarps * 32;
     constexpr int kBatch = 8;  // loads in flight per lane before the folds
-    for (int j0 = lane; j0 < n_tiles; j0 += 32 * kBatch) {
-        int4 q[kBatch];
+    for (int j0 = q * 32 + lane; j0 < n_tiles; j0 += kStride * kBatch) {
+        int4 v[kBatch];
 #pragma unroll
         for (int b = 0; b < kBatch; ++b)
-            if (j0 + 32 * b < n_tiles)
-                q[b] = __ldcg(reinterpret_cast<const int4 *>(p + j0 + 32 * b));
+            if (j0 + kStride * b < n_tiles)
+                v[b] = __ldcg(reinterpret_cast<const int4 *>(p + j0 + kStride * b));
 #pragma unroll
         for (int b = 0; b < kBatch; ++b)
-            if (j0 + 32 * b < n_tiles) {
-                Part y{__int_as_float(q[b].x), __int_as_float(q[b].y), (uint32_t)q[b].z, false};
+            if (j0 + kStride * b < n_tiles) {
+                Part y{__int_as_float(v[b].x), __int_as_float(v[b].y), (uint32_t)v[b].z, false};
                 y.nan = y.M != y.M;
                 if (y.nan)
                     y.M = -__int_as_float(0x7F800000);
@@ -527,7 +533,13 @@ __global__ void combine_rows_kernel(const UnitPartial *partials, int n_tiles,
         y.nan = __shfl_xor_sync(0xFFFFFFFFu, (int)acc.nan, o) != 0;
         acc = fold(acc, y);
     }
-    if (lane == 0) {
+    if (lane == 0)
+        s_part[q] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        acc = s_part[0];
+        for (int w = 1; w < kCombineWarps; ++w)
+            acc = fold(acc, s_part[w]);
         const int row = row_ids[r];
         const bool finite = fabsf(acc.M) <= 3.402823466e38f && fabsf(acc.S) <= 3.402823466e38f;
         if (acc.nan || !finite || !(acc.S > 0.0f) || acc.idx == kNoIdx) {
@@ -801,8 +813,7 @@ fdllm_status run_lmhead(const void *hidden, const void *w, int B, int L, int H, 
     if (e != cudaSuccess)
         return FDLLM_ERR_CUDA;
     if (epi == kReduce) {
-        const int warps = 8;
-        if (launch_pdl(pdl, combine_rows_kernel, (unsigned)((rows + warps - 1) / warps), warps * 32,
+        if (launch_pdl(pdl, combine_rows_kernel, (unsigned)rows, kCombineWarps * 32,
                        s, (const UnitPartial *)g.partials, n_tiles, (const int32_t *)row_ids,
                        (const int32_t *)row_count, reinterpret_cast<float *>(ws + lay.conf),
                        reinterpret_cast<int32_t *>(ws + lay.tok)) != cudaSuccess)
