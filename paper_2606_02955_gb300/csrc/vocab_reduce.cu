@@ -304,7 +304,7 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
         }
         return true;
     };
-    bool first_issued = false;
+    bool first_tried = false, first_issued = false;
     uint32_t u_next = 0;
     if (warp == 0) {
         if (EVICT)
@@ -312,12 +312,16 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
         const uint32_t kth = blockIdx.x / upr;
         uint32_t seen = 0;
         int64_t grow = -1;
-        for (int64_t base = 0; base < a.rows && grow < 0; base += 8 * 32) {
+        // A bounded scan: with few masked rows among the first kScanRows, the first unit is
+        // issued after the compaction instead (below), not after a long serial scan.
+        constexpr int64_t kScanRows = 2048;
+        const int64_t scan_end = a.rows < kScanRows ? a.rows : kScanRows;
+        for (int64_t base = 0; base < scan_end && grow < 0; base += 8 * 32) {
             uint32_t ball[8];
 #pragma unroll
             for (int i = 0; i < 8; ++i) {
                 const int64_t r = base + i * 32 + lane;
-                ball[i] = __ballot_sync(0xFFFFFFFFu, r < a.rows && a.mask[r] != 0);
+                ball[i] = __ballot_sync(0xFFFFFFFFu, r < scan_end && a.mask[r] != 0);
             }
 #pragma unroll
             for (int i = 0; i < 8; ++i) {
@@ -328,12 +332,11 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
             }
         }
         if (grow >= 0) {
-            first_issued = true;
+            first_tried = true;
             if (lane == 0) {
                 // the next unit's request is in flight while the first one streams
                 u_next = gridDim.x + atomicAdd(a.next_unit, 1u);
-                if (!issue_unit(blockIdx.x, grow))
-                    first_issued = false;
+                first_issued = issue_unit(blockIdx.x, grow);
             }
         }
     } else {
@@ -391,6 +394,12 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
         // ------------------------------------------------------------ producer (one lane)
         if (lane != 0)
             return;
+        if (!first_tried && blockIdx.x < total) {
+            // the first unit was not within the producer's scan
+            u_next = gridDim.x + atomicAdd(a.next_unit, 1u);
+            first_issued = issue_unit(blockIdx.x,
+                                      masked_row(blockIdx.x / upr, sm.bits, sm.pref, nwords));
+        }
         if (first_issued) {
             // Then the work queue, which hands out units gridDim.x, gridDim.x + 1, ...
             uint32_t u = u_next;

@@ -131,3 +131,20 @@ def test_misaligned_logits_rejected(fd):
         fd.fdllm_select(torch.randn(2, 4, 999, device="cuda", dtype=torch.bfloat16), mask, 1.0,
                         PROFILE)
     assert e.value.status == 2
+
+
+@pytest.mark.parametrize("first_masked", [2048, 60000, 65500])
+def test_masked_rows_only_far_into_the_batch(fd, orc, first_masked):
+    """Every masked row lies beyond the first 2048 rows (beyond the producer's own scan for
+    its first unit): the units are then found through the CTA's compaction; results match."""
+    B, L, V = 2048, 32, 1024
+    w = syn.Workload("far", B, L, V, "bf16", 1.0, "target", 0.3, 4.0)
+    logits = syn.make_logits(w, seed=first_masked, device="cuda")
+    mask = np.zeros((B, L), np.uint8)
+    flat = mask.reshape(-1)
+    rng = np.random.default_rng(first_masked)
+    rows = rng.choice(np.arange(first_masked, B * L), size=min(300, B * L - first_masked),
+                      replace=False)
+    flat[rows] = 1
+    check_confidence(fd, orc, logits, mask)
+    assert check_select(fd, orc, logits, mask, 0, 0.75) <= 2
