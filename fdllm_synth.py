@@ -237,7 +237,8 @@ def build_synth_cuda(force: bool = False) -> str:
     nvcc = shutil.which("nvcc") or "/usr/local/cuda/bin/nvcc"
     os.makedirs(os.path.dirname(_SYNTH_LIB), exist_ok=True)
     subprocess.run([nvcc, "-gencode", "arch=compute_103a,code=sm_103a", "-O3", "-std=c++17",
-                    "-Xcompiler", "-fPIC", "-shared", _SYNTH_SRC, "-o", _SYNTH_LIB + ".tmp"],
+                    "-lineinfo", "-Xcompiler", "-fPIC", "-shared", _SYNTH_SRC, "-o",
+                    _SYNTH_LIB + ".tmp"],
                    check=True, capture_output=True, text=True)
     os.replace(_SYNTH_LIB + ".tmp", _SYNTH_LIB)
     return _SYNTH_LIB
