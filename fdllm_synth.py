@@ -38,7 +38,7 @@ class Workload:
     B: int
     L: int
     V: int
-    dtype: str                 # "bf16" | "fp32"
+    dtype: str                 # "bf16" | "fp16" | "fp32"
     sigma: float = 1.0         # noise standard deviation
     peak: str = "uniform"      # "uniform" | "zipf" | "levels" | "target" | "none"
     peak_lo: float = 0.0       # uniform: h ~ U[lo, hi]; target: u = 1 - 10^-a, a ~ U[lo, hi]
@@ -53,11 +53,11 @@ class Workload:
 
     @property
     def elem_bytes(self) -> int:
-        return 2 if self.dtype == "bf16" else 4
+        return 4 if self.dtype == "fp32" else 2
 
     @property
     def torch_dtype(self):
-        return torch.bfloat16 if self.dtype == "bf16" else torch.float32
+        return {"bf16": torch.bfloat16, "fp16": torch.float16, "fp32": torch.float32}[self.dtype]
 
 
 WORKLOADS = {
@@ -90,6 +90,11 @@ WORKLOADS = {
         "target_b8_l32_bf16", 8, 32, LLADA_VOCAB, "bf16", 1.0, "target", 0.3, 4.0,
         masked="frac_u01",
         description="B=8, L=32, confidence near u = 1 - 10^-a, a~U[0.3,4]"),
+    # Supplementary: fp16 logits (models that emit half precision).
+    "target_b8_l32_fp16": Workload(
+        "target_b8_l32_fp16", 8, 32, LLADA_VOCAB, "fp16", 1.0, "target", 0.3, 4.0,
+        masked="frac_u01",
+        description="B=8, L=32, fp16, confidence near u = 1 - 10^-a, a~U[0.3,4]"),
     "target_ties_b16_l64_fp32": Workload(
         "target_ties_b16_l64_fp32", 16, 64, LLADA_VOCAB, "fp32", 1.0, "levels",
         levels=(0.9, 0.99, 0.999, 0.9999), tie_group=8, level_is_target=True,
@@ -179,15 +184,16 @@ def make_logits(w: Workload, seed: int, device="cpu", step: int = 0,
         flat[rows, cols] += vals
     else:
         flat[rows, cols] = vals
-    return x.to(w.torch_dtype) if w.dtype == "bf16" else x
+    return x if w.dtype == "fp32" else x.to(w.torch_dtype)
 
 
 def host_bits(logits: torch.Tensor) -> np.ndarray:
-    """Exact host copy of device/host logits for the oracle: bf16 -> uint16 bits, fp32 as is."""
+    """Exact host copy of device/host logits for the oracle: bf16 -> uint16 bits, fp16 and
+    fp32 as they are."""
     t = logits.detach().to("cpu").contiguous()
     if t.dtype == torch.bfloat16:
         return t.view(torch.int16).numpy().view(np.uint16)
-    if t.dtype == torch.float32:
+    if t.dtype in (torch.float32, torch.float16):
         return t.numpy()
     raise TypeError(t.dtype)
 

@@ -21,9 +21,10 @@
  *   - Pointers named logits, mask, out_*, conf, argmax and workspace are DEVICE pointers
  *     owned by the caller; the library never frees them.  `stream` is a cudaStream_t
  *     (NULL = legacy default stream) passed as void* so this header needs no CUDA headers.
- *   - logits is [B, L, V] row-major with V contiguous; dtype FDLLM_BF16 (bfloat16) or
- *     FDLLM_FP32.  The base must be 16-byte aligned and V * sizeof(dtype) a multiple of 16
- *     (V % 8 == 0 for bf16, V % 4 == 0 for fp32); otherwise FDLLM_ERR_ALIGN.  A vocabulary
+ *   - logits is [B, L, V] row-major with V contiguous; dtype FDLLM_BF16 (bfloat16),
+ *     FDLLM_FP16 (IEEE half) or FDLLM_FP32.  The base must be 16-byte aligned and
+ *     V * sizeof(dtype) a multiple of 16 (V % 8 == 0 for bf16 and fp16, V % 4 == 0 for
+ *     fp32); otherwise FDLLM_ERR_ALIGN.  A vocabulary
  *     that is not a multiple can be padded with -inf columns, which change nothing.
  *   - mask is uint8 [B, L], nonzero = masked.  Only masked positions are read from logits.
  *   - Limits: 1 <= B, 1 <= L <= FDLLM_MAX_L, B * L <= FDLLM_MAX_ROWS, V >= 1.
@@ -46,7 +47,7 @@ extern "C" {
 #define FDLLM_MAX_L 1024       /* positions per batch row (one CTA sorts a row in smem) */
 #define FDLLM_MAX_ROWS 65536   /* B * L: masked-row compaction lives in shared memory */
 
-typedef enum { FDLLM_BF16 = 0, FDLLM_FP32 = 1 } fdllm_dtype;
+typedef enum { FDLLM_BF16 = 0, FDLLM_FP32 = 1, FDLLM_FP16 = 2 } fdllm_dtype;
 
 typedef enum {
     FDLLM_PROFILE = 0,   /* Frechet profile rule, Sec. 3: param = f, margin delta = 1 - f */

@@ -23,7 +23,7 @@ import threading
 import numpy as np
 
 PROFILE, FACTOR, THRESHOLD = 0, 1, 2
-BF16, FP32, F64 = 0, 1, 2
+BF16, FP32, F64, F16 = 0, 1, 2, 3
 
 HERE = os.path.dirname(os.path.abspath(__file__))
 SOURCE = os.path.join(HERE, "fdllm_oracle.c")
@@ -63,7 +63,8 @@ def _ptr(a: np.ndarray) -> int:
 
 
 def _logits_view(logits: np.ndarray):
-    """Accept fp32 or fp64 arrays, or bf16 given as raw uint16 bits; return (array, code)."""
+    """Accept fp16, fp32 or fp64 arrays, or bf16 given as raw uint16 bits; return (array,
+    code)."""
     a = np.ascontiguousarray(logits)
     if a.dtype == np.uint16:
         return a, BF16
@@ -71,8 +72,10 @@ def _logits_view(logits: np.ndarray):
         return a, FP32
     if a.dtype == np.float64:
         return a, F64
-    raise TypeError("oracle logits must be float32, float64 or uint16 (bf16 bits), got %s"
-                    % a.dtype)
+    if a.dtype == np.float16:
+        return a, F16
+    raise TypeError("oracle logits must be float16, float32, float64 or uint16 (bf16 bits), "
+                    "got %s" % a.dtype)
 
 
 class Oracle:
@@ -100,6 +103,8 @@ class Oracle:
         lib.oracle_decode_loop.restype = i64
         lib.oracle_synth_block_hidden.argtypes = [p, p, i64, i64, i64, i64, p, u64, u64, d]
         lib.oracle_synth_block_hidden.restype = None
+        lib.oracle_half_to_double.argtypes = [p, i64, p]
+        lib.oracle_half_to_double.restype = None
         lib.oracle_lmhead_logits.argtypes = [p, p, i64, i64, i64, p, p, p, i32]
         lib.oracle_lmhead_logits.restype = None
         self.lib = lib
@@ -144,6 +149,13 @@ class Oracle:
         self.lib.oracle_profile_terms(_ptr(c), _ptr(m), B, L, _ptr(G), _ptr(F), _ptr(Bn),
                                       _ptr(order))
         return dict(G=G, F=F, B=Bn, order=order)
+
+    def half_to_double(self, bits: np.ndarray) -> np.ndarray:
+        """The oracle's fp16 widening of raw half bit patterns (uint16) to float64."""
+        b = np.ascontiguousarray(bits, np.uint16).reshape(-1)
+        out = np.zeros(b.shape, np.float64)
+        self.lib.oracle_half_to_double(_ptr(b), b.size, _ptr(out))
+        return out
 
     def lmhead_logits(self, hidden_bits: np.ndarray, w_bits: np.ndarray, mask=None,
                       with_abs: bool = False, nthreads: int = 1):

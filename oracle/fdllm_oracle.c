@@ -18,13 +18,32 @@
 #include <omp.h>
 #endif
 
+/* IEEE binary16 bits to double, exactly, from the format's definition: sign, 5 exponent
+ * bits with bias 15, 10 fraction bits; exponent 0 holds zero and the subnormals
+ * (fraction x 2^-24), exponent 31 the infinities and NaNs. */
+static double half_to_double(uint16_t h)
+{
+    const int sign = (h >> 15) & 1, e = (h >> 10) & 0x1F, frac = h & 0x3FF;
+    double v;
+    if (e == 0)
+        v = ldexp((double)frac, -24);
+    else if (e == 31)
+        v = frac ? NAN : INFINITY;
+    else
+        v = ldexp((double)(1024 + frac), e - 25);
+    return sign ? -v : v;
+}
+
 /* One logit widened to double.  bf16 is the upper half of an IEEE fp32 word, so the
- * widening is exact; fp64 logits (the LM head's exact products) are taken as they are. */
+ * widening is exact, as is the half's; fp64 logits (the LM head's exact products) are taken
+ * as they are. */
 static double logit_at(const void *logits, int dtype, int64_t i)
 {
     float f;
     if (dtype == ORACLE_F64)
         return ((const double *)logits)[i];
+    if (dtype == ORACLE_F16)
+        return half_to_double(((const uint16_t *)logits)[i]);
     if (dtype == ORACLE_BF16) {
         uint32_t u = (uint32_t)((const uint16_t *)logits)[i] << 16;
         memcpy(&f, &u, sizeof f);
@@ -586,4 +605,12 @@ void oracle_synth_block_hidden(uint16_t *out, const uint8_t *mask, int64_t B, in
                 out[row * H + j] = bf16_round(hj);
             }
         }
+}
+
+/* The widening of oracle_confidence's fp16 input, exposed for its pin: n IEEE half bit
+ * patterns to doubles. */
+void oracle_half_to_double(const uint16_t *h, int64_t n, double *out)
+{
+    for (int64_t i = 0; i < n; ++i)
+        out[i] = half_to_double(h[i]);
 }

@@ -12,7 +12,7 @@
  *
  * Conventions shared with the CUDA library's public interface (not its code):
  *   logits  [B, L, V] row-major, V contiguous; dtype 0 = bf16 (raw uint16 bits), 1 = fp32,
- *           2 = fp64 (exact LM-head products).
+ *           2 = fp64 (exact LM-head products), 3 = IEEE half (raw uint16 bits).
  *   mask    uint8 [B, L], 1 = masked; updated in place by the reveal (committed -> 0).
  *   mode    0 = profile (Frechet), 1 = factor, 2 = threshold.
  *   param   profile: f, with margin delta = 1 - f (matched parameter, Cor. factor-reduction);
@@ -27,7 +27,7 @@
 extern "C" {
 #endif
 
-enum { ORACLE_BF16 = 0, ORACLE_FP32 = 1, ORACLE_F64 = 2 };
+enum { ORACLE_BF16 = 0, ORACLE_FP32 = 1, ORACLE_F64 = 2, ORACLE_F16 = 3 };
 enum { ORACLE_PROFILE = 0, ORACLE_FACTOR = 1, ORACLE_THRESHOLD = 2 };
 
 /* Per masked position (b,l): x_hat = lowest v attaining max_v logit, c = max_v softmax(v)
@@ -135,6 +135,9 @@ void oracle_lmhead_logits(const uint16_t *hidden, const uint16_t *w, int64_t row
 void oracle_synth_block_hidden(uint16_t *out, const uint8_t *mask, int64_t B, int64_t L,
                                int64_t H, int64_t V, const uint16_t *w, uint64_t seed,
                                uint64_t step, double beta_max);
+
+/* IEEE half bit patterns to doubles (the fp16 widening of oracle_confidence). */
+void oracle_half_to_double(const uint16_t *h, int64_t n, double *out);
 
 #ifdef __cplusplus
 }

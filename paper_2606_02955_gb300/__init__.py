@@ -26,7 +26,7 @@ __all__ = [
     "fdllm_gather_masked_rows", "fdllm_decode_loop_lmhead",
 ]
 
-BF16, FP32 = 0, 1
+BF16, FP32, FP16 = 0, 1, 2
 PROFILE, FACTOR, THRESHOLD = 0, 1, 2
 ROW_NONFINITE, ROW_DEVICE_ERROR = -1, -2
 OK, ERR_ARG, ERR_ALIGN, ERR_NONFINITE, ERR_CUDA, ERR_WORKSPACE, ERR_DEVICE = range(7)
@@ -128,7 +128,9 @@ def _dtype_code(t: torch.Tensor) -> int:
         return BF16
     if t.dtype == torch.float32:
         return FP32
-    raise TypeError("logits must be bfloat16 or float32, got %s" % t.dtype)
+    if t.dtype == torch.float16:
+        return FP16
+    raise TypeError("logits must be bfloat16, float16 or float32, got %s" % t.dtype)
 
 
 def _stream(stream) -> int:

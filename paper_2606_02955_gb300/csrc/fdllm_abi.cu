@@ -37,9 +37,9 @@ Layout layout_for(int64_t rows, int64_t row_bytes)
     return l;
 }
 
-bool valid_dtype(int d) { return d == FDLLM_BF16 || d == FDLLM_FP32; }
+bool valid_dtype(int d) { return d == FDLLM_BF16 || d == FDLLM_FP32 || d == FDLLM_FP16; }
 bool valid_mode(int m) { return m == FDLLM_PROFILE || m == FDLLM_FACTOR || m == FDLLM_THRESHOLD; }
-int esize_of(int d) { return d == FDLLM_BF16 ? 2 : 4; }
+int esize_of(int d) { return d == FDLLM_FP32 ? 4 : 2; }
 
 fdllm_status check_shape(int B, int L, int V)
 {
@@ -133,7 +133,7 @@ fdllm_status run_select(const void *logits, int dtype, int B, int L, int V, uint
 {
     VocabReduceArgs ra = reduce_args(logits, dtype, B, L, V, mask, ws, lay);
     ra.pdl = pdl;
-    if (launch_vocab_reduce(ra, esize_of(dtype), stream) != cudaSuccess)
+    if (launch_vocab_reduce(ra, dtype, stream) != cudaSuccess)
         return FDLLM_ERR_CUDA;
     ProfileSelectArgs pa;
     pa.units_per_row = ra.units_per_row;
@@ -344,7 +344,7 @@ fdllm_status fdllm_confidence(const void *logits, int dtype, int B, int L, int V
         return st;
     VocabReduceArgs ra = reduce_args(logits, dtype, B, L, V, mask, static_cast<uint8_t *>(ws),
                                      lay);
-    if (launch_vocab_reduce(ra, esize_of(dtype), s) != cudaSuccess)
+    if (launch_vocab_reduce(ra, dtype, s) != cudaSuccess)
         return FDLLM_ERR_CUDA;
     FinalizeArgs fa;
     fa.mask = mask;

@@ -75,7 +75,7 @@ inline UnitPlan plan_units(int64_t row_bytes)
 
 // Enqueue the vocab reduction on all SMs, as a programmatic dependent of the previous
 // kernel on the stream.
-cudaError_t launch_vocab_reduce(const VocabReduceArgs &a, int esize, cudaStream_t stream);
+cudaError_t launch_vocab_reduce(const VocabReduceArgs &a, int dtype, cudaStream_t stream);
 
 // One thread waits, bounded by limit_ns, on an mbarrier that never completes.
 cudaError_t launch_bounded_wait_probe(uint32_t *status, uint64_t limit_ns, cudaStream_t stream);
@@ -165,10 +165,30 @@ __device__ __forceinline__ float ex2_mufu(float x)
     return y;
 }
 
-// S re-based from reference a2 to b2 (both already scaled by log2e): S * 2^(a2 - b2).
-__device__ __forceinline__ float rebase(float S, float a2, float b2)
+// Every partial (M, S) holds S = sum exp(x - M) relative to its own maximum M exactly.
+//
+// Sums are accumulated as 2^(x * s - r2) with a scale s and an fp32 reference r2.
+//  * |ref| < kBigRef: s = log2e, r2 = round(ref * log2e).  The FMA forms x * log2e exactly;
+//    the rounding residual r = ref * log2e - r2 is at most half an ulp of a value below 2^31,
+//    so |r| <= 64, and it scales every term by the same 2^r, which rebase_scaled removes.
+//  * |ref| >= kBigRef: s = 1, r2 = ref.  Distinct fp32 values there are at least 64 apart, so
+//    every term but those equal to ref is below 2^-64 of them (under e^-64 in exp as well):
+//    the sum counts the maxima, and the terms it drops weigh under 2^-40 for V < 2^24.
+constexpr float kBigRef = 0x1p30f;
+
+// S accumulated against (s, r2) -> relative to M: S * 2^(r2 - M s).  M s - r2 is formed in
+// one FMA from the exact product, so the rounding of r2 cancels instead of scaling S.
+__device__ __forceinline__ float rebase_scaled(float S, float s, float r2, float M)
 {
-    return S != 0.0f ? S * ex2_mufu(a2 - b2) : 0.0f;  // keeps NaN, avoids 0 * inf
+    return S != 0.0f ? S * ex2_mufu(-fmaf(M, s, -r2)) : 0.0f;  // keeps NaN, avoids 0 * inf
+}
+
+// S relative to the maximum a -> relative to b >= a: S * exp(a - b).  a - b is exact when the
+// two are within a factor of two and carries a relative 2^-24 otherwise, where the factor is
+// below exp(-|b| / 2).  Infinite or NaN maxima give NaN, reported by the caller.
+__device__ __forceinline__ float rebase(float S, float a, float b)
+{
+    return S != 0.0f ? S * ex2_mufu((a - b) * kLog2e) : 0.0f;
 }
 
 // Position result from its units, folded in unit order (a fixed order, so identical rows
@@ -198,13 +218,12 @@ __device__ __forceinline__ void combine_position(const UnitPartial *p, int upr, 
         for (int j = 0; j < 8; ++j)
             if (j < cnt)
                 Mb = fmaxf(Mb, Mj[j]);
-        const float Mb2 = Mb * kLog2e;
-        float Sb = rebase(S, M * kLog2e, Mb2);
+        float Sb = rebase(S, M, Mb);
         uint32_t ib = (M == Mb) ? idx : kNoIdx;
 #pragma unroll
         for (int j = 0; j < 8; ++j)
             if (j < cnt) {
-                Sb += rebase(Sj[j], Mj[j] * kLog2e, Mb2);
+                Sb += rebase(Sj[j], Mj[j], Mb);
                 if (Mj[j] == Mb && ib == kNoIdx)
                     ib = Ij[j];
             }

@@ -46,9 +46,10 @@ extern "C" fdllm_status fdllm_gather_masked_rows(const void *src, void *dst, int
                                                  int L, int V, const uint8_t *mask, void *stream)
 {
     if (!src || !dst || !mask || B < 1 || L < 1 || L > FDLLM_MAX_L || V < 1 ||
-        (int64_t)B * L > FDLLM_MAX_ROWS || (dtype != FDLLM_BF16 && dtype != FDLLM_FP32))
+        (int64_t)B * L > FDLLM_MAX_ROWS ||
+        (dtype != FDLLM_BF16 && dtype != FDLLM_FP32 && dtype != FDLLM_FP16))
         return FDLLM_ERR_ARG;
-    const int64_t row_bytes = (int64_t)V * (dtype == FDLLM_BF16 ? 2 : 4);
+    const int64_t row_bytes = (int64_t)V * (dtype == FDLLM_FP32 ? 4 : 2);
     if (row_bytes % 16 != 0 || (reinterpret_cast<uintptr_t>(src) & 15u) ||
         (reinterpret_cast<uintptr_t>(dst) & 15u))
         return FDLLM_ERR_ALIGN;

@@ -339,8 +339,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                     }
                 }
-                // Pass 2: sum of exp(x - M) = 2^(x log2e - M log2e), four partial sums.
-                const float M2 = M * kLog2e;
+                // Pass 2: sum of exp(x - M) = 2^(x sc - M2), four partial sums, with the
+                // scale sc and reference M2 of rebase_scaled (sc = 1 and M2 = M for |M| at or
+                // beyond kBigRef, where only x == M contributes).
+                const bool big = !(fabsf(M) < kBigRef);
+                const float sc = big ? 1.0f : kLog2e;
+                const float M2 = big ? M : M * kLog2e;
                 float S4[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll 1
                 for (int c = 0; c < (BN + 31) / 32; ++c) {
@@ -349,7 +353,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int j = 0; j < 32; ++j) {
                         const int col = col0 + c * 32 + j;
                         if (c * 32 + j < BN && col < a.V)
-                            S4[j & 3] += ex2_mufu(fmaf(v[j], kLog2e, -M2));
+                            S4[j & 3] += ex2_mufu(fmaf(v[j], sc, -M2));
                     }
                 }
                 tc::fence_before_sync();
@@ -359,7 +363,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (r < R) {
                     UnitPartial p;
                     p.M = nan ? __int_as_float(0x7FC00000) : M;
-                    p.S = (S4[0] + S4[1]) + (S4[2] + S4[3]);
+                    // relative to M exactly; a tile with no finite logit adds exactly 0
+                    p.S = M == -INFINITY
+                              ? 0.0f
+                              : rebase_scaled((S4[0] + S4[1]) + (S4[2] + S4[3]), sc, M2, M);
                     p.idx = idx;
                     p.pad = 0;
                     a.partials[(int64_t)r * a.n_tiles + n] = p;
@@ -477,8 +484,7 @@ __device__ __forceinline__ Part fold(const Part &x, const Part &y)
     Part r;
     r.nan = x.nan || y.nan;
     r.M = fmaxf(x.M, y.M);
-    const float M2 = r.M * kLog2e;
-    r.S = rebase(x.S, x.M * kLog2e, M2) + rebase(y.S, y.M * kLog2e, M2);
+    r.S = rebase(x.S, x.M, r.M) + rebase(y.S, y.M, r.M);
     const uint32_t ix = x.M == r.M ? x.idx : kNoIdx;
     const uint32_t iy = y.M == r.M ? y.idx : kNoIdx;
     r.idx = ix < iy ? ix : iy;

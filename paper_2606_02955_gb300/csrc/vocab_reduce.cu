@@ -14,14 +14,15 @@
 //    with 1-D bulk copies (cp.async.bulk, completion on mbarriers); chunk metadata travels
 //    with the stage.
 //  * NW math warps read the ring with conflict-free 16-byte shared loads.  Per lane: running
-//    max and the index of its first vector; per warp: a lagging reference `ref` for the sum
-//    of 2^(x*log2e - ref2), raised (with one rescale) only when a logit exceeds it by
+//    max and the index of its first maximal logit; per warp: a lagging reference `ref` for
+//    the sum of 2^(x*log2e - ref2), raised (with one rescale) only when a logit exceeds it by
 //    kRebaseSlack, so a logit costs half a packed f32x2 FMA, one MUFU ex2 and half a packed
-//    f32x2 add; the vector max uses packed bf16x2 max for bf16.
+//    f32x2 add; the vector max uses packed bf16x2 / f16x2 max for 16-bit logits.  Beyond
+//    |ref| = kBigRef the same FMA runs with scale 1 (see rebase_scaled).
 //  * At the end of a unit each math warp reduces its lanes (redux + shuffles) and queues
-//    (M, S, vec) for the epilogue warp, which combines the warps in a fixed order and stores
-//    the unit's partial.  The consumer kernel (profile select, or finalize) folds a position's
-//    units in unit order and resolves the argmax element inside the winning 16-byte vector.
+//    (M, S, idx), S re-based to M exactly, for the epilogue warp, which combines the warps in
+//    a fixed order and stores the unit's partial.  The consumer kernel (profile select, or
+//    finalize) folds a position's units in unit order.
 #include <cfloat>
 #include <cmath>
 #include <cstdio>
@@ -65,6 +66,23 @@ __device__ __forceinline__ uint32_t hmax2_nan(uint32_t a, uint32_t b)
     return d;
 }
 
+__device__ __forceinline__ uint32_t hmax2_nan_f16(uint32_t a, uint32_t b)
+{
+    uint32_t d;
+    asm("max.NaN.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+    return d;
+}
+
+// fp16 (IEEE binary16) -> fp32, exact.
+__device__ __forceinline__ float f16_to_f32(uint32_t h)
+{
+    float f;
+    asm("{\n\t.reg .b16 x;\n\tcvt.u16.u32 x, %1;\n\tcvt.f32.f16 %0, x;\n\t}"
+        : "=f"(f)
+        : "r"(h));
+    return f;
+}
+
 // Packed fp32 pairs (Blackwell f32x2 arithmetic); element order inside a pair is irrelevant
 // here because every operation is elementwise.
 __device__ __forceinline__ uint64_t pack2(float lo, float hi)
@@ -100,11 +118,12 @@ __device__ __forceinline__ uint64_t fmul2(uint64_t a, uint64_t b)
     return d;
 }
 
-template <int ESIZE>
+// Keyed by the library's dtype code (fdllm_dtype).
+template <int KIND>
 struct VecOps;
 
 template <>
-struct VecOps<2> {  // 8 x bf16 per 16-byte vector; widening to fp32 is exact
+struct VecOps<FDLLM_BF16> {  // 8 x bf16 per 16-byte vector; widening to fp32 is exact
     static constexpr uint32_t kPadWord = 0xFF80FF80u;  // two bf16 -inf
     // max of the 8 logits; NaN if any is NaN
     __device__ __forceinline__ static float vmax(const uint4 &r)
@@ -141,7 +160,44 @@ struct VecOps<2> {  // 8 x bf16 per 16-byte vector; widening to fp32 is exact
 };
 
 template <>
-struct VecOps<4> {  // 4 x fp32 per 16-byte vector
+struct VecOps<FDLLM_FP16> {  // 8 x fp16 per 16-byte vector; widening to fp32 is exact
+    static constexpr uint32_t kPadWord = 0xFC00FC00u;  // two fp16 -inf
+    // max of the 8 logits; NaN if any is NaN
+    __device__ __forceinline__ static float vmax(const uint4 &r)
+    {
+        const uint32_t m = hmax2_nan_f16(hmax2_nan_f16(r.x, r.y), hmax2_nan_f16(r.z, r.w));
+        return fmax_nan(f16_to_f32(m & 0xFFFFu), f16_to_f32(m >> 16));
+    }
+    __device__ __forceinline__ static uint64_t pair(uint32_t w)
+    {
+        return pack2(f16_to_f32(w & 0xFFFFu), f16_to_f32(w >> 16));
+    }
+    __device__ __forceinline__ static void pairs(const uint4 &r, uint64_t (&p)[4])
+    {
+        p[0] = pair(r.x);
+        p[1] = pair(r.y);
+        p[2] = pair(r.z);
+        p[3] = pair(r.w);
+    }
+    // first element of the vector equal to M (8 if none)
+    __device__ __forceinline__ static uint32_t first_index(const uint4 &r, float M)
+    {
+        const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+        uint32_t hit = 8;
+#pragma unroll
+        for (int e = 7; e >= 0; --e) {
+            const uint32_t bits = (e & 1) ? (w[e >> 1] >> 16) : (w[e >> 1] & 0xFFFFu);
+            if (f16_to_f32(bits) == M)
+                hit = e;
+        }
+        return hit;
+    }
+    static constexpr int kPairs = 4;
+    static constexpr int kElems = 8;
+};
+
+template <>
+struct VecOps<FDLLM_FP32> {  // 4 x fp32 per 16-byte vector
     static constexpr uint32_t kPadWord = 0xFF800000u;  // fp32 -inf
     __device__ __forceinline__ static float vmax(const uint4 &r)
     {
@@ -177,7 +233,7 @@ __device__ __forceinline__ UnitPartial warp_combine(UnitPartial p, bool valid)
         p.idx = kNoIdx;
     }
     const float M = unordered(__reduce_max_sync(0xFFFFFFFFu, ordered(p.M)));
-    float s = rebase(p.S, p.M * kLog2e, M * kLog2e);
+    float s = rebase(p.S, p.M, M);
 #pragma unroll
     for (int o = 16; o >= 1; o >>= 1)
         s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
@@ -232,9 +288,9 @@ constexpr size_t smem_bytes()
     return (size_t)STAGES * CHUNK + sizeof(Smem<NW, STAGES>);
 }
 
-// ESIZE: bytes per logit; NW: math warps; STAGES x CHUNK: the shared-memory ring;
+// KIND: the logits' dtype code; NW: math warps; STAGES x CHUNK: the shared-memory ring;
 // EVICT: L2 evict-first hint on the stream.
-template <int ESIZE, int NW, int STAGES, int CHUNK, bool EVICT>
+template <int KIND, int NW, int STAGES, int CHUNK, bool EVICT>
 __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const VocabReduceArgs a)
 {
     constexpr int kStages = STAGES;
@@ -245,7 +301,7 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
     Smem<NW, STAGES> &sm =
         *reinterpret_cast<Smem<NW, STAGES> *>(smem_raw + (size_t)kStages * kChunkBytes);
     constexpr int kWarps = NW + 2;
-    using Ops = VecOps<ESIZE>;
+    using Ops = VecOps<KIND>;
     constexpr int kP = Ops::kPairs;
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -426,18 +482,21 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
         const int ct = threadIdx.x - 32;
         constexpr int kPer = kChunkVecs / (NW * 32);
         static_assert(kChunkVecs % (NW * 32) == 0, "chunk must split evenly over math warps");
-        const uint64_t log2e2 = pack2(kLog2e, kLog2e);
         float m = -INFINITY;     // lane max (the first logit attaining it wins ties)
         float mnan = -INFINITY;  // lane max propagating NaN (NaN detection, rebase trigger)
         uint32_t idx = kNoIdx;   // row-relative index of that first logit
         uint64_t acc[kP];
-        float ref = -FLT_MAX, ref2 = -FLT_MAX;  // warp-uniform reference
+        // Warp-uniform reference ref, its fp32 form ref2 and the scale sc of rebase_scaled
+        // (sc = log2e, or 1 for |ref| >= kBigRef).  Before the first finite logit ref = -inf,
+        // so that logit always rebases, and the sums stay 0.
+        float ref = -INFINITY, ref2 = -FLT_MAX, sc = kLog2e;
+        uint64_t sc2 = pack2(kLog2e, kLog2e);
 #pragma unroll
         for (int q = 0; q < kP; ++q)
             acc[q] = 0;
 
         // One chunk: vector maxima and the first maximal logit, the reference update, then
-        // 2^(x*log2e - ref2) accumulated.  FULL: every vector of the chunk exists.
+        // 2^(x*sc - ref2) accumulated.  FULL: every vector of the chunk exists.
         auto process_chunk = [&](auto full_tag, const uint4 *buf, const ChunkMeta &cm) {
             constexpr bool FULL = decltype(full_tag)::value;
             const uint4 pad = make_uint4(Ops::kPadWord, Ops::kPadWord, Ops::kPadWord,
@@ -472,14 +531,21 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
             }
             if (__any_sync(0xFFFFFFFFu, mnan > ref + kRebaseSlack)) {
                 const float wmax = unordered(__reduce_max_sync(0xFFFFFFFFu, ordered(mnan)));
-                const float r2 = wmax * kLog2e;
-                const float f = ex2_mufu(ref2 - r2);
+                const bool big = !(fabsf(wmax) < kBigRef);
+                const float r2 = big ? wmax : wmax * kLog2e;
+                // Old sums -> the new reference: 2^(ref2 - r2) between two fp32 references.
+                // Where either reference has magnitude >= kBigRef every old logit lies at
+                // least 56 below the new maximum and the old terms are dropped (under e^-56
+                // each); the first sums are 0.
+                const float f = (big || sc != kLog2e) ? 0.0f : ex2_mufu(ref2 - r2);
                 const uint64_t f2 = pack2(f, f);
 #pragma unroll
                 for (int q = 0; q < kP; ++q)
                     acc[q] = fmul2(acc[q], f2);
                 ref = wmax;
                 ref2 = r2;
+                sc = big ? 1.0f : kLog2e;
+                sc2 = pack2(sc, sc);
             }
             const uint64_t nref2 = pack2(-ref2, -ref2);
 #pragma unroll
@@ -489,7 +555,7 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
 #pragma unroll
                 for (int q = 0; q < kP; ++q) {
                     float t0, t1;
-                    unpack2(ffma2(p[q], log2e2, nref2), t0, t1);
+                    unpack2(ffma2(p[q], sc2, nref2), t0, t1);
                     acc[q] = fadd2(acc[q], pack2(ex2_mufu(t0), ex2_mufu(t1)));
                 }
             }
@@ -533,7 +599,7 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
             // NaN anywhere poisons the sum; a warp that saw no finite logit adds exactly 0.
             const bool bad = __any_sync(0xFFFFFFFFu, mnan != mnan);
             p.S = bad ? __int_as_float(0x7FC00000)
-                      : (p.M == -INFINITY ? 0.0f : rebase(S, ref2, p.M * kLog2e));
+                      : (p.M == -INFINITY ? 0.0f : rebase_scaled(S, sc, ref2, p.M));
             p.idx = __reduce_min_sync(0xFFFFFFFFu, m == p.M ? idx : kNoIdx);
             p.pad = 0;
             if (lane == 0) {
@@ -548,8 +614,10 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
             m = -INFINITY;
             mnan = -INFINITY;
             idx = kNoIdx;
-            ref = -FLT_MAX;
+            ref = -INFINITY;
             ref2 = -FLT_MAX;
+            sc = kLog2e;
+            sc2 = pack2(kLog2e, kLog2e);
 #pragma unroll
             for (int j = 0; j < kP; ++j)
                 acc[j] = 0;
@@ -593,7 +661,7 @@ __global__ void finalize_kernel(const FinalizeArgs a)
     a.out_tok[row] = tok;
 }
 
-template <int ESIZE, int NW, int STAGES, int CHUNK, bool EVICT>
+template <int KIND, int NW, int STAGES, int CHUNK, bool EVICT>
 cudaError_t launch_variant(const VocabReduceArgs &a, cudaStream_t stream)
 {
     static int attr_done[64] = {0};
@@ -606,7 +674,7 @@ cudaError_t launch_variant(const VocabReduceArgs &a, cudaStream_t stream)
         return cudaErrorInvalidDevice;
     constexpr size_t smem = smem_bytes<NW, STAGES, CHUNK>();
     static_assert(smem <= 227 * 1024, "ring does not fit in shared memory");
-    auto *kern = vocab_reduce_kernel<ESIZE, NW, STAGES, CHUNK, EVICT>;
+    auto *kern = vocab_reduce_kernel<KIND, NW, STAGES, CHUNK, EVICT>;
     if (!attr_done[dev]) {
         err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (err != cudaSuccess)
@@ -633,14 +701,14 @@ cudaError_t launch_variant(const VocabReduceArgs &a, cudaStream_t stream)
 
 // Tuning table (math warps, ring stages x chunk bytes, L2 hint).  Entry 0 is the
 // configuration in use; FDLLM_K1_VARIANT=<index> selects another for measurements.
-template <int ESIZE>
-cudaError_t launch_esize(const VocabReduceArgs &a, cudaStream_t stream, int which)
+template <int KIND>
+cudaError_t launch_kind(const VocabReduceArgs &a, cudaStream_t stream, int which)
 {
     switch (which) {
-    case 1: return launch_variant<ESIZE, 16, 3, 65536, false>(a, stream);
-    case 2: return launch_variant<ESIZE, 8, 3, 65536, true>(a, stream);
-    case 3: return launch_variant<ESIZE, 16, 6, 32768, true>(a, stream);
-    default: return launch_variant<ESIZE, 16, 3, 65536, true>(a, stream);
+    case 1: return launch_variant<KIND, 16, 3, 65536, false>(a, stream);
+    case 2: return launch_variant<KIND, 8, 3, 65536, true>(a, stream);
+    case 3: return launch_variant<KIND, 16, 6, 32768, true>(a, stream);
+    default: return launch_variant<KIND, 16, 3, 65536, true>(a, stream);
     }
 }
 
@@ -671,10 +739,14 @@ cudaError_t launch_bounded_wait_probe(uint32_t *status, uint64_t limit_ns, cudaS
     return cudaGetLastError();
 }
 
-cudaError_t launch_vocab_reduce(const VocabReduceArgs &a, int esize, cudaStream_t stream)
+cudaError_t launch_vocab_reduce(const VocabReduceArgs &a, int dtype, cudaStream_t stream)
 {
     const int which = variant_index();
-    return esize == 2 ? launch_esize<2>(a, stream, which) : launch_esize<4>(a, stream, which);
+    switch (dtype) {
+    case FDLLM_BF16: return launch_kind<FDLLM_BF16>(a, stream, which);
+    case FDLLM_FP16: return launch_kind<FDLLM_FP16>(a, stream, which);
+    default: return launch_kind<FDLLM_FP32>(a, stream, which);
+    }
 }
 
 cudaError_t launch_finalize(const FinalizeArgs &a, cudaStream_t stream)

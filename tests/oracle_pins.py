@@ -65,14 +65,15 @@ def G_of_subset(cs):
 def pin_confidence_vs_torch(o):
     """c = exp(M - logsumexp) and x_hat = first argmax, against torch float64 (Sec. 3)."""
     rng = np.random.default_rng(11)
-    for dt in ("fp32", "bf16"):
+    for dt in ("fp32", "bf16", "fp16"):
         for V in (1, 2, 7, 1000, 4099):
             B, L = 3, 5
             x = rng.normal(0.0, 3.0, (B, L, V)).astype(np.float32)
             if V > 2:
                 x[0, 1, 1::2] = -np.inf          # -inf entries contribute nothing
                 x[1, 2, : V // 2] = x[1, 2, V // 2]  # repeated values
-            arr = bf16_bits(x) if dt == "bf16" else x
+            arr = bf16_bits(x) if dt == "bf16" else (x.astype(np.float16) if dt == "fp16"
+                                                     else x)
             mask = (rng.random((B, L)) < 0.7).astype(np.uint8)
             mask[0, 1] = mask[1, 2] = 1
             conf, tok, bad = o.confidence(arr, mask)
@@ -84,6 +85,17 @@ def pin_confidence_vs_torch(o):
             np.testing.assert_allclose(conf[mk], ref_c[mk], rtol=1e-12, atol=0)
             assert np.array_equal(tok[mk], ref_t[mk])
             assert np.all(tok[~mk] == -1)
+
+
+def pin_half_widening(o):
+    """The fp16 widening: every one of the 65536 half bit patterns against numpy's own
+    float16 -> float64 conversion (NaN patterns: NaN)."""
+    bits = np.arange(65536, dtype=np.uint32).astype(np.uint16)
+    got = o.half_to_double(bits)
+    ref = bits.view(np.float16).astype(np.float64)
+    nan = np.isnan(ref)
+    assert np.array_equal(np.isnan(got), nan)
+    assert np.array_equal(got[~nan], ref[~nan])
 
 
 def pin_confidence_closed_forms(o):
@@ -509,5 +521,5 @@ ALL_PINS = [
     pin_matched_dominance, pin_greedy_equivalence, pin_monotone_prefix, pin_special_cases,
     pin_reveal_and_ties, pin_end_to_end, pin_robust_zero_eta_is_profile,
     pin_robust_calibration_penalty, pin_robust_bruteforce, pin_robust_monotone_and_clipped,
-    pin_bonus_terms,
+    pin_bonus_terms, pin_half_widening,
 ]

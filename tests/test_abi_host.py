@@ -68,11 +68,12 @@ A2 = 0x10002
     ((A16, 0, 2, 1025, 1024), ERR_ARG),        # L > 1024
     ((A16, 0, 128, 1024, 1024), ERR_ARG),      # B * L > 65536
     ((A16, 0, 2, 32, 0), ERR_ARG),             # V = 0
-    ((A16, 2, 2, 32, 1024), ERR_ARG),          # unknown dtype
+    ((A16, 3, 2, 32, 1024), ERR_ARG),          # unknown dtype
     ((None, 0, 2, 32, 1024), ERR_ARG),         # null logits
     ((A2, 0, 2, 32, 1024), ERR_ALIGN),         # logits not 16-byte aligned
     ((A16, 0, 2, 32, 1001), ERR_ALIGN),        # V * 2 not a multiple of 16
     ((A16, 1, 2, 32, 1002), ERR_ALIGN),        # V * 4 not a multiple of 16
+    ((A16, 2, 2, 32, 1001), ERR_ALIGN),        # fp16: V * 2 not a multiple of 16
 ])
 def test_select_rejects_bad_shapes(lib, args, want):
     logits, dtype, B, L, V = args
@@ -171,7 +172,7 @@ def test_gather_masked_rows_rejects(lib):
         lib.fdllm_gather_masked_rows(src, dst, dtype, B, L, V, mask, None)
     assert f(src=None) == ERR_ARG
     assert f(mask=None) == ERR_ARG
-    assert f(dtype=2) == ERR_ARG
+    assert f(dtype=3) == ERR_ARG
     assert f(L=1025) == ERR_ARG
     assert f(V=1001) == ERR_ALIGN
     assert f(src=A2) == ERR_ALIGN

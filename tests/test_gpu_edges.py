@@ -82,6 +82,55 @@ def test_nonfinite_rows(fd, orc):
     check_select(fd, orc, logits, mask_np, PROFILE, 0.75)
 
 
+@pytest.mark.parametrize("dtype", ["bf16", "fp16", "fp32"])
+def test_large_magnitude_logits(fd, orc, dtype):
+    """Logits far from 0: a row shifted by a large constant (softmax is shift-invariant), rows
+    filled with the type's most negative finite value (a common masking value), the largest
+    finite value tied twice, and (fp32, bf16) maxima on both sides of 2^30, where the sum
+    switches from the scaled FMA form to counting the maxima, up to 1e30 and beyond."""
+    np_t = {"bf16": np.float32, "fp16": np.float16, "fp32": np.float32}[dtype]
+    info = {"bf16": torch.finfo(torch.bfloat16), "fp16": torch.finfo(torch.float16),
+            "fp32": torch.finfo(torch.float32)}[dtype]
+    lo, hi = float(info.min), float(info.max)
+    V = 126464 if dtype != "fp16" else 8192
+    rng = np.random.default_rng(12)
+    x = rng.normal(0.0, 1.0, (2, 8, V))
+    x[0, 0] = x[0, 0] * 0.05 + (3.0e4 if dtype == "fp32" else 600.0)   # shifted, tight
+    x[0, 1] = lo                                                       # c = 1 / V
+    x[0, 2] = lo
+    x[0, 2, [5, V // 2, V - 1]] = rng.normal(0.0, 1.0, 3)              # a few ordinary values
+    x[0, 3, [7, V - 9]] = hi                                           # tied largest value
+    x[0, 4] = x[0, 4] - (3.0e4 if dtype == "fp32" else 600.0)          # shifted down
+    x[0, 5, V // 3] = hi / 2
+    x[0, 6] = -x[0, 6] ** 2 * 1e3                                      # wide negative spread
+    x[0, 6, 11] = 0.5
+    x[0, 7] = lo / 4
+    x[0, 7, [1, V // 3 + 1]] = lo / 8                                  # tied, all far below 0
+    if dtype != "fp16":
+        b = 2.0 ** 30
+        below = float(np.nextafter(np.float32(b), np.float32(0)))      # b - 64
+        x[1, 0, 3] = b                                                 # exactly the switch
+        x[1, 0, 9] = below                                             # e^-64 below it
+        x[1, 1] = -b
+        x[1, 1, ::7] = lo
+        x[1, 2, [0, 4000]] = below                                     # tied, scaled form
+        x[1, 3] = rng.normal(0.0, 1.0, V) * 1e30
+        x[1, 4] = -2.0 * b
+        x[1, 4, [17, V - 5]] = -b                                      # max -2^30, tied
+        x[1, 5, ::1000] = hi
+        x[1, 6] = x[1, 6] * 4.0 + 1e8                                  # rounding residual 8
+        x[1, 7] = x[1, 7] * 2.0 ** 24 + 2.0 ** 29                      # residual up to 32
+    else:
+        x[1, :4] = x[1, :4] * 8.0 + 60000.0 * np.sign(x[1, :4])
+    x = np.clip(x, lo, hi).astype(np_t)
+    logits = _bf16(x) if dtype == "bf16" else torch.from_numpy(x).cuda()
+    mask_np = np.ones((2, 8), np.uint8)
+    conf, tok, rc, rt = check_confidence(fd, orc, logits, mask_np)
+    assert abs(conf[0, 1] * V - 1.0) <= 1e-5 and tok[0, 1] == 0
+    assert abs(conf[0, 3] - 0.5) <= 1e-6 and tok[0, 3] == 7
+    check_select(fd, orc, logits, mask_np, PROFILE, 0.75)
+
+
 def test_argmax_ties_across_chunks_and_ctas(fd, orc):
     """Equal maxima far apart in a row (different chunks and, at this size, different CTAs),
     and maxima in the last, ragged chunk: the lowest index must win."""

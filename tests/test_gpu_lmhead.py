@@ -103,6 +103,30 @@ def test_fused_confidence_matches_oracle_on_the_same_accumulators(fd, orc, clust
     assert np.isnan(g_conf[~mk]).all() and (g_tok[~mk] == -1).all()
 
 
+@pytest.mark.parametrize("k", [12, 26, 122])
+def test_fused_confidence_at_large_magnitude(fd, orc, cluster, k):
+    """Hidden states scaled by 2^k (exact in bf16): logits near 1e5 (k = 12), where the fp32
+    reference M log2e carries a rounding residual up to 4e-3; near 2^30 (k = 26), residuals
+    up to 64 and both forms of the epilogue's sum; up to 2^126.3 (k = 122), the maxima
+    counted."""
+    B, L, H, V = 2, 32, 256, 3000
+    h, w, mask_np = inputs(B, L, H, V, seed=31 + k)
+    h = h * (2.0 ** k)
+    conf, tok = fd.fdllm_lmhead_confidence(h, w, torch.from_numpy(mask_np).cuda())
+    torch.cuda.synchronize()
+    x32 = gpu_logits(fd, h, w, mask_np)
+    mk = mask_np.astype(bool)
+    assert np.isfinite(x32[mk]).all()
+    if k >= 26:
+        assert (np.abs(x32[mk]).max(axis=-1) >= 2.0 ** 30).any()
+    rc, rt, bad = orc.confidence(x32, mask_np, nthreads=oracle_threads())
+    assert bad == 0
+    g_conf, g_tok = conf.cpu().numpy().astype(np.float64), tok.cpu().numpy()
+    assert np.array_equal(g_tok[mk], rt[mk])
+    rel = np.abs(g_conf[mk] - rc[mk]) / rc[mk]
+    assert rel.max() <= CONF_RTOL, rel.max()
+
+
 @pytest.mark.parametrize("mode,param", [(oracle.PROFILE, 1.0), (oracle.PROFILE, 0.75),
                                         (oracle.FACTOR, 1.0), (oracle.THRESHOLD, 0.9)])
 @pytest.mark.parametrize("B,L,H,V", [(4, 32, 512, 5000), (8, 64, 256, 3000)])

@@ -26,7 +26,7 @@ def _mask(B, L, seed, frac=0.7, empty_rows=()):
     return m
 
 
-@pytest.mark.parametrize("dtype", ["bf16", "fp32"])
+@pytest.mark.parametrize("dtype", ["bf16", "fp16", "fp32"])
 @pytest.mark.parametrize("V", [8, 1000, 8200, 20000, 126464])
 @pytest.mark.parametrize("B,L", [(1, 1), (3, 7), (2, 33), (4, 64)])
 def test_confidence_shapes(fd, orc, dtype, V, B, L):
@@ -39,7 +39,7 @@ def test_confidence_shapes(fd, orc, dtype, V, B, L):
 
 @pytest.mark.parametrize("name", ["single_block_b1_l32_bf16", "mixed_mask_b8_l32_bf16",
                                   "tie_groups_b16_l64_fp32", "target_b8_l32_bf16",
-                                  "target_ties_b16_l64_fp32"])
+                                  "target_ties_b16_l64_fp32", "target_b8_l32_fp16"])
 def test_confidence_workloads_full_vocab(fd, orc, name):
     w = W[name]
     logits = syn.make_logits(w, seed=101, device="cuda")
@@ -51,7 +51,7 @@ def test_confidence_workloads_full_vocab(fd, orc, name):
                                         (FACTOR, 0.5), (FACTOR, 2.0), (THRESHOLD, 0.9),
                                         (THRESHOLD, 0.5)])
 @pytest.mark.parametrize("name", ["single_block_b1_l32_bf16", "mixed_mask_b8_l32_bf16",
-                                  "target_b8_l32_bf16"])
+                                  "target_b8_l32_bf16", "target_b8_l32_fp16"])
 def test_select_workloads(fd, orc, name, mode, param):
     w = W[name]
     logits = syn.make_logits(w, seed=202, device="cuda")
@@ -136,3 +136,24 @@ def test_deterministic_rerun(fd):
     c1, t1 = fd.fdllm_confidence(logits, mask)
     c2, t2 = fd.fdllm_confidence(logits, mask)
     assert torch.equal(c1.view(torch.int32), c2.view(torch.int32)) and torch.equal(t1, t2)
+
+
+def test_fp16_nonfinite_ties_and_extremes(fd, orc):
+    """fp16 rows: a NaN, a +inf maximum, all -inf, -inf entries, the largest finite half
+    (65504), subnormals, and maxima tied within and across 16-byte vectors."""
+    B, L, V = 2, 8, 4096
+    rng = np.random.default_rng(5)
+    x = rng.normal(0.0, 2.0, (B, L, V)).astype(np.float16)
+    x[0, 0, 17] = np.nan
+    x[0, 1, 100] = np.inf
+    x[0, 2, :] = -np.inf
+    x[0, 3, ::3] = -np.inf
+    x[0, 4, 5] = 65504.0
+    x[0, 4, 4000] = 65504.0                    # tied maximum, later index
+    x[0, 5, :] = np.float16(6e-8)              # all subnormal and equal: c = 1/V, x_hat = 0
+    x[1, 0, 8:16] = 30.0                       # a tie inside one vector and the next
+    x[1, 1, 4095] = 40.0                       # maximum in the last element
+    logits = torch.from_numpy(x).cuda()
+    mask = np.ones((B, L), np.uint8)
+    check_confidence(fd, orc, logits, mask)
+    check_select(fd, orc, logits, mask, PROFILE, 0.75)

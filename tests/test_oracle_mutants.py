@@ -40,6 +40,9 @@ MUTANTS = {
     "bf16_widened_wrong": ("(uint32_t)((const uint16_t *)logits)[i] << 16",
                            "(uint32_t)((const uint16_t *)logits)[i] << 15"),
     "nan_not_flagged": ("if (saw_nan || !isfinite(M))", "if (!isfinite(M))"),
+    "fp16_exponent_bias_off": ("ldexp((double)(1024 + frac), e - 25)",
+                               "ldexp((double)(1024 + frac), e - 24)"),
+    "fp16_subnormals_scaled_wrong": ("ldexp((double)frac, -24)", "ldexp((double)frac, -25)"),
     "robust_no_clipping": ("const double c_low = c_hat - eta_i > 0.0 ? c_hat - eta_i : 0.0;",
                            "const double c_low = c_hat - eta_i;"),
     "robust_eta_added": ("const double c_low = c_hat - eta_i > 0.0 ? c_hat - eta_i : 0.0;",
