@@ -143,7 +143,7 @@ fdllm_status fdllm_select_robust(const void *logits, int dtype, int B, int L, in
  * the library holds it until the process exits.  A shape whose scratch need,
  * fdllm_workspace_bytes(B, L, V, dtype), exceeds that size is rejected with
  * FDLLM_ERR_WORKSPACE before anything is enqueued.  8 MiB covers, for example, every shape
- * with V <= 126464 in bf16 or fp32 (up to B * L = 65536 rows), and fp32 V = 2^20 up to
+ * with V <= 126464 in any dtype (up to B * L = 65536 rows), and fp32 V = 2^20 up to
  * B * L = 16383 rows.
  * The call allocates nothing: no cudaMalloc, no cudaFree, no allocating library routine.
  *

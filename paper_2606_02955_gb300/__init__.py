@@ -163,7 +163,7 @@ def _outputs(B, L, device, out_tokens, out_commit, out_n):
 
 def fdllm_select(logits: torch.Tensor, mask: torch.Tensor, param: float, mode=PROFILE,
                  out_tokens=None, out_commit=None, out_n=None, stream=None):
-    """One selection step (fdllm_select).  ``logits`` [B, L, V] bf16/fp32, ``mask`` [B, L]
+    """One selection step (fdllm_select).  ``logits`` [B, L, V] bf16/fp16/fp32, ``mask`` [B, L]
     uint8 (updated in place).  Returns (out_tokens, out_commit, out_n).
 
     Device tensors run asynchronously on ``stream`` (default: current stream).  With host

@@ -13,8 +13,10 @@
 //                            stages, warp 1 issues tcgen05.mma into one of two TMEM
 //                            accumulators, warps 2-5 reduce (or store) the other one; solo,
 //                            W-multicast or CTA-pair (cta_group::2) variants
-//   4. combine_rows_kernel   four warps per row fold its ceil(V / BN) tile partials in a
-//                            fixed order
+//      lmhead_slab_kernel    (at most 32 rows) the operands swapped, W as the M = 128 side:
+//                            each CTA streams one vocabulary slab, one partial per row
+//   4. combine_rows_kernel   four warps per row fold its tile (or slab) partials in a fixed
+//                            order
 //   5. profile_select        steps a2-a5 on the confidences (profile_select.cu)
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -50,6 +52,8 @@ enum Mode {
                      // multicasts it into both CTAs
     kPair = 2,       // 2-CTA pair MMA (tcgen05 cta_group::2, M = 256): each CTA holds its 128
                      // rows and half of the W tile; the even CTA issues the MMAs for both
+    kSlab = 3,       // at most 32 rows: W as the M = 128 operand, each CTA a vocabulary slab
+                     // (lmhead_slab_kernel)
 };
 
 // Vocabulary entries per tile (the MMA's N and the fp32 accumulator's width): 256, or 208,
@@ -75,8 +79,9 @@ struct GemmArgs {
     const int32_t *row_count;  // R, written by compact_rows_kernel
     const int32_t *row_ids;    // [R] global row (b * L + l) of each packed row
     int32_t V;
-    int32_t n_tiles;           // ceil(V / BN)
+    int32_t n_tiles;           // partials per row: ceil(V / BN), or the slab variant's grid
     int32_t k_blocks;          // ceil(H / BK)
+    int32_t n_groups;          // slab variant: ceil(V / 64)
     UnitPartial *partials;     // kReduce: [R][n_tiles]
     float *logits;             // kStore: [B * L][V] fp32, written at masked rows
     uint32_t *status;          // sticky device error bits
@@ -193,6 +198,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     if (warp == 0) {
         if (lane == 0) {
+            // With one row-tile group every W tile is read once: mark it first to evict.
+            const bool w_once = num_mc == 1;
+            const uint64_t pol = make_evict_first_policy();
             int s = 0;
             uint32_t ph = 0;
             uint32_t last_ph[kStages];
@@ -218,7 +226,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                     } else {
                         mbar_arrive_expect_tx(&full[s], kStageBytes);
                         tc::tma_load_2d(sA + s * kABytes, &map_h, kb * BK, m * BM, &full[s]);
-                        if (CL == 1)
+                        if (CL == 1 && w_once)
+                            tc::tma_load_2d_hint(sB + s * kBBytes, &map_w, kb * BK, n * BN,
+                                                 &full[s], pol);
+                        else if (CL == 1)
                             tc::tma_load_2d(sB + s * kBBytes, &map_w, kb * BK, n * BN, &full[s]);
                         else
                             tc::tma_load_2d_multicast(sB + s * kBBytes + rank * (kBBytes / CL),
@@ -406,6 +417,276 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     if (CL > 1)
         tc::cluster_sync();  // no CTA leaves while its peer may still write into it
+}
+
+// ----------------------------------------------------------------------------- slab variant
+// For at most kSlabRows masked rows the operands swap roles: W is the MMA's A operand (M =
+// 128 vocabulary entries, TMEM lane = entry) and the packed rows are its B operand (N = 32,
+// TMEM column = row).  CTA c of P owns the 64-entry groups c, c + P, c + 2P, ... of the G
+// groups (LLaDA's 1976 groups are 13 per SM on 152 SMs, an even split) and streams them as
+// tiles of two groups, groups c + 2jP and c + (2j + 1)P, the last tile possibly one; so the
+// CTAs read W in a window that moves through it, as a grid of one tile per CTA would.
+// The padded row tile costs 4 KB per stage instead of 16 KB, so 10 stages (160 KB of W)
+// are in flight per SM.  Each epilogue thread keeps, for every row, a running maximum, sum
+// of exp relative to it and first index over its own entry of each tile; after the last
+// tile the 128 threads' states are folded per row (a transposing butterfly in each warp,
+// then the four warps in order) into one partial per (row, CTA).
+constexpr int kSlabRows = 32;
+constexpr int kGroup = 64;                               // W rows per TMA box
+constexpr int kSlabABytes = BM * BK * 2;                 // two groups
+constexpr int kSlabBBytes = kSlabRows * BK * 2;
+constexpr int kSlabStages = 10;
+constexpr int kSlabAccs = 4;                             // accumulators of 32 columns
+constexpr uint32_t kSlabTmemCols = 128;
+constexpr size_t kSlabSmemBytes =
+    1024 + (size_t)kSlabStages * (kSlabABytes + kSlabBBytes) + kBarrierBytes;
+static_assert(kSlabSmemBytes <= 227 * 1024, "slab ring");
+static_assert((2 * kSlabStages + 2 * kSlabAccs + 1) * 8 + 8 <= (int)kBarrierBytes, "barriers");
+
+// Two (max, sum relative to it, first index) states of one row -> one.  NaN logits reach
+// only S (they never raise the max), which then stays NaN.
+__device__ __forceinline__ void fold_state(float &M, float &S, uint32_t &I, float M2, float S2,
+                                           uint32_t I2)
+{
+    const float Mn = fmaxf(M, M2);
+    S = rebase(S, M, Mn) + rebase(S2, M2, Mn);
+    const uint32_t i1 = M == Mn ? I : kNoIdx, i2 = M2 == Mn ? I2 : kNoIdx;
+    I = i1 < i2 ? i1 : i2;
+    M = Mn;
+}
+
+template <int EPI>
+__global__ void __launch_bounds__(kThreads, 1)
+    lmhead_slab_kernel(const __grid_constant__ CUtensorMap map_h,
+                       const __grid_constant__ CUtensorMap map_w, const GemmArgs a)
+{
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ float s_M[4][kSlabRows], s_S[4][kSlabRows];
+    __shared__ uint32_t s_I[4][kSlabRows];
+    uint8_t *smem = reinterpret_cast<uint8_t *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *sA = smem;                              // kSlabStages x [128 W rows][128 B]
+    uint8_t *sB = smem + kSlabStages * kSlabABytes;  // kSlabStages x [32 rows][128 B]
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sB + kSlabStages * kSlabBBytes);
+    uint64_t *full = bars;
+    uint64_t *empty = bars + kSlabStages;
+    uint64_t *tfull = bars + 2 * kSlabStages;
+    uint64_t *tempty = tfull + kSlabAccs;
+    uint64_t *done = tempty + kSlabAccs;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 1);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kSlabStages; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int i = 0; i < kSlabAccs; ++i) {
+            mbar_init(&tfull[i], 1);
+            mbar_init(&tempty[i], 4);
+        }
+        mbar_init(done, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+        tc::prefetch_tensormap(&map_h);
+        tc::prefetch_tensormap(&map_w);
+    }
+    if (warp == 1)
+        tc::tmem_alloc(tmem_slot, kSlabTmemCols);
+    tc::fence_before_sync();
+    __syncthreads();
+    tc::fence_after_sync();
+    const uint32_t tmem_base = *tmem_slot;
+
+    pdl_wait();  // the packed rows and their count are complete
+
+    const int R = *a.row_count;  // <= kSlabRows: the host takes this variant only then
+    const int64_t G = a.n_groups, P = gridDim.x, c = blockIdx.x;
+    const int64_t n_g = c < G ? (G - c + P - 1) / P : 0;   // groups of this CTA
+    const int n_t = R > 0 ? (int)((n_g + 1) / 2) : 0;      // tiles of (up to) two groups
+
+    if (warp == 0) {
+        if (lane == 0) {
+            const uint64_t pol = make_evict_first_policy();  // W is read once
+            int s = 0;
+            uint32_t ph = 0;
+            uint32_t last_ph[kSlabStages];
+            bool used[kSlabStages];
+            for (int i = 0; i < kSlabStages; ++i)
+                used[i] = false;
+            bool ok = true;
+            for (int t = 0; ok && t < n_t; ++t) {
+                const int64_t ga = c + 2 * t * P, gb = ga + P;
+                const bool two = 2 * t + 1 < n_g;
+                const uint32_t bytes = (two ? 2u : 1u) * (kGroup * BK * 2) + kSlabBBytes;
+                for (int kb = 0; kb < a.k_blocks; ++kb) {
+                    if (!wait_or_abort(&empty[s], ph ^ 1u, a.status, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(&full[s], bytes);
+                    uint8_t *dst = sA + s * kSlabABytes;
+                    tc::tma_load_2d_hint(dst, &map_w, kb * BK, (int32_t)(ga * kGroup),
+                                         &full[s], pol);
+                    if (two)
+                        tc::tma_load_2d_hint(dst + kGroup * BK * 2, &map_w, kb * BK,
+                                             (int32_t)(gb * kGroup), &full[s], pol);
+                    tc::tma_load_2d(sB + s * kSlabBBytes, &map_h, kb * BK, 0, &full[s]);
+                    used[s] = true;
+                    last_ph[s] = ph;
+                    if (++s == kSlabStages) {
+                        s = 0;
+                        ph ^= 1u;
+                    }
+                }
+            }
+            for (int i = 0; i < kSlabStages; ++i)  // none of this CTA's copies in flight at exit
+                if (used[i])
+                    mbar_wait(&full[i], last_ph[i], a.status, kDrainLimitNs);
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idesc = tc::idesc_bf16_f32(BM, kSlabRows);
+            int s = 0;
+            uint32_t ph = 0;
+            bool ok = true;
+            for (int t = 0; ok && t < n_t; ++t) {
+                const int acc = t % kSlabAccs;
+                const uint32_t aph = (uint32_t)(t / kSlabAccs) & 1u;
+                if (!wait_or_abort(&tempty[acc], aph ^ 1u, a.status, abort_flag))
+                    break;
+                tc::fence_after_sync();
+                const uint32_t d = tmem_base + (uint32_t)(acc * kSlabRows);
+                for (int kb = 0; kb < a.k_blocks; ++kb) {
+                    if (!wait_or_abort(&full[s], ph, a.status, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    tc::fence_after_sync();
+                    // A single-group tile leaves the second half of the A stage stale: those
+                    // 64 TMEM lanes hold meaningless sums that the epilogue skips.
+                    const uint64_t ad = tc::sw128_kmajor_desc(sA + s * kSlabABytes);
+                    const uint64_t bd = tc::sw128_kmajor_desc(sB + s * kSlabBBytes);
+#pragma unroll
+                    for (int k = 0; k < BK / 16; ++k)
+                        tc::mma_bf16(d, ad + 2u * k, bd + 2u * k, idesc, (kb | k) != 0);
+                    tc::commit(&empty[s]);
+                    if (++s == kSlabStages) {
+                        s = 0;
+                        ph ^= 1u;
+                    }
+                }
+                if (ok)
+                    tc::commit(&tfull[acc]);
+            }
+            tc::commit(done);
+            mbar_wait(done, 0, a.status, kDrainLimitNs);
+        }
+        __syncwarp();
+    } else {
+        // Epilogue: warp w reads TMEM lanes [32 (w % 4), +32): thread = one vocabulary entry
+        // of the tile, its 32 columns = the rows.
+        const int q = warp & 3;
+        float M[kSlabRows], S[kSlabRows];
+        uint32_t I[kSlabRows];
+#pragma unroll
+        for (int r = 0; r < kSlabRows; ++r) {
+            M[r] = -__int_as_float(0x7F800000);
+            S[r] = 0.0f;
+            I[r] = kNoIdx;
+        }
+        bool aborted = false;
+        for (int t = 0; t < n_t; ++t) {
+            const int acc = t % kSlabAccs;
+            const uint32_t aph = (uint32_t)(t / kSlabAccs) & 1u;
+            const bool ok = wait_or_abort(&tfull[acc], aph, a.status, abort_flag);
+            if (!__all_sync(0xFFFFFFFFu, ok)) {
+                aborted = true;
+                break;
+            }
+            tc::fence_after_sync();
+            float v[32];
+            tc::tmem_ld_32cols(tmem_base + ((uint32_t)(q * 32) << 16) +
+                                   (uint32_t)(acc * kSlabRows),
+                               v);
+            tc::fence_before_sync();
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(&tempty[acc]);
+            // lanes 0-63 of the tile: group c + 2tP; lanes 64-127: group c + (2t + 1)P
+            const int64_t g = c + (2 * t + (q >> 1)) * P;
+            const int64_t ent = g * kGroup + (q & 1) * 32 + lane;
+            if (2 * t + (q >> 1) >= n_g || ent >= a.V)
+                continue;
+            if (EPI == kStore) {
+#pragma unroll
+                for (int r = 0; r < kSlabRows; ++r)
+                    if (r < R)
+                        a.logits[(int64_t)a.row_ids[r] * a.V + ent] = v[r];
+            } else {
+#pragma unroll
+                for (int r = 0; r < kSlabRows; ++r) {
+                    // exp(x - M) in the form (x - M) * log2e, exact at any magnitude; a
+                    // larger x re-bases the sum; -inf adds nothing; NaN poisons S
+                    const float x = v[r];
+                    const bool up = x > M[r];
+                    const float e = ex2_mufu((up ? M[r] - x : x - M[r]) * kLog2e);
+                    S[r] = up ? fmaf(S[r], e, 1.0f) : (x == -INFINITY ? S[r] : S[r] + e);
+                    I[r] = up ? (uint32_t)ent : I[r];
+                    M[r] = up ? x : M[r];
+                }
+            }
+        }
+        if (EPI == kReduce) {
+            // Transposing butterfly: at offset o each lane keeps the half of its remaining
+            // row slots selected by its lane bit o and folds in the partner's values for them;
+            // slot 0 ends as row `lane`, folded over the warp's 32 entries.
+#pragma unroll
+            for (int o = 16; o >= 1; o >>= 1) {
+                const bool hi = (lane & o) != 0;
+#pragma unroll
+                for (int j = 0; j < o; ++j) {
+                    const float sM = hi ? M[j] : M[j + o], sS = hi ? S[j] : S[j + o];
+                    const uint32_t sI = hi ? I[j] : I[j + o];
+                    float kM = hi ? M[j + o] : M[j], kS = hi ? S[j + o] : S[j];
+                    uint32_t kI = hi ? I[j + o] : I[j];
+                    const float rM = __shfl_xor_sync(0xFFFFFFFFu, sM, o);
+                    const float rS = __shfl_xor_sync(0xFFFFFFFFu, sS, o);
+                    const uint32_t rI = __shfl_xor_sync(0xFFFFFFFFu, sI, o);
+                    fold_state(kM, kS, kI, rM, rS, rI);
+                    M[j] = kM;
+                    S[j] = kS;
+                    I[j] = kI;
+                }
+            }
+            s_M[q][lane] = M[0];
+            s_S[q][lane] = S[0];
+            s_I[q][lane] = I[0];
+            // every epilogue warp arrives exactly once, aborted or not
+            asm volatile("bar.sync 1, 128;" ::: "memory");
+            if (q == 0 && !aborted && !*abort_flag && lane < R) {
+                float fM = s_M[0][lane], fS = s_S[0][lane];
+                uint32_t fI = s_I[0][lane];
+                for (int w = 1; w < 4; ++w)
+                    fold_state(fM, fS, fI, s_M[w][lane], s_S[w][lane], s_I[w][lane]);
+                UnitPartial p;
+                p.M = fS != fS ? __int_as_float(0x7FC00000) : fM;
+                p.S = fS;
+                p.idx = fI;
+                p.pad = 0;
+                a.partials[(int64_t)lane * a.n_tiles + blockIdx.x] = p;
+            }
+        }
+    }
+    if (threadIdx.x == 0)
+        pdl_launch_dependents();  // the row combination may start launching
+    __syncthreads();
+    if (warp == 1) {
+        __syncwarp();
+        tc::fence_after_sync();
+        tc::tmem_dealloc(tmem_base, kSlabTmemCols);
+    }
 }
 
 // One CTA: the packed list of masked rows (ascending) and its length.
@@ -655,11 +936,30 @@ fdllm_status check_lmhead(const void *hidden, const void *w, int B, int L, int H
     return FDLLM_OK;
 }
 
-// The GEMM variant: kPair (cta_group::2) when at least 8 row tiles can share every W tile,
-// kSolo below that (the pair pads to an even number of row tiles, and W streaming from HBM,
-// not shared-memory bandwidth, is the limit there).  FDLLM_LMHEAD_GEMM = solo, multicast or
-// pair forces one.
-int gemm_mode(int64_t rows)
+int sm_count();
+int choose_bn(int64_t rows, int V);
+
+// Rows of W per CTA on the longest-running SM: for the slab variant ceil(G / P) groups of 64;
+// for the tile variants (one row tile) whole waves of vocabulary tiles times their width.
+// Measured on LLaDA-sized heads, the slab variant is faster when each CTA's group count is
+// even and its rows do not exceed the tile variant's; with an odd count every CTA ends on a
+// one-group tile, half as many W bytes in flight, and the tile variant is faster.
+bool slab_preferred(int V)
+{
+    const int64_t sms = sm_count();
+    const int64_t groups = ((int64_t)V + kGroup - 1) / kGroup;
+    const int64_t per_cta = (groups + sms - 1) / sms;
+    const int bn = choose_bn(1, V);
+    const int64_t tile_rows = ((V + bn - 1) / bn + sms - 1) / sms * bn;
+    return per_cta % 2 == 0 && per_cta * kGroup <= tile_rows;
+}
+
+// The GEMM variant: for at most kSlabRows rows the slab variant where slab_preferred; else
+// kPair (cta_group::2) when at least 8 row tiles can share every W tile, kSolo below that
+// (the pair pads to an even number of row tiles, and W streaming from HBM, not
+// shared-memory bandwidth, is the limit there).  FDLLM_LMHEAD_GEMM = solo, multicast, pair
+// or slab forces one (slab only where B * L <= kSlabRows).
+int gemm_mode(int64_t rows, int V)
 {
     if (const char *e = std::getenv("FDLLM_LMHEAD_GEMM")) {
         const std::string v(e);
@@ -669,7 +969,11 @@ int gemm_mode(int64_t rows)
             return kMulticast;
         if (v == "pair")
             return kPair;
+        if (v == "slab" && rows <= kSlabRows)
+            return kSlab;
     }
+    if (rows <= kSlabRows && slab_preferred(V))
+        return kSlab;
     return (rows + BM - 1) / BM >= 8 ? kPair : kSolo;
 }
 
@@ -762,10 +1066,48 @@ cudaError_t launch_gemm_mode(const CUtensorMap &mh, const CUtensorMap &mw, const
                      : launch_gemm_cfg<EPI, MODE, 256>(mh, mw, g, stream);
 }
 
+// The slab variant's grid: one CTA per SM, or one per 64-entry group if there are fewer.
+int slab_grid(int V)
+{
+    const int64_t groups = ((int64_t)V + kGroup - 1) / kGroup;
+    return (int)(groups < sm_count() ? groups : sm_count());
+}
+
+template <int EPI>
+cudaError_t launch_slab(const CUtensorMap &mh, const CUtensorMap &mw, const GemmArgs &g,
+                        cudaStream_t stream)
+{
+    static std::once_flag once[64];
+    int dev = 0;
+    cudaError_t err = cudaGetDevice(&dev);
+    if (err != cudaSuccess)
+        return err;
+    if (dev < 0 || dev >= 64)
+        return cudaErrorInvalidDevice;
+    auto kern = lmhead_slab_kernel<EPI>;
+    std::call_once(once[dev], [&] {
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)kSlabSmemBytes);
+    });
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)g.n_tiles);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kSlabSmemBytes;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = g.pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kern, mh, mw, g);
+}
+
 template <int EPI>
 cudaError_t launch_gemm(const CUtensorMap &mh, const CUtensorMap &mw, const GemmArgs &g,
                         int mode, int bn, cudaStream_t stream)
 {
+    if (mode == kSlab)
+        return launch_slab<EPI>(mh, mw, g, stream);
     switch (mode) {
     case kPair: return launch_gemm_mode<EPI, kPair>(mh, mw, g, bn, stream);
     case kMulticast: return launch_gemm_mode<EPI, kMulticast>(mh, mw, g, bn, stream);
@@ -779,8 +1121,10 @@ fdllm_status run_lmhead(const void *hidden, const void *w, int B, int L, int H, 
                         uint8_t **ws_out, LmLayout *lay_out, bool pdl = true)
 {
     const int64_t rows = (int64_t)B * L;
-    const int bn = choose_bn(rows, V);
-    const int n_tiles = (V + bn - 1) / bn;
+    const int mode = gemm_mode(rows, V);
+    const int bn = mode == kSlab ? kGroup : choose_bn(rows, V);
+    // partials per row: one per vocabulary tile, or one per CTA of the slab variant
+    const int n_tiles = mode == kSlab ? slab_grid(V) : (V + bn - 1) / bn;
     const LmLayout lay = lm_layout(rows, H, n_tiles);
     void *wsv = nullptr;
     fdllm_status st = owned_workspace(lay.total, s, &wsv);
@@ -791,10 +1135,9 @@ fdllm_status run_lmhead(const void *hidden, const void *w, int B, int L, int H, 
     int32_t *row_ids = reinterpret_cast<int32_t *>(ws + lay.row_ids);
     uint8_t *packed = ws + lay.packed;
 
-    const int mode = gemm_mode(rows);
     CUtensorMap mh, mw;
-    if (!make_map(&mh, packed, H, rows, BM) ||
-        !make_map(&mw, w, H, V, mode == kSolo ? bn : bn / 2))
+    if (!make_map(&mh, packed, H, rows, mode == kSlab ? kSlabRows : BM) ||
+        !make_map(&mw, w, H, V, mode == kSolo || mode == kSlab ? bn : bn / 2))
         return FDLLM_ERR_CUDA;
 
     if (launch_pdl(pdl, compact_rows_kernel, 1, 1024, s, mask, (int)rows, row_ids, row_count) !=
@@ -810,6 +1153,7 @@ fdllm_status run_lmhead(const void *hidden, const void *w, int B, int L, int H, 
     g.V = V;
     g.n_tiles = n_tiles;
     g.k_blocks = (H + BK - 1) / BK;
+    g.n_groups = (V + kGroup - 1) / kGroup;
     g.partials = reinterpret_cast<UnitPartial *>(ws + lay.partials);
     g.logits = out_logits;
     g.status = reinterpret_cast<uint32_t *>(ws);

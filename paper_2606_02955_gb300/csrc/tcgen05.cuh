@@ -25,6 +25,18 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, i
         : "memory");
 }
 
+// tma_load_2d with an L2 eviction-priority hint (a policy from make_evict_first_policy): for
+// operands read once, so that they do not displace lines that are read again.
+__device__ __forceinline__ void tma_load_2d_hint(void *dst, const CUtensorMap *map, int32_t x,
+                                                 int32_t y, uint64_t *bar, uint64_t policy)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        ".L2::cache_hint [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(smem_addr(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar)), "l"(policy)
+        : "memory");
+}
+
 // The same load delivered to the same shared-memory offset, and signalled on the mbarrier at
 // the same offset, in every CTA of the cluster whose bit is set in cta_mask.
 __device__ __forceinline__ void tma_load_2d_multicast(void *dst, const CUtensorMap *map,

@@ -227,3 +227,128 @@ def test_hidden_sizes_below_one_stage(fd, orc, H):
     rc, rt, _ = orc.confidence(np.nan_to_num(x.cpu().numpy(), nan=0.0), mask_np)
     assert np.array_equal(tok.cpu().numpy()[mk], rt[mk])
     assert (np.abs(conf.cpu().numpy()[mk] - rc[mk]) / rc[mk]).max() <= CONF_RTOL
+
+
+# ----------------------------------------------------------------------------- slab variant
+SLAB_SHAPES = [
+    # (B, L, H, V) with B * L <= 32: ragged 64-entry groups, CTAs with an odd number of
+    # groups (a single-group last tile), V below one group, LLaDA's head.
+    (1, 32, 256, 5000),
+    (1, 3, 72, 40),
+    (2, 8, 128, 300),
+    (1, 17, 512, 20000),
+    (4, 8, 64, 129),
+    (1, 32, 4096, syn.LLADA_VOCAB),
+]
+
+
+@pytest.fixture
+def slab(monkeypatch):
+    """The swapped-operand variant (W as the M = 128 side, one vocabulary slab per CTA)."""
+    monkeypatch.setenv("FDLLM_LMHEAD_GEMM", "slab")
+
+
+@pytest.mark.parametrize("B,L,H,V", SLAB_SHAPES)
+def test_slab_gemm_within_fp32_accumulation_bound(fd, orc, slab, B, L, H, V):
+    h, w, mask_np = inputs(B, L, H, V, seed=B * 100 + V)
+    x = fd.fdllm_lmhead_logits(h, w, torch.from_numpy(mask_np).cuda())
+    torch.cuda.synchronize()
+    xg = x.cpu().numpy().astype(np.float64)
+    ref, mag = orc.lmhead_logits(bits(h), bits(w), mask=mask_np, with_abs=True,
+                                 nthreads=oracle_threads())
+    mk = mask_np.astype(bool)
+    err = np.abs(xg[mk] - ref[mk])
+    assert (err <= gemm_bound(mag[mk], ref[mk], H)).all(), err.max()
+    assert np.isnan(xg[~mk]).all()
+
+
+@pytest.mark.parametrize("B,L,H,V", SLAB_SHAPES)
+def test_slab_fused_confidence_matches_oracle_on_the_same_accumulators(fd, orc, slab, B, L,
+                                                                       H, V):
+    h, w, mask_np = inputs(B, L, H, V, seed=5 + V)
+    conf, tok = fd.fdllm_lmhead_confidence(h, w, torch.from_numpy(mask_np).cuda())
+    torch.cuda.synchronize()
+    x32 = gpu_logits(fd, h, w, mask_np)
+    rc, rt, bad = orc.confidence(x32, mask_np, nthreads=oracle_threads())
+    mk = mask_np.astype(bool)
+    assert bad == 0
+    g_conf, g_tok = conf.cpu().numpy().astype(np.float64), tok.cpu().numpy()
+    assert np.array_equal(g_tok[mk], rt[mk])
+    rel = np.abs(g_conf[mk] - rc[mk]) / rc[mk]
+    assert rel.max() <= CONF_RTOL, rel.max()
+    assert np.isnan(g_conf[~mk]).all() and (g_tok[~mk] == -1).all()
+
+
+@pytest.mark.parametrize("mode,param", [(oracle.PROFILE, 1.0), (oracle.PROFILE, 0.75),
+                                        (oracle.FACTOR, 1.0), (oracle.THRESHOLD, 0.9)])
+def test_slab_select_matches_oracle(fd, orc, slab, mode, param):
+    B, L, H, V = 1, 32, 512, 30000
+    h, w, mask_np = inputs(B, L, H, V, seed=13, frac=0.9)
+    x32 = gpu_logits(fd, h, w, mask_np)
+    mask = torch.from_numpy(mask_np.copy()).cuda()
+    tok, commit, n = fd.fdllm_lmhead_select(h, w, mask, param, mode)
+    torch.cuda.synchronize()
+    ref = orc.select(x32, mask_np, mode, param, nthreads=oracle_threads())
+    ok = ref["margin"] >= MARGIN
+    assert np.array_equal(n.cpu().numpy()[ok], ref["n"][ok])
+    assert np.array_equal(commit.cpu().numpy()[ok], ref["commit"][ok])
+    assert np.array_equal(mask.cpu().numpy()[ok], ref["mask"][ok])
+    t = tok.cpu().numpy()
+    c = ref["commit"].astype(bool) & ok[:, None]
+    assert np.array_equal(t[c], ref["tokens"][c])
+
+
+@pytest.mark.parametrize("k", [12, 26, 122])
+def test_slab_confidence_at_large_magnitude(fd, orc, slab, k):
+    B, L, H, V = 1, 32, 256, 3000
+    h, w, mask_np = inputs(B, L, H, V, seed=31 + k)
+    h = h * (2.0 ** k)
+    conf, tok = fd.fdllm_lmhead_confidence(h, w, torch.from_numpy(mask_np).cuda())
+    torch.cuda.synchronize()
+    x32 = gpu_logits(fd, h, w, mask_np)
+    mk = mask_np.astype(bool)
+    assert np.isfinite(x32[mk]).all()
+    rc, rt, bad = orc.confidence(x32, mask_np, nthreads=oracle_threads())
+    assert bad == 0
+    g_conf, g_tok = conf.cpu().numpy().astype(np.float64), tok.cpu().numpy()
+    assert np.array_equal(g_tok[mk], rt[mk])
+    assert (np.abs(g_conf[mk] - rc[mk]) / rc[mk]).max() <= CONF_RTOL
+
+
+def test_slab_empty_mask_and_bit_identical_repeats(fd, slab):
+    B, L, H, V = 2, 16, 128, 1000
+    h, w, _ = inputs(B, L, H, V, seed=3)
+    mask = torch.zeros((B, L), dtype=torch.uint8, device="cuda")
+    tok, commit, n = fd.fdllm_lmhead_select(h, w, mask, 1.0)
+    torch.cuda.synchronize()
+    assert (n == 0).all().item() and (commit == 0).all().item()
+    m = torch.ones((B, L), dtype=torch.uint8, device="cuda")
+    c1, t1 = fd.fdllm_lmhead_confidence(h, w, m)
+    c2, t2 = fd.fdllm_lmhead_confidence(h, w, m)
+    torch.cuda.synchronize()
+    assert torch.equal(c1.view(torch.int32), c2.view(torch.int32)) and torch.equal(t1, t2)
+    assert fd.fdllm_device_status() == 0
+
+
+def test_slab_agrees_with_the_tile_variant(fd, orc, monkeypatch):
+    """The same rows through the slab variant and the 128-row tile variant: argmax equal where
+    the top two logits are apart by more than both GEMMs' error, confidences within it."""
+    B, L, H, V = 1, 32, 1024, 50000
+    h, w, mask_np = inputs(B, L, H, V, seed=77)
+    m = torch.from_numpy(mask_np).cuda()
+    out = {}
+    for mode in ("slab", "solo"):
+        monkeypatch.setenv("FDLLM_LMHEAD_GEMM", mode)
+        c, t = fd.fdllm_lmhead_confidence(h, w, m)
+        torch.cuda.synchronize()
+        out[mode] = (c.cpu().numpy().astype(np.float64), t.cpu().numpy())
+    ref, mag = orc.lmhead_logits(bits(h), bits(w), mask=mask_np, with_abs=True,
+                                 nthreads=oracle_threads())
+    mk = mask_np.astype(bool)
+    E = gemm_bound(mag, ref, H).max(axis=-1)
+    srt = np.sort(ref, axis=-1)
+    clear = mk & (srt[..., -1] - srt[..., -2] > 4 * E)
+    assert clear.sum() > 0.5 * mk.sum()
+    assert np.array_equal(out["slab"][1][clear], out["solo"][1][clear])
+    rel = np.abs(out["slab"][0][mk] - out["solo"][0][mk]) / out["solo"][0][mk]
+    assert (rel <= np.expm1(4 * E[mk]) + 2 * CONF_RTOL).all()
