@@ -198,8 +198,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     if (warp == 0) {
         if (lane == 0) {
-            // With one row-tile group every W tile is read once: mark it first to evict.
-            const bool w_once = num_mc == 1;
+            // W tiles are marked first to evict: each is read from HBM once, and the other row
+            // tiles that share it (consecutive work items) read it from L2 right away.
             const uint64_t pol = make_evict_first_policy();
             int s = 0;
             uint32_t ph = 0;
@@ -226,11 +226,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                     } else {
                         mbar_arrive_expect_tx(&full[s], kStageBytes);
                         tc::tma_load_2d(sA + s * kABytes, &map_h, kb * BK, m * BM, &full[s]);
-                        if (CL == 1 && w_once)
+                        if (CL == 1)
                             tc::tma_load_2d_hint(sB + s * kBBytes, &map_w, kb * BK, n * BN,
                                                  &full[s], pol);
-                        else if (CL == 1)
-                            tc::tma_load_2d(sB + s * kBBytes, &map_w, kb * BK, n * BN, &full[s]);
                         else
                             tc::tma_load_2d_multicast(sB + s * kBBytes + rank * (kBBytes / CL),
                                                       &map_w, kb * BK, n * BN + rank * (BN / CL),
