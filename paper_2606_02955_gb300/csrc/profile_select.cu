@@ -128,10 +128,18 @@ __global__ void __launch_bounds__(T) profile_select_kernel(const ProfileSelectAr
     pdl_wait();
     if (threadIdx.x == 0)
         pdl_launch_dependents();  // a following vocab reduction may start its prologue
-    const bool masked = t < L && a.mask[base + t] != 0;
+    // The mask byte, the position's (c, x_hat), its allowance and the status word are loaded
+    // together (one memory round trip on the critical path of a decode step instead of
+    // three); an unmasked position's values are in-bounds leftovers and are discarded.
+    const bool dev_err = a.status != nullptr && *((volatile const uint32_t *)a.status) != 0;
+    const bool in_row = t < L;
+    const bool masked = in_row && a.mask[base + t] != 0;
     float c = 0.0f;
     int32_t tok = -1;
-    if (masked) {
+    const float eta = a.mode == kModeRobust && a.eta_pos != nullptr && in_row
+                          ? a.eta_pos[base + t]
+                          : (float)a.eta;
+    if (in_row) {
         if (a.partials != nullptr) {
             combine_position(a.partials + (base + t) * a.units_per_row, a.units_per_row, c,
                              tok);
@@ -140,21 +148,22 @@ __global__ void __launch_bounds__(T) profile_select_kernel(const ProfileSelectAr
             tok = a.tok[base + t];
         }
     }
+    if (!masked) {
+        c = 0.0f;
+        tok = -1;
+    }
     s_tok[t] = tok;
     if (a.partials != nullptr && a.next_unit != nullptr && blockIdx.x == 0 && t == 0)
         *a.next_unit = 0;  // the vocab reduction before this kernel has finished
     const bool bad = masked && !(c > 0.0f && c <= 1.0f);  // NaN fails both
     // The robust rule ranks and scans lower confidences max{0, c - eta} (App. C).
     float c_rank = c;
-    if (a.mode == kModeRobust && masked && !bad) {
-        const float eta = a.eta_pos != nullptr ? a.eta_pos[base + t] : (float)a.eta;
+    if (a.mode == kModeRobust && masked && !bad)
         c_rank = fmaxf(0.0f, c - eta);
-    }
     uint64_t key = t < L ? make_key(masked, c_rank, t) : kPadKey;
 
     const int m = __syncthreads_count(masked);
     const int any_bad = __syncthreads_or(bad);
-    const bool dev_err = a.status != nullptr && *((volatile const uint32_t *)a.status) != 0;
 
     key = bitonic_sort<T>(key, sk);
 

@@ -652,11 +652,16 @@ __global__ void finalize_kernel(const FinalizeArgs a)
     if (blockIdx.x == 0 && threadIdx.x == 0)
         *a.next_unit = 0;
     const int64_t row = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (row >= a.rows || a.mask[row] == 0)
+    if (row >= a.rows)
         return;
+    // The mask byte and the partials are loaded together; an unmasked row's partials are
+    // in-bounds leftovers and are discarded.
+    const bool masked = a.mask[row] != 0;
     float c;
     int32_t tok;
     combine_position(a.partials + row * a.units_per_row, a.units_per_row, c, tok);
+    if (!masked)
+        return;
     a.out_conf[row] = c;
     a.out_tok[row] = tok;
 }
