@@ -199,10 +199,14 @@ fdllm_status fdllm_gather_masked_rows(const void *src, void *dst, int dtype, int
  *            16-byte aligned.
  *   H        hidden size, a multiple of 8 (16-byte rows); V >= 1, any value.
  * mask, param, mode and the outputs as in fdllm_select (B*L <= FDLLM_MAX_ROWS, L <=
- * FDLLM_MAX_L).  Uses the library-owned workspace (B*L*(2H + 16*ceil(V/256) + 12) bytes
- * and a header), allocated outside the step as for fdllm_select.  Asynchronous on `stream`.
+ * FDLLM_MAX_L).  Uses the library-owned workspace (at most B*L*(2H + 16*ceil(V/208) + 12)
+ * bytes and a header), allocated outside the step as for fdllm_select.  Asynchronous on
+ * `stream`.  The GEMM's tiling (row tiles of 128, CTA pairs, or vocabulary slabs for at most
+ * 32 rows) is chosen from B*L and V; the environment variables FDLLM_LMHEAD_GEMM (solo,
+ * multicast, pair, slab) and FDLLM_LMHEAD_BN (256, 208) force one, for measurements.
  * Results agree with fdllm_select applied to the fp32 logits fdllm_lmhead_logits writes
- * (the same tensor-core accumulation): tokens bit-exact, confidences within 1e-5. */
+ * under the same tiling (the same tensor-core accumulation): tokens bit-exact, confidences
+ * within 1e-5. */
 fdllm_status fdllm_lmhead_select(const void *hidden, const void *w_vocab, int B, int L, int H,
                                  int V, uint8_t *mask, double param, int mode,
                                  int32_t *out_tokens, uint8_t *out_commit, int32_t *out_n,
