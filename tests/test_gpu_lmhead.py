@@ -352,3 +352,22 @@ def test_slab_agrees_with_the_tile_variant(fd, orc, monkeypatch):
     assert np.array_equal(out["slab"][1][clear], out["solo"][1][clear])
     rel = np.abs(out["slab"][0][mk] - out["solo"][0][mk]) / out["solo"][0][mk]
     assert (rel <= np.expm1(4 * E[mk]) + 2 * CONF_RTOL).all()
+
+
+def test_automatic_tiling_small_batch(fd, orc, monkeypatch):
+    """No variant forced: at most 32 rows with V = 19456 (304 groups of 64, two per CTA on
+    152 SMs) is where the host takes the slab variant by itself; any other SM count takes
+    another variant, which must agree with the oracle all the same."""
+    monkeypatch.delenv("FDLLM_LMHEAD_GEMM", raising=False)
+    monkeypatch.delenv("FDLLM_LMHEAD_BN", raising=False)
+    B, L, H, V = 1, 32, 256, 19456
+    h, w, mask_np = inputs(B, L, H, V, seed=8)
+    conf, tok = fd.fdllm_lmhead_confidence(h, w, torch.from_numpy(mask_np).cuda())
+    torch.cuda.synchronize()
+    x32 = gpu_logits(fd, h, w, mask_np)
+    rc, rt, bad = orc.confidence(x32, mask_np, nthreads=oracle_threads())
+    mk = mask_np.astype(bool)
+    assert bad == 0
+    g_conf, g_tok = conf.cpu().numpy().astype(np.float64), tok.cpu().numpy()
+    assert np.array_equal(g_tok[mk], rt[mk])
+    assert (np.abs(g_conf[mk] - rc[mk]) / rc[mk]).max() <= CONF_RTOL
