@@ -25,8 +25,9 @@ constexpr int kMaskWords = kMaxRows / 32;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr uint32_t kNoIdx = 0xFFFFFFFFu;
 
-// Reduction of one unit: max logit M, S = sum of 2^(x*log2e - fl(M*log2e)) over the unit
-// (fl = rounding to fp32) and the row-relative index of the first logit equal to M.
+// Reduction of one unit (or one vocabulary tile or slab of the LM head): max logit M,
+// S = sum of exp(x - M) over it, relative to M exactly (see rebase_scaled), and the
+// row-relative index of the first logit equal to M.
 struct UnitPartial {
     float M;
     float S;

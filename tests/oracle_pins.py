@@ -31,7 +31,7 @@ def bf16_bits(x: np.ndarray) -> np.ndarray:
 
 
 def widen(arr: np.ndarray) -> torch.Tensor:
-    """Exact float64 view of fp32 or bf16-bits logits, via torch's own conversion."""
+    """Exact float64 view of fp32, fp16 or bf16-bits logits, via torch's own conversion."""
     if arr.dtype == np.uint16:
         return torch.from_numpy(arr.view(np.int16).copy()).view(torch.bfloat16).to(torch.float64)
     return torch.from_numpy(arr).to(torch.float64)
