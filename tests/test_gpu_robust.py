@@ -36,7 +36,7 @@ def _check(fd, orc, logits, mask_np, param, eta, eta_pos=None):
 
 @pytest.mark.parametrize("eta", [0.0, 0.01, 0.05, 0.2])
 @pytest.mark.parametrize("name", ["target_b8_l32_bf16", "target_ties_b16_l64_fp32",
-                                  "mixed_mask_b8_l32_bf16"])
+                                  "mixed_mask_b8_l32_bf16", "target_b8_l32_fp16"])
 def test_robust_uniform_eta(fd, orc, name, eta):
     w = syn.WORKLOADS[name]
     logits = syn.make_logits(w, seed=606, device="cuda")
@@ -45,7 +45,8 @@ def test_robust_uniform_eta(fd, orc, name, eta):
         _check(fd, orc, logits, mask_np, f, eta)
 
 
-@pytest.mark.parametrize("name", ["target_b8_l32_bf16", "target_ties_b16_l64_fp32"])
+@pytest.mark.parametrize("name", ["target_b8_l32_bf16", "target_ties_b16_l64_fp32",
+                                  "target_b8_l32_fp16"])
 def test_robust_per_position_eta(fd, orc, name):
     w = syn.WORKLOADS[name]
     logits = syn.make_logits(w, seed=707, device="cuda")

@@ -34,11 +34,12 @@ def _c_entry(path):
     ("mixed_mask_b8_l32_bf16", 0, 0.75),
     ("target_ties_b16_l64_fp32", 1, 1.0),
     ("serving_b64_l32_bf16", 0, 1.0),
+    ("target_b8_l32_fp16", 0, 0.75),
 ])
 def test_static_scratch_matches_select_on_two_calls(fd, name, mode, param):
     lib = _c_entry(fd.library_path())
     w = syn.WORKLOADS[name]
-    dtype = 0 if w.dtype == "bf16" else 1
+    dtype = {"bf16": 0, "fp32": 1, "fp16": 2}[w.dtype]
     assert lib.fdllm_workspace_bytes(w.B, w.L, w.V, dtype) <= STATIC_BYTES
     logits = syn.make_logits(w, seed=77, device="cuda")
     mask_np = syn.make_mask(w, seed=77)
