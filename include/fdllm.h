@@ -167,6 +167,14 @@ fdllm_status fdllm_confidence(const void *logits, int dtype, int B, int L, int V
                               const uint8_t *mask, float *out_conf, int32_t *out_argmax,
                               void *stream);
 
+/* Step a1's vocabulary reduction alone: the per-unit (max, sum of exp, first index)
+ * partials of every masked position, written into the library workspace and not folded
+ * into (c, x_hat); then a one-thread kernel resets the reduction's work counter.  Its use is
+ * timing the reduction kernel by itself (a CUDA graph of these calls); arguments and
+ * errors as for fdllm_confidence. */
+fdllm_status fdllm_vocab_reduce(const void *logits, int dtype, int B, int L, int V,
+                                const uint8_t *mask, void *stream);
+
 /* Steps a2-a5 alone (Alg. 1 sort, scan, select, reveal) on given confidences.
  *   conf    [B, L] fp32 device, read at masked positions; a masked value outside (0, 1]
  *           (NaN included) makes the row FDLLM_ROW_NONFINITE.

@@ -16,14 +16,14 @@ import torch
 from .build import LIB_PATH
 
 __all__ = [
-    "BF16", "FP32", "PROFILE", "FACTOR", "THRESHOLD", "ROW_NONFINITE", "ROW_DEVICE_ERROR",
+    "BF16", "FP32", "FP16", "PROFILE", "FACTOR", "THRESHOLD", "ROW_NONFINITE", "ROW_DEVICE_ERROR",
     "FdllmError", "fdllm_select", "fdllm_select_ws", "fdllm_workspace_bytes",
     "fdllm_confidence", "fdllm_select_from_conf", "fdllm_device_status",
     "fdllm_workspace_status", "fdllm_release_workspace", "fdllm_status_string",
     "fdllm_version", "library_path", "fdllm_select_static", "fdllm_select_robust",
     "fdllm_profile_terms", "fdllm_check_bounded_wait", "fdllm_decode_loop", "FORWARD_FN",
     "fdllm_lmhead_select", "fdllm_lmhead_confidence", "fdllm_lmhead_logits",
-    "fdllm_gather_masked_rows", "fdllm_decode_loop_lmhead",
+    "fdllm_gather_masked_rows", "fdllm_decode_loop_lmhead", "fdllm_vocab_reduce",
 ]
 
 BF16, FP32, FP16 = 0, 1, 2
@@ -70,6 +70,8 @@ def _load():
     lib.fdllm_gather_masked_rows.restype = i
     lib.fdllm_confidence.argtypes = [p, i, i, i, i, p, p, p, p]
     lib.fdllm_confidence.restype = i
+    lib.fdllm_vocab_reduce.argtypes = [p, i, i, i, i, p, p]
+    lib.fdllm_vocab_reduce.restype = i
     lib.fdllm_select_from_conf.argtypes = [p, p, i, i, p, d, i, p, p, p, p]
     lib.fdllm_select_from_conf.restype = i
     lib.fdllm_profile_terms.argtypes = [p, p, i, i, p, p, p, p, p]
@@ -288,6 +290,15 @@ def fdllm_confidence(logits: torch.Tensor, mask: torch.Tensor, out_conf=None, ou
                                _stream(stream))
     _check(st, "fdllm_confidence")
     return out_conf, out_argmax
+
+
+def fdllm_vocab_reduce(logits: torch.Tensor, mask: torch.Tensor, stream=None):
+    """Step a1's vocabulary reduction alone (unit partials in the library workspace, not
+    folded into confidences), for timing the reduction kernel by itself."""
+    B, L, V = logits.shape
+    st = _load().fdllm_vocab_reduce(_dev(logits, "logits"), _dtype_code(logits), B, L, V,
+                                    _dev(mask, "mask", torch.uint8, (B, L)), _stream(stream))
+    _check(st, "fdllm_vocab_reduce")
 
 
 def _lmhead_shapes(hidden: torch.Tensor, w_vocab: torch.Tensor):

@@ -109,6 +109,16 @@ fdllm_status owned_workspace(size_t need, cudaStream_t stream, void **out)
 
 namespace {
 
+// The vocab reduction's work counter back to zero once the reduction has completed (the
+// consumer kernels do this as part of their own work).
+__global__ void reset_queue_kernel(uint32_t *next_unit)
+{
+    pdl_wait();
+    if (threadIdx.x == 0)
+        pdl_launch_dependents();
+    *next_unit = 0;
+}
+
 VocabReduceArgs reduce_args(const void *logits, int dtype, int B, int L, int V,
                             const uint8_t *mask, uint8_t *ws, const Layout &lay)
 {
@@ -357,6 +367,43 @@ fdllm_status fdllm_confidence(const void *logits, int dtype, int B, int L, int V
     if (launch_finalize(fa, s) != cudaSuccess)
         return FDLLM_ERR_CUDA;
     return FDLLM_OK;
+}
+
+fdllm_status fdllm_vocab_reduce(const void *logits, int dtype, int B, int L, int V,
+                                const uint8_t *mask, void *stream)
+{
+    fdllm_status st = check_shape(B, L, V);
+    if (st != FDLLM_OK)
+        return st;
+    if (!mask)
+        return FDLLM_ERR_ARG;
+    st = check_logits(logits, dtype, V);
+    if (st != FDLLM_OK)
+        return st;
+    if (!plan_fits((int64_t)B * L, (int64_t)V * esize_of(dtype)))
+        return FDLLM_ERR_ARG;
+    const Layout lay = layout_for((int64_t)B * L, (int64_t)V * esize_of(dtype));
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    void *ws = nullptr;
+    st = owned_workspace(lay.total, s, &ws);
+    if (st != FDLLM_OK)
+        return st;
+    VocabReduceArgs ra = reduce_args(logits, dtype, B, L, V, mask, static_cast<uint8_t *>(ws),
+                                     lay);
+    if (launch_vocab_reduce(ra, dtype, s) != cudaSuccess)
+        return FDLLM_ERR_CUDA;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(1);
+    cfg.blockDim = dim3(32);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, reset_queue_kernel, ra.next_unit) == cudaSuccess
+               ? FDLLM_OK
+               : FDLLM_ERR_CUDA;
 }
 
 fdllm_status fdllm_select_from_conf(const float *conf, const int32_t *argmax, int B, int L,

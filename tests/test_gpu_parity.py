@@ -157,3 +157,18 @@ def test_fp16_nonfinite_ties_and_extremes(fd, orc):
     mask = np.ones((B, L), np.uint8)
     check_confidence(fd, orc, logits, mask)
     check_select(fd, orc, logits, mask, PROFILE, 0.75)
+
+
+def test_vocab_reduce_alone_leaves_the_library_consistent(fd, orc):
+    """fdllm_vocab_reduce (the reduction kernel by itself, for timing) resets its work counter:
+    selections and confidences after it still match the oracle."""
+    w = W["mixed_mask_b8_l32_bf16"]
+    logits = syn.make_logits(w, seed=808, device="cuda")
+    mask_np = syn.make_mask(w, seed=808)
+    m = torch.from_numpy(mask_np).cuda()
+    for _ in range(3):
+        fd.fdllm_vocab_reduce(logits, m)
+    check_confidence(fd, orc, logits, mask_np)
+    fd.fdllm_vocab_reduce(logits, m)
+    check_select(fd, orc, logits, mask_np, PROFILE, 0.75)
+    assert fd.fdllm_device_status() == 0
