@@ -1,0 +1,72 @@
+"""bench.py's JSON contract on the CPU: the reference arm (the oracle timed on the host cores)
+prints one line with the fields a run is judged by, and under torchrun only rank 0 prints."""
+import json
+import os
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _run(cmd, timeout=600):
+    env = dict(os.environ, MASTER_ADDR="127.0.0.1")
+    p = subprocess.run(cmd, cwd=ROOT, env=env, capture_output=True, text=True, timeout=timeout)
+    assert p.returncode == 0, p.stderr[-2000:]
+    return [l for l in p.stdout.splitlines() if l.startswith("{")]
+
+
+def _check_line(d, n_gpus):
+    sys.path.insert(0, ROOT)
+    import bench
+    assert d["impl"] == "reference"
+    assert d["metric"] == bench.METRIC and d["unit"] == bench.UNIT
+    assert d["value"] > 0 and d["ms_per_step"] > 0 and d["higher_is_better"] is True
+    assert d["n_gpus"] == n_gpus and d["steps"] >= 1 and d["scaling"] == "weak"
+    assert d["data"] == "synthetic" and d["vs_baseline"] is None
+    assert d["config"]["workload"] and "model" not in d["config"]
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["sample"]
+    assert cb["value"] == d["value"] and cb["unit"] == d["unit"]
+    e = d["e2e"]
+    assert e["value"] == d["value"] and e["unit"] == d["unit"]
+    assert e["h2d_bytes_per_step"] == 0 and e["d2h_bytes_per_step"] == 0
+
+
+def test_reference_arm_prints_one_contract_line():
+    lines = _run([sys.executable, "bench.py", "--impl", "reference", "--steps", "1",
+                  "--warmup", "0"])
+    assert len(lines) == 1
+    _check_line(json.loads(lines[0]), 1)
+
+
+def test_reference_arm_under_torchrun_prints_on_rank_0_only():
+    pytest.importorskip("torch.distributed.run")
+    lines = _run([sys.executable, "-m", "torch.distributed.run", "--nnodes=1",
+                  "--nproc-per-node=2", "--master-addr", "127.0.0.1", "--master-port", "29517",
+                  "bench.py", "--impl", "reference", "--gpus", "2", "--steps", "1",
+                  "--warmup", "0"])
+    assert len(lines) == 1
+    _check_line(json.loads(lines[0]), 2)
+
+
+@pytest.mark.gpu
+def test_main_arm_prints_one_contract_line():
+    lines = _run([sys.executable, "bench.py", "--steps", "8", "--warmup", "4"])
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    sys.path.insert(0, ROOT)
+    import bench
+    assert d["metric"] == bench.METRIC and d["unit"] == bench.UNIT and "impl" not in d
+    assert d["value"] > 0 and d["n_gpus"] == 1 and d["steps"] >= 8 and d["warmup"] >= 3
+    r = d["roofline"]
+    assert r["bound"] == "hbm" and r["unit"] == "GB/s" and r["peak"] > 0
+    assert 0 < r["frac"] == pytest.approx(r["achieved"] / r["peak"])
+    assert r["traffic"] is None or r["traffic"] > 0
+    assert d["gpu_launches"] == 2 * d["steps"]
+    assert d["clocks"]["sm_max_mhz"] > 0
+    e = d["e2e"]
+    assert e["value"] > 0 and e["h2d_bytes_per_step"] > 0 and e["d2h_bytes_per_step"] > 0
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] > 0 and cb["sample"]
