@@ -368,9 +368,10 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
         const uint32_t kth = blockIdx.x / upr;
         uint32_t seen = 0;
         int64_t grow = -1;
-        // A bounded scan: with few masked rows among the first kScanRows, the first unit is
-        // issued after the compaction instead (below), not after a long serial scan.
-        constexpr int64_t kScanRows = 2048;
+        // A bounded scan (two memory round trips at most): with few masked rows among the
+        // first kScanRows, the first unit is issued after the compaction instead (below),
+        // which the other warps finish in about the same time.
+        constexpr int64_t kScanRows = 512;
         const int64_t scan_end = a.rows < kScanRows ? a.rows : kScanRows;
         for (int64_t base = 0; base < scan_end && grow < 0; base += 8 * 32) {
             uint32_t ball[8];
