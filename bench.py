@@ -568,7 +568,7 @@ def run_lmhead(args) -> dict:
     wl = syn.WORKLOADS["serving_b64_l32_bf16"]
     if args.lmhead_batch != wl.B:
         wl = dataclasses.replace(wl, B=args.lmhead_batch)
-    B, L, H, V = wl.B, wl.L, syn.LLADA_HIDDEN, syn.LLADA_VOCAB
+    B, L, H, V = wl.B, wl.L, syn.LLADA_HIDDEN, args.lmhead_vocab
     variants = set(args.lmhead_variants.split(","))
     hidden, w, _ = syn.make_lmhead_inputs(B, L, H, V, seed=1234, device=dev)
     mask0_np = syn.make_mask(wl, seed=1234)
@@ -915,6 +915,8 @@ def main(argv=None):
                          "the throughput line")
     ap.add_argument("--lmhead-steps", type=int, default=50)
     ap.add_argument("--lmhead-batch", type=int, default=64)
+    ap.add_argument("--lmhead-vocab", type=int, default=126464,
+                    help="vocabulary size of the LM head (LLaDA-8B: 126464)")
     ap.add_argument("--lmhead-variants", default="fused,gemm,ours,cublas,cublas_masked",
                     help="comma list of: fused, gemm, ours, cublas, cublas_masked")
     args = ap.parse_args(argv)
