@@ -41,10 +41,18 @@ def test_reference_arm_prints_one_contract_line():
     _check_line(json.loads(lines[0]), 1)
 
 
+def _free_port():
+    import socket
+    with socket.socket() as sk:
+        sk.bind(("127.0.0.1", 0))
+        return sk.getsockname()[1]
+
+
 def test_reference_arm_under_torchrun_prints_on_rank_0_only():
     pytest.importorskip("torch.distributed.run")
     lines = _run([sys.executable, "-m", "torch.distributed.run", "--nnodes=1",
-                  "--nproc-per-node=2", "--master-addr", "127.0.0.1", "--master-port", "29517",
+                  "--nproc-per-node=2", "--master-addr", "127.0.0.1",
+                  "--master-port", str(_free_port()),
                   "bench.py", "--impl", "reference", "--gpus", "2", "--steps", "1",
                   "--warmup", "0"])
     assert len(lines) == 1
