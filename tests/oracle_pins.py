@@ -126,6 +126,40 @@ def pin_confidence_closed_forms(o):
     assert math.isclose(conf[0, 0], 1.0 / (3 + 61 * math.exp(-3.5)), rel_tol=1e-12)
 
 
+def pin_extreme_magnitudes(o):
+    """Finite logits of any magnitude: rows of the dtype's most negative finite value give
+    c = 1/V and x_hat = 0; the largest finite value tied twice over very negative logits
+    gives exactly 1/2 at the first of them; a spread far beyond exp's range leaves only the
+    maximum (c = 1); a constant shift by a power of two is exact in fp32 and leaves c
+    unchanged.  (A sum of exp(x) not re-based to the maximum overflows on every case.)"""
+    V = 300
+    f32 = np.finfo(np.float32)
+    for dt, lo, hi in (("fp32", float(f32.min), float(f32.max)),
+                       ("fp16", -65504.0, 65504.0),
+                       ("bf16", -3.3895313892515355e38, 3.3895313892515355e38)):
+        def run(x):
+            a = x.astype(np.float16) if dt == "fp16" else x.astype(np.float32)
+            if dt == "bf16":
+                a = bf16_bits(a)
+            return o.confidence(a[None, None], np.ones((1, 1), np.uint8))
+        conf, tok, bad = run(np.full(V, lo))
+        assert bad == 0 and math.isclose(conf[0, 0], 1.0 / V, rel_tol=1e-12) and tok[0, 0] == 0
+        x = np.full(V, lo / 2)
+        x[[7, 200]] = hi
+        conf, tok, _ = run(x)
+        assert conf[0, 0] == 0.5 and tok[0, 0] == 7
+        x = np.linspace(lo / 4, hi / 4, V)
+        conf, tok, _ = run(x)
+        assert conf[0, 0] == 1.0 and tok[0, 0] == V - 1
+    # a row shifted by 2^20 against the same row shifted back (both shifts exact in fp32)
+    x = np.random.default_rng(3).normal(0.0, 2.0, V).astype(np.float32)
+    xs = x + np.float32(2.0 ** 20)
+    xr = xs - np.float32(2.0 ** 20)
+    c1, t1, _ = o.confidence(xs[None, None], np.ones((1, 1), np.uint8))
+    c2, t2, _ = o.confidence(xr[None, None], np.ones((1, 1), np.uint8))
+    assert math.isclose(c1[0, 0], c2[0, 0], rel_tol=1e-12) and t1[0, 0] == t2[0, 0]
+
+
 def pin_nonfinite(o):
     """NaN anywhere, or a max of +inf / -inf, marks the row invalid; other rows unaffected."""
     x = np.zeros((1, 5, 16), np.float32)
@@ -521,5 +555,5 @@ ALL_PINS = [
     pin_matched_dominance, pin_greedy_equivalence, pin_monotone_prefix, pin_special_cases,
     pin_reveal_and_ties, pin_end_to_end, pin_robust_zero_eta_is_profile,
     pin_robust_calibration_penalty, pin_robust_bruteforce, pin_robust_monotone_and_clipped,
-    pin_bonus_terms, pin_half_widening,
+    pin_bonus_terms, pin_half_widening, pin_extreme_magnitudes,
 ]

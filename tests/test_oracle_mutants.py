@@ -37,6 +37,9 @@ MUTANTS = {
     "confidence_is_sum": ("*c_out = 1.0 / S;", "*c_out = S / (double)V;"),
     "exp_sign_flipped": ("S += exp(logit_at(logits, dtype, base + v) - M);",
                          "S += exp(M - logit_at(logits, dtype, base + v));"),
+    # the same sum in exact arithmetic, but exp(x) overflows for large logits
+    "exp_not_rebased": ("S += exp(logit_at(logits, dtype, base + v) - M);",
+                        "S += exp(logit_at(logits, dtype, base + v)) * exp(-M);"),
     "bf16_widened_wrong": ("(uint32_t)((const uint16_t *)logits)[i] << 16",
                            "(uint32_t)((const uint16_t *)logits)[i] << 15"),
     "nan_not_flagged": ("if (saw_nan || !isfinite(M))", "if (!isfinite(M))"),
