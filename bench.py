@@ -10,7 +10,14 @@ profile rule with f = 1 (delta = 0).
                   [--workload NAME] [--no-graph]
 
 Prints one JSON line (rank 0).  Under torchrun (N > 1) every rank runs its own batch on its
-own GPU (weak scaling, no data exchange); the time is the max over ranks.
+own GPU (weak scaling, no data exchange); the time is the max over ranks.  The roofline
+object times the vocabulary reduction by itself (fdllm_vocab_reduce) against the measured
+copy bandwidth.  Other measurements, each one JSON line:
+  --evolving      masks evolving from step to step until every row has finished
+  --loop          the full-sequence workload (B = 16, L = 1024) selected until no mask remains
+  --lmhead        the LM-head-fused step against cuBLAS logits + selection
+                  (--lmhead-batch, --lmhead-vocab, --lmhead-variants)
+  --decode-loop   the device-resident block loop against a host-driven loop
 
 --impl reference times the fp64 CPU oracle (the reference arm of this benchmark) on the
 host cores, each step a bounded sample of the same workload.
