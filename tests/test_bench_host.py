@@ -1,5 +1,5 @@
 """bench.py's JSON contract on the CPU: the reference arm (the oracle timed on the host cores)
-prints one line with the fields a run is judged by, and under torchrun only rank 0 prints."""
+prints one line with the fields its consumers parse, and under torchrun only rank 0 prints."""
 import json
 import os
 import subprocess
