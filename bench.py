@@ -892,7 +892,7 @@ def main(argv=None):
     ap.add_argument("--eta", type=float, default=0.02,
                     help="calibration allowance of the robust rule (App. C)")
     ap.add_argument("--param", type=float, default=1.0)
-    ap.add_argument("--buffers", type=int, default=4)
+    ap.add_argument("--buffers", type=int, default=8)
     ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--skip-e2e", action="store_true")
     ap.add_argument("--skip-cpu-baseline", action="store_true")
