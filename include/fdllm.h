@@ -287,17 +287,20 @@ fdllm_status fdllm_decode_loop_lmhead(int B, int gen_len, int block_len, int H, 
  *   out_G[b, n-1]     = G_n = max{0, sum_{j<=n} c_(j) - (n-1)} - (1 - c_(n))
  *   out_F[b, n-1]     = F_n = (n+1) c_(n) - n                (factor core)
  *   out_B[b, n-1]     = B_n = sum_{j<n} (c_(j) - c_(n))       (heterogeneity bonus)
+ *   out_feff[b, n-1]  = f_eff(n) = 1 - delta + B_n           (Remark adaptive-factor)
  *   out_order[b, n-1] = the position holding c_(n)
  * Ranks n > m_b get NaN (order -1).  G_n = F_n + B_n wherever the lower bound is positive,
- * and the profile rule with margin delta behaves as the factor rule with the effective
- * factor f_eff(n) = 1 - delta + B_n.
- *   conf  [B, L] fp32 device (e.g. from fdllm_confidence), read at masked positions.
- *   mask  [B, L] uint8 device, nonzero = masked (not modified).
- *   out_G, out_F, out_B  [B, L] fp64 device, each nullable; out_order [B, L] int32, nullable.
+ * so the profile rule with margin delta behaves as the factor rule with the effective
+ * factor f_eff(n).
+ *   conf   [B, L] fp32 device (e.g. from fdllm_confidence), read at masked positions.
+ *   mask   [B, L] uint8 device, nonzero = masked (not modified).
+ *   delta  the profile rule's margin (delta = 1 - param of fdllm_select), finite.
+ *   out_G, out_F, out_B, out_feff  [B, L] fp64 device, each nullable; out_order [B, L]
+ *   int32, nullable.
  * Asynchronous on `stream`; needs no workspace. */
 fdllm_status fdllm_profile_terms(const float *conf, const uint8_t *mask, int B, int L,
-                                 double *out_G, double *out_F, double *out_B,
-                                 int32_t *out_order, void *stream);
+                                 double delta, double *out_G, double *out_F, double *out_B,
+                                 double *out_feff, int32_t *out_order, void *stream);
 
 /* Health check of the library's failure detection: every wait inside the kernels is
  * bounded, and a wait that runs out records a device error and lets the kernel return

@@ -74,7 +74,7 @@ def _load():
     lib.fdllm_vocab_reduce.restype = i
     lib.fdllm_select_from_conf.argtypes = [p, p, i, i, p, d, i, p, p, p, p]
     lib.fdllm_select_from_conf.restype = i
-    lib.fdllm_profile_terms.argtypes = [p, p, i, i, p, p, p, p, p]
+    lib.fdllm_profile_terms.argtypes = [p, p, i, i, d, p, p, p, p, p, p]
     lib.fdllm_profile_terms.restype = i
     lib.fdllm_decode_loop.argtypes = [i, i, i, i, i, d, i, FORWARD_FN, p, p, p, p, i,
                                       ctypes.POINTER(ctypes.c_int), p]
@@ -377,19 +377,22 @@ def fdllm_select_from_conf(conf: torch.Tensor, argmax: torch.Tensor, mask: torch
     return out_tokens, out_commit, out_n
 
 
-def fdllm_profile_terms(conf: torch.Tensor, mask: torch.Tensor, stream=None):
+def fdllm_profile_terms(conf: torch.Tensor, mask: torch.Tensor, delta: float = 0.0,
+                        stream=None):
     """Heterogeneity-bonus diagnostics by rank of each row's sorted masked profile:
-    dict(G, F, B) fp64 [B, L] and order int32 [B, L] (NaN / -1 beyond the masked count)."""
+    dict(G, F, B, f_eff) fp64 [B, L] (f_eff = 1 - delta + B, the effective factor of the
+    profile rule with margin ``delta``) and order int32 [B, L] (NaN / -1 beyond the masked
+    count)."""
     B, L = conf.shape
     dev = conf.device
-    G, F, Bn = (torch.empty((B, L), dtype=torch.float64, device=dev) for _ in range(3))
+    G, F, Bn, Fe = (torch.empty((B, L), dtype=torch.float64, device=dev) for _ in range(4))
     order = torch.empty((B, L), dtype=torch.int32, device=dev)
     st = _load().fdllm_profile_terms(_dev(conf, "conf", torch.float32, (B, L)),
                                      _dev(mask, "mask", torch.uint8, (B, L)), B, L,
-                                     G.data_ptr(), F.data_ptr(), Bn.data_ptr(),
-                                     order.data_ptr(), _stream(stream))
+                                     float(delta), G.data_ptr(), F.data_ptr(), Bn.data_ptr(),
+                                     Fe.data_ptr(), order.data_ptr(), _stream(stream))
     _check(st, "fdllm_profile_terms")
-    return dict(G=G, F=F, B=Bn, order=order)
+    return dict(G=G, F=F, B=Bn, f_eff=Fe, order=order)
 
 
 def fdllm_decode_loop(forward, logits: torch.Tensor, gen_len: int, param: float, mode=PROFILE,

@@ -439,12 +439,12 @@ fdllm_status fdllm_select_from_conf(const float *conf, const int32_t *argmax, in
 }
 
 fdllm_status fdllm_profile_terms(const float *conf, const uint8_t *mask, int B, int L,
-                                 double *out_G, double *out_F, double *out_B,
-                                 int32_t *out_order, void *stream)
+                                 double delta, double *out_G, double *out_F, double *out_B,
+                                 double *out_feff, int32_t *out_order, void *stream)
 {
     if (B < 1 || L < 1 || L > FDLLM_MAX_L || (int64_t)B * L > FDLLM_MAX_ROWS)
         return FDLLM_ERR_ARG;
-    if (!conf || !mask)
+    if (!conf || !mask || !std::isfinite(delta))
         return FDLLM_ERR_ARG;
     ProfileTermsArgs a;
     a.conf = conf;
@@ -454,6 +454,8 @@ fdllm_status fdllm_profile_terms(const float *conf, const uint8_t *mask, int B, 
     a.out_G = out_G;
     a.out_F = out_F;
     a.out_B = out_B;
+    a.delta = delta;
+    a.out_feff = out_feff;
     a.out_order = out_order;
     return launch_profile_terms(a, static_cast<cudaStream_t>(stream)) == cudaSuccess
                ? FDLLM_OK

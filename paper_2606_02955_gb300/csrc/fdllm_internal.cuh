@@ -152,6 +152,8 @@ struct ProfileTermsArgs {
     double *out_G;           // [B, L] by rank, nullable
     double *out_F;           // [B, L] by rank, nullable
     double *out_B;           // [B, L] by rank, nullable
+    double delta;            // the profile rule's margin, for out_feff
+    double *out_feff;        // [B, L] by rank: 1 - delta + B_n, nullable
     int32_t *out_order;      // [B, L] position at each rank, nullable
 };
 

@@ -211,7 +211,8 @@ __global__ void __launch_bounds__(T) profile_select_kernel(const ProfileSelectAr
 // Heterogeneity-bonus diagnostics of one batch row per CTA (Prop. heterogeneity-bonus,
 // Eq. heterogeneity_decomp): the masked confidences sorted as in the selection, an fp64
 // inclusive scan S_n = sum_{j<=n} c_(j), and at rank n: G_n = max{0, S_n - (n-1)} - (1 - c_(n)),
-// F_n = (n+1) c_(n) - n and B_n = S_n - n c_(n) (= sum_{j<n} (c_(j) - c_(n))).
+// F_n = (n+1) c_(n) - n and B_n = S_n - n c_(n) (= sum_{j<n} (c_(j) - c_(n))); and the
+// effective factor f_eff(n) = 1 - delta + B_n of Remark adaptive-factor.
 template <int T>
 __global__ void __launch_bounds__(T) profile_terms_kernel(const ProfileTermsArgs a)
 {
@@ -238,6 +239,8 @@ __global__ void __launch_bounds__(T) profile_terms_kernel(const ProfileTermsArgs
         a.out_F[base + t] = live ? (n + 1.0) * cn - n : nan;
     if (a.out_B != nullptr)
         a.out_B[base + t] = live ? S - n * cn : nan;
+    if (a.out_feff != nullptr)
+        a.out_feff[base + t] = live ? 1.0 - a.delta + (S - n * cn) : nan;
     if (a.out_order != nullptr)
         a.out_order[base + t] = live ? (int32_t)(key & 0xFFFFFFFFu) : -1;
 }

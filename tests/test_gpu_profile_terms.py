@@ -14,10 +14,13 @@ def test_profile_terms_match_oracle(fd, orc, B, L):
     mask_np = (rng.random((B, L)) < 0.8).astype(np.uint8)
     if B > 1:
         mask_np[-1] = 0
-    t = fd.fdllm_profile_terms(torch.from_numpy(c).cuda(), torch.from_numpy(mask_np).cuda())
+    delta = 0.25
+    t = fd.fdllm_profile_terms(torch.from_numpy(c).cuda(), torch.from_numpy(mask_np).cuda(),
+                               delta)
     ref = orc.profile_terms(c.astype(np.float64), mask_np)
+    ref = dict(ref, f_eff=1.0 - delta + ref["B"])  # Remark adaptive-factor, on the oracle's B
     assert np.array_equal(t["order"].cpu().numpy(), ref["order"])
-    for k in ("G", "F", "B"):
+    for k in ("G", "F", "B", "f_eff"):
         g, r = t[k].cpu().numpy(), ref[k]
         assert np.array_equal(np.isnan(g), np.isnan(r))
         ok = ~np.isnan(r)
@@ -37,3 +40,23 @@ def test_profile_terms_decomposition_on_gpu_confidences(fd):
     active = S - (n - 1) > 0
     assert np.all(Bn >= -1e-12)
     assert np.allclose(G[active], F[active] + Bn[active], atol=1e-12)
+
+
+@pytest.mark.parametrize("delta", [0.0, 0.25, 0.5])
+def test_profile_rule_is_the_factor_rule_with_f_eff(fd, delta):
+    """Remark adaptive-factor: where the lower bound is positive, G_n > delta exactly when
+    (n+1)(1 - c_(n)) < f_eff(n) (dyadic confidences: no rounding at the comparisons)."""
+    rng = np.random.default_rng(11)
+    c = (rng.integers(128, 257, (8, 32)) / 256).astype(np.float32)
+    mask = torch.ones((8, 32), dtype=torch.uint8, device="cuda")
+    t = fd.fdllm_profile_terms(torch.from_numpy(c).cuda(), mask, delta)
+    G, Fe = t["G"].cpu().numpy(), t["f_eff"].cpu().numpy()
+    cs = -np.sort(-c.astype(np.float64), axis=1)
+    n = np.arange(1, 33)
+    active = np.cumsum(cs, axis=1) - (n - 1) > 0
+    lhs = G > delta
+    rhs = (n + 1) * (1.0 - cs) < Fe
+    boundary = np.isclose(G, delta, atol=1e-12) | np.isclose((n + 1) * (1.0 - cs), Fe, atol=1e-12)
+    keep = active & ~boundary
+    assert keep.sum() > 50
+    assert np.array_equal(lhs[keep], rhs[keep])
