@@ -177,3 +177,30 @@ def test_gather_masked_rows_rejects(lib):
     assert f(V=1001) == ERR_ALIGN
     assert f(src=A2) == ERR_ALIGN
     assert f(dst=A2) == ERR_ALIGN
+
+
+def test_vocab_reduce_rejects_before_any_device_call(lib):
+    p, i = ctypes.c_void_p, ctypes.c_int
+    lib.fdllm_vocab_reduce.argtypes = [p, i, i, i, i, p, p]
+    A16 = 1 << 20  # a 16-byte aligned (never dereferenced) address
+    assert lib.fdllm_vocab_reduce(A16, 0, 0, 32, 1024, A16, None) == ERR_ARG       # B < 1
+    assert lib.fdllm_vocab_reduce(A16, 0, 2, 2000, 1024, A16, None) == ERR_ARG     # L > max
+    assert lib.fdllm_vocab_reduce(A16, 0, 2, 32, 1024, None, None) == ERR_ARG      # no mask
+    assert lib.fdllm_vocab_reduce(A16, 3, 2, 32, 1024, A16, None) == ERR_ARG       # dtype
+    assert lib.fdllm_vocab_reduce(A16 + 2, 0, 2, 32, 1024, A16, None) == ERR_ALIGN  # base
+    assert lib.fdllm_vocab_reduce(A16, 0, 2, 32, 1001, A16, None) == ERR_ALIGN     # V * 2
+
+
+def test_profile_terms_rejects_before_any_device_call(lib):
+    p, i, d = ctypes.c_void_p, ctypes.c_int, ctypes.c_double
+    lib.fdllm_profile_terms.argtypes = [p, p, i, i, d, p, p, p, p, p, p]
+    A16 = 1 << 20
+    call = lambda B, L, delta, conf=A16, mask=A16: lib.fdllm_profile_terms(
+        conf, mask, B, L, delta, None, None, None, None, None, None)
+    assert call(0, 32, 0.0) == ERR_ARG
+    assert call(2, 0, 0.0) == ERR_ARG
+    assert call(2, 2000, 0.0) == ERR_ARG
+    assert call(2, 32, 0.0, conf=None) == ERR_ARG
+    assert call(2, 32, 0.0, mask=None) == ERR_ARG
+    assert call(2, 32, float("nan")) == ERR_ARG
+    assert call(2, 32, float("inf")) == ERR_ARG
