@@ -169,9 +169,8 @@ fdllm_status fdllm_confidence(const void *logits, int dtype, int B, int L, int V
 
 /* Step a1's vocabulary reduction alone: the per-unit (max, sum of exp, first index)
  * partials of every masked position, written into the library workspace and not folded
- * into (c, x_hat); then a one-thread kernel resets the reduction's work counter.  Its use is
- * timing the reduction kernel by itself (a CUDA graph of these calls); arguments and
- * errors as for fdllm_confidence. */
+ * into (c, x_hat).  One kernel.  Its use is timing the reduction kernel by itself (a CUDA
+ * graph of these calls); arguments and errors as for fdllm_confidence. */
 fdllm_status fdllm_vocab_reduce(const void *logits, int dtype, int B, int L, int V,
                                 const uint8_t *mask, void *stream);
 

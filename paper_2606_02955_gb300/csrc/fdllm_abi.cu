@@ -109,16 +109,6 @@ fdllm_status owned_workspace(size_t need, cudaStream_t stream, void **out)
 
 namespace {
 
-// The vocab reduction's work counter back to zero once the reduction has completed (the
-// consumer kernels do this as part of their own work).
-__global__ void reset_queue_kernel(uint32_t *next_unit)
-{
-    pdl_wait();
-    if (threadIdx.x == 0)
-        pdl_launch_dependents();
-    *next_unit = 0;
-}
-
 VocabReduceArgs reduce_args(const void *logits, int dtype, int B, int L, int V,
                             const uint8_t *mask, uint8_t *ws, const Layout &lay)
 {
@@ -390,20 +380,8 @@ fdllm_status fdllm_vocab_reduce(const void *logits, int dtype, int B, int L, int
         return st;
     VocabReduceArgs ra = reduce_args(logits, dtype, B, L, V, mask, static_cast<uint8_t *>(ws),
                                      lay);
-    if (launch_vocab_reduce(ra, dtype, s) != cudaSuccess)
-        return FDLLM_ERR_CUDA;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(1);
-    cfg.blockDim = dim3(32);
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, reset_queue_kernel, ra.next_unit) == cudaSuccess
-               ? FDLLM_OK
-               : FDLLM_ERR_CUDA;
+    // The reduction leaves its work counter at zero itself (its last fetch resets it).
+    return launch_vocab_reduce(ra, dtype, s) == cudaSuccess ? FDLLM_OK : FDLLM_ERR_CUDA;
 }
 
 fdllm_status fdllm_select_from_conf(const float *conf, const int32_t *argmax, int B, int L,

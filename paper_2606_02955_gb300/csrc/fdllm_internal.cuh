@@ -45,7 +45,7 @@ struct VocabReduceArgs {
     int32_t unit_vecs;
     UnitPartial *partials;   // [rows][units_per_row]; written for masked rows
     uint32_t *next_unit;     // work queue past the first gridDim.x units: zero on entry,
-                             // reset by the consumer kernel
+                             // zero again after the launch's last fetch
     uint32_t *status;        // sticky device error bits
     bool pdl = true;         // launch as a programmatic dependent of the previous kernel
 };

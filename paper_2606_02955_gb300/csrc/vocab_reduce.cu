@@ -23,6 +23,9 @@
 //    (M, S, idx), S re-based to M exactly, for the epilogue warp, which combines the warps in
 //    a fixed order and stores the unit's partial.  The consumer kernel (profile select, or
 //    finalize) folds a position's units in unit order.
+//  * The work counter is put back to zero by the launch's last fetch, so the kernel leaves
+//    the workspace ready for the next launch by itself (the consumer kernels reset it too,
+//    which also covers a launch that gave up a bounded wait).
 #include <cfloat>
 #include <cmath>
 #include <cstdio>
@@ -451,9 +454,22 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
         // ------------------------------------------------------------ producer (one lane)
         if (lane != 0)
             return;
-        if (!first_tried && blockIdx.x < total) {
+        // Every CTA that has a first unit fetches from the queue until it draws a unit past
+        // the last one: the launch makes exactly n_fetch fetches, and the one drawing
+        // n_fetch - 1 is the last, after which the counter is put back to zero for the next
+        // launch.
+        const uint32_t G = gridDim.x;
+        const uint32_t n_fetch = (total > G ? total - G : 0u) + (total < G ? total : G);
+        auto fetched = [&](uint32_t u) {
+            if (u - G == n_fetch - 1u)
+                *a.next_unit = 0;
+            return u;
+        };
+        if (first_tried) {
+            fetched(u_next);
+        } else if (blockIdx.x < total) {
             // the first unit was not within the producer's scan
-            u_next = gridDim.x + atomicAdd(a.next_unit, 1u);
+            u_next = fetched(G + atomicAdd(a.next_unit, 1u));
             first_issued = issue_unit(blockIdx.x,
                                       masked_row(blockIdx.x / upr, sm.bits, sm.pref, nwords));
         }
@@ -461,7 +477,7 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
             // Then the work queue, which hands out units gridDim.x, gridDim.x + 1, ...
             uint32_t u = u_next;
             while (u < total) {
-                const uint32_t un = gridDim.x + atomicAdd(a.next_unit, 1u);
+                const uint32_t un = fetched(G + atomicAdd(a.next_unit, 1u));
                 if (!issue_unit(u, masked_row(u / upr, sm.bits, sm.pref, nwords)))
                     return;
                 u = un;
