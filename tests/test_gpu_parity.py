@@ -172,3 +172,57 @@ def test_vocab_reduce_alone_leaves_the_library_consistent(fd, orc):
     fd.fdllm_vocab_reduce(logits, m)
     check_select(fd, orc, logits, mask_np, PROFILE, 0.75)
     assert fd.fdllm_device_status() == 0
+
+
+def test_concurrent_streams_with_own_workspaces(fd):
+    """Two selection streams, each with its own caller workspace, launched with no ordering
+    between them (the documented way to run concurrent steps): every repetition gives each
+    stream exactly the decisions of the same call run alone."""
+    wa, wb = W["mixed_mask_b8_l32_bf16"], W["target_b8_l32_bf16"]
+    logits = [syn.make_logits(wa, seed=606, device="cuda"),
+              syn.make_logits(wb, seed=607, device="cuda")]
+    masks_np = [syn.make_mask(wa, seed=606), syn.make_mask(wb, seed=607)]
+    shapes = [(wa.B, wa.L), (wb.B, wb.L)]
+    ref = []
+    for x, m_np, (B, L) in zip(logits, masks_np, shapes):
+        m = torch.from_numpy(m_np.copy()).cuda()
+        tok = torch.full((B, L), -1, dtype=torch.int32, device="cuda")
+        r = fd.fdllm_select(x, m, 0.75, PROFILE, tok)
+        torch.cuda.synchronize()
+        ref.append([t.cpu().numpy() for t in r] + [m.cpu().numpy()])
+    ws = [torch.zeros(fd.fdllm_workspace_bytes(w.B, w.L, w.V, fd.BF16), dtype=torch.uint8,
+                      device="cuda") for w in (wa, wb)]
+    streams = [torch.cuda.Stream(), torch.cuda.Stream()]
+    for _ in range(20):
+        masks = [torch.from_numpy(m.copy()).cuda() for m in masks_np]
+        toks = [torch.full(s, -1, dtype=torch.int32, device="cuda") for s in shapes]
+        torch.cuda.synchronize()
+        res = []
+        for i in range(2):
+            with torch.cuda.stream(streams[i]):
+                res.append(fd.fdllm_select_ws(logits[i], masks[i], 0.75, PROFILE, ws[i],
+                                              out_tokens=toks[i], stream=streams[i]))
+        torch.cuda.synchronize()
+        for i in range(2):
+            got = [t.cpu().numpy() for t in res[i]] + [masks[i].cpu().numpy()]
+            for a, b in zip(ref[i], got):
+                assert np.array_equal(a, b)
+    for w in ws:
+        assert fd.fdllm_workspace_status(w) == 0
+
+
+@pytest.mark.parametrize("masked_rows", [0, 1, 5, 76, 77, 152])
+def test_work_counter_reset_by_the_last_fetch(fd, orc, masked_rows):
+    """The reduction puts its work counter back to zero with the launch's last fetch, for
+    any number of units against the grid (none, fewer than the CTAs, about one per CTA,
+    more): a dense selection right after still matches the oracle."""
+    w = W["mixed_mask_b8_l32_bf16"]
+    logits = syn.make_logits(w, seed=909, device="cuda")
+    sparse = np.zeros((w.B, w.L), np.uint8)
+    sparse.reshape(-1)[np.random.default_rng(masked_rows).choice(w.B * w.L, masked_rows,
+                                                                  replace=False)] = 1
+    for _ in range(3):
+        fd.fdllm_vocab_reduce(logits, torch.from_numpy(sparse).cuda())
+        fd.fdllm_select(logits, torch.from_numpy(sparse.copy()).cuda(), 0.75, PROFILE)
+    check_select(fd, orc, logits, np.ones((w.B, w.L), np.uint8), PROFILE, 0.75)
+    assert fd.fdllm_device_status() == 0
