@@ -12,7 +12,9 @@ profile rule with f = 1 (delta = 0).
 Prints one JSON line (rank 0).  Under torchrun (N > 1) every rank runs its own batch on its
 own GPU (weak scaling, no data exchange); the time is the max over ranks.  The roofline
 object times the vocabulary reduction by itself (fdllm_vocab_reduce) against the measured
-copy bandwidth.  Other measurements, each one JSON line:
+copy bandwidth.  At N = 1 the line also carries `evolving`: the serving workload with masks
+evolving from step to step until every row has finished, measured after the timed region
+(--skip-evolving leaves it out).  Other measurements, each one JSON line:
   --evolving      masks evolving from step to step until every row has finished
   --loop          the full-sequence workload (B = 16, L = 1024) selected until no mask remains
   --lmhead        the LM-head-fused step against cuBLAS logits + selection
@@ -896,6 +898,8 @@ def main(argv=None):
     ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--skip-e2e", action="store_true")
     ap.add_argument("--skip-cpu-baseline", action="store_true")
+    ap.add_argument("--skip-evolving", action="store_true",
+                    help="leave out the evolving-mask run that follows the timed region")
     ap.add_argument("--sample-rows", type=int, default=4,
                     help="batch rows per oracle step (reference arm / CPU baseline)")
     ap.add_argument("--cpu-budget-s", type=float, default=10.0)
@@ -958,6 +962,14 @@ def main(argv=None):
         out = run_reference(args, rank, world)
     else:
         out = run_ours(args, rank, world, local_rank)
+        if (out is not None and world == 1 and not args.skip_evolving
+                and args.workload == "serving_b64_l32_bf16"):
+            # the serving workload's second form: masks evolving from step to step until
+            # every row has finished (after the timed region, not part of `value`)
+            ev = run_evolving(args)
+            out["evolving"] = {k: ev[k] for k in ("us_per_step", "selections_per_s",
+                                                  "logits_gbs", "period_steps",
+                                                  "masked_rows_per_step")}
         if out is not None and world == 1 and not args.skip_cpu_baseline:
             out["cpu_baseline"] = run_oracle_timed(args, 1, 1, args.cpu_budget_s)
     if out is not None:

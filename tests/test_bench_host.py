@@ -74,6 +74,8 @@ def test_main_arm_prints_one_contract_line():
     assert r["traffic"] is None or r["traffic"] > 0
     assert d["gpu_launches"] == 2 * d["steps"]
     assert d["clocks"]["sm_max_mhz"] > 0
+    ev = d["evolving"]  # the serving workload with masks evolving until every row finishes
+    assert ev["us_per_step"] > 0 and ev["period_steps"] == len(ev["masked_rows_per_step"])
     e = d["e2e"]
     assert e["value"] > 0 and e["h2d_bytes_per_step"] > 0 and e["d2h_bytes_per_step"] > 0
     cb = d["cpu_baseline"]
