@@ -9,6 +9,7 @@ fallback implementation.
 from __future__ import annotations
 
 import ctypes
+import functools
 import os
 
 import torch
@@ -108,6 +109,26 @@ def library_path() -> str:
     return LIB_PATH
 
 
+
+def _on_device(fn):
+    """Runs an entry point on the device of its CUDA tensor arguments (the library works on
+    the current device: its workspace and launches), and rejects calls whose CUDA tensors
+    live on different devices."""
+    @functools.wraps(fn)
+    def call(*args, **kwargs):
+        cuda = [a for a in (*args, *kwargs.values()) if isinstance(a, torch.Tensor) and a.is_cuda]
+        if not cuda:
+            return fn(*args, **kwargs)
+        dev = cuda[0].device
+        for t in cuda[1:]:
+            if t.device != dev:
+                raise ValueError("the CUDA tensors of one call must share a device (%s, %s)"
+                                 % (dev, t.device))
+        with torch.cuda.device(dev):
+            return fn(*args, **kwargs)
+    return call
+
+
 def fdllm_status_string(status: int) -> str:
     return _load().fdllm_status_string(int(status)).decode()
 
@@ -163,6 +184,7 @@ def _outputs(B, L, device, out_tokens, out_commit, out_n):
     return out_tokens, out_commit, out_n
 
 
+@_on_device
 def fdllm_select(logits: torch.Tensor, mask: torch.Tensor, param: float, mode=PROFILE,
                  out_tokens=None, out_commit=None, out_n=None, stream=None):
     """One selection step (fdllm_select).  ``logits`` [B, L, V] bf16/fp16/fp32, ``mask`` [B, L]
@@ -215,6 +237,7 @@ def _select_from_host(logits, mask, param, mode, out_tokens, out_commit, out_n):
     return h_tok, h_commit, h_n
 
 
+@_on_device
 def fdllm_select_robust(logits: torch.Tensor, mask: torch.Tensor, param: float, eta: float = 0.0,
                         eta_per_position=None, out_tokens=None, out_commit=None, out_n=None,
                         stream=None):
@@ -235,6 +258,7 @@ def fdllm_select_robust(logits: torch.Tensor, mask: torch.Tensor, param: float, 
     return out_tokens, out_commit, out_n
 
 
+@_on_device
 def fdllm_select_static(logits: torch.Tensor, mask: torch.Tensor, param: float, mode=PROFILE,
                         out_tokens=None, out_commit=None, out_n=None, stream=None):
     """fdllm_select using the library's fixed device scratch array instead of an allocated
@@ -256,6 +280,7 @@ def fdllm_workspace_bytes(B: int, L: int, V: int, dtype=BF16) -> int:
     return int(_load().fdllm_workspace_bytes(B, L, V, dtype))
 
 
+@_on_device
 def fdllm_select_ws(logits: torch.Tensor, mask: torch.Tensor, param: float, mode,
                     workspace: torch.Tensor, out_tokens=None, out_commit=None, out_n=None,
                     stream=None):
@@ -274,6 +299,7 @@ def fdllm_select_ws(logits: torch.Tensor, mask: torch.Tensor, param: float, mode
     return out_tokens, out_commit, out_n
 
 
+@_on_device
 def fdllm_confidence(logits: torch.Tensor, mask: torch.Tensor, out_conf=None, out_argmax=None,
                      stream=None):
     """Step a1 alone: (conf fp32 [B, L], argmax int32 [B, L]) written at masked positions
@@ -292,6 +318,7 @@ def fdllm_confidence(logits: torch.Tensor, mask: torch.Tensor, out_conf=None, ou
     return out_conf, out_argmax
 
 
+@_on_device
 def fdllm_vocab_reduce(logits: torch.Tensor, mask: torch.Tensor, stream=None):
     """Step a1's vocabulary reduction alone (unit partials in the library workspace, not
     folded into confidences), for timing the reduction kernel by itself."""
@@ -311,6 +338,7 @@ def _lmhead_shapes(hidden: torch.Tensor, w_vocab: torch.Tensor):
     return B, L, H, V, hp, wp
 
 
+@_on_device
 def fdllm_lmhead_select(hidden: torch.Tensor, w_vocab: torch.Tensor, mask: torch.Tensor,
                         param: float, mode=PROFILE, out_tokens=None, out_commit=None, out_n=None,
                         stream=None):
@@ -328,6 +356,7 @@ def fdllm_lmhead_select(hidden: torch.Tensor, w_vocab: torch.Tensor, mask: torch
     return out_tokens, out_commit, out_n
 
 
+@_on_device
 def fdllm_lmhead_confidence(hidden: torch.Tensor, w_vocab: torch.Tensor, mask: torch.Tensor,
                             out_conf=None, out_argmax=None, stream=None):
     """Step a1 on the LM head: (conf fp32 [B, L], argmax int32 [B, L]) at masked positions."""
@@ -345,6 +374,7 @@ def fdllm_lmhead_confidence(hidden: torch.Tensor, w_vocab: torch.Tensor, mask: t
     return out_conf, out_argmax
 
 
+@_on_device
 def fdllm_lmhead_logits(hidden: torch.Tensor, w_vocab: torch.Tensor, mask: torch.Tensor,
                         out_logits=None, stream=None):
     """The LM-head GEMM's fp32 logits [B, L, V] at masked rows (other rows untouched; a
@@ -360,6 +390,7 @@ def fdllm_lmhead_logits(hidden: torch.Tensor, w_vocab: torch.Tensor, mask: torch
     return out_logits
 
 
+@_on_device
 def fdllm_select_from_conf(conf: torch.Tensor, argmax: torch.Tensor, mask: torch.Tensor,
                            param: float, mode=PROFILE, out_tokens=None, out_commit=None,
                            out_n=None, stream=None):
@@ -377,6 +408,7 @@ def fdllm_select_from_conf(conf: torch.Tensor, argmax: torch.Tensor, mask: torch
     return out_tokens, out_commit, out_n
 
 
+@_on_device
 def fdllm_profile_terms(conf: torch.Tensor, mask: torch.Tensor, delta: float = 0.0,
                         stream=None):
     """Heterogeneity-bonus diagnostics by rank of each row's sorted masked profile:
@@ -395,6 +427,7 @@ def fdllm_profile_terms(conf: torch.Tensor, mask: torch.Tensor, delta: float = 0
     return dict(G=G, F=F, B=Bn, f_eff=Fe, order=order)
 
 
+@_on_device
 def fdllm_decode_loop(forward, logits: torch.Tensor, gen_len: int, param: float, mode=PROFILE,
                       max_steps: int | None = None, stream=None):
     """Algorithm 1's outer loop on the GPU (fdllm_decode_loop).  ``logits`` is the
@@ -429,6 +462,7 @@ def fdllm_decode_loop(forward, logits: torch.Tensor, gen_len: int, param: float,
     return seq, nfe, steps.value
 
 
+@_on_device
 def fdllm_gather_masked_rows(src: torch.Tensor, mask: torch.Tensor, dst=None, stream=None):
     """Copy the masked positions' rows of ``src`` [B, L, V] (a CUDA tensor or a pinned host
     tensor, read by the GPU directly) into ``dst`` (a CUDA tensor of the same shape and
@@ -448,6 +482,7 @@ def fdllm_gather_masked_rows(src: torch.Tensor, mask: torch.Tensor, dst=None, st
     return dst
 
 
+@_on_device
 def fdllm_decode_loop_lmhead(forward, hidden: torch.Tensor, w_vocab: torch.Tensor, gen_len: int,
                              param: float, mode=PROFILE, max_steps: int | None = None,
                              stream=None):
@@ -495,6 +530,7 @@ def fdllm_device_status(stream=None) -> int:
     return _load().fdllm_device_status(_stream(stream))
 
 
+@_on_device
 def fdllm_workspace_status(workspace: torch.Tensor, stream=None) -> int:
     return _load().fdllm_workspace_status(_dev(workspace, "workspace", torch.uint8), _stream(stream))
 

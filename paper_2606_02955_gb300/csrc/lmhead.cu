@@ -977,15 +977,16 @@ int gemm_mode(int64_t rows, int V)
 
 int sm_count()
 {
-    static int cache[64] = {0};
+    static std::once_flag once[64];
+    static int cache[64];
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64)
         return 152;
-    if (cache[dev] == 0) {
+    std::call_once(once[dev], [&] {
         int n = 0;
         cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
         cache[dev] = n > 0 ? n : 152;
-    }
+    });
     return cache[dev];
 }
 

@@ -30,6 +30,7 @@
 #include <cmath>
 #include <cstdio>
 #include <cstdlib>
+#include <mutex>
 #include <type_traits>
 
 #include "fdllm_internal.cuh"
@@ -686,8 +687,11 @@ __global__ void finalize_kernel(const FinalizeArgs a)
 template <int KIND, int NW, int STAGES, int CHUNK, bool EVICT>
 cudaError_t launch_variant(const VocabReduceArgs &a, cudaStream_t stream)
 {
-    static int attr_done[64] = {0};
-    static int grid_cache[64] = {0};
+    // Per device, once (host threads may make their first calls concurrently): the shared
+    // memory attribute and the grid of every CTA resident at once.
+    static std::once_flag once[64];
+    static cudaError_t setup_err[64];
+    static int grid_cache[64];
     int dev = 0;
     cudaError_t err = cudaGetDevice(&dev);
     if (err != cudaSuccess)
@@ -697,17 +701,18 @@ cudaError_t launch_variant(const VocabReduceArgs &a, cudaStream_t stream)
     constexpr size_t smem = smem_bytes<NW, STAGES, CHUNK>();
     static_assert(smem <= 227 * 1024, "ring does not fit in shared memory");
     auto *kern = vocab_reduce_kernel<KIND, NW, STAGES, CHUNK, EVICT>;
-    if (!attr_done[dev]) {
-        err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (err != cudaSuccess)
-            return err;
+    std::call_once(once[dev], [&] {
+        setup_err[dev] =
+            cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         int sms = 0, per_sm = 0;
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
         cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, (NW + 2) * 32, smem);
-        int g = sms * (per_sm > 0 ? per_sm : 1);
+        (void)cudaGetLastError();
+        const int g = (sms > 0 ? sms : 1) * (per_sm > 0 ? per_sm : 1);
         grid_cache[dev] = g < kMaxGrid ? g : kMaxGrid;
-        attr_done[dev] = 1;
-    }
+    });
+    if (setup_err[dev] != cudaSuccess)
+        return setup_err[dev];
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)grid_cache[dev]);
     cfg.blockDim = dim3((NW + 2) * 32);
