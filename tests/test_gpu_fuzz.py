@@ -11,7 +11,7 @@ import numpy as np
 import pytest
 
 import fdllm_synth as syn
-from gpu_util import check_confidence, check_select
+from gpu_util import CONF_RTOL, check_confidence, check_select
 
 PROFILE, FACTOR, THRESHOLD = 0, 1, 2
 
@@ -60,3 +60,48 @@ def test_draws_cover_the_space():
     assert {c[0].peak for c in cases} == {"none", "uniform", "zipf", "target"}
     assert {c[2] for c in cases} == {PROFILE, FACTOR, THRESHOLD}
     assert any((c[1].sum(axis=1) == 0).any() for c in cases)
+
+
+def draw_lmhead_case(seed):
+    rng = np.random.default_rng(30_000 + seed)
+    B = int(rng.integers(1, 5))
+    L = int(rng.integers(1, 65))
+    H = int(rng.choice([8, 40, 72, 256, 520, 1024]))
+    V = int(rng.choice([40, 300, 1000, 2050, 5000, 20000]))
+    variant = ("auto", "solo", "multicast", "pair", "slab")[rng.integers(5)]
+    bn = int(rng.choice([256, 208]))
+    frac = float(rng.uniform(0.2, 1.0))
+    return B, L, H, V, variant, bn, frac
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("seed", range(16))
+def test_random_lmhead_case_matches_oracle(fd, orc, monkeypatch, seed):
+    """The LM-head path on drawn shapes (H not a multiple of the K stage, V ragged against
+    every tile), GEMM variants and tile widths: the stored logits within the fp32
+    accumulation bound of the exact ones, and the fused confidences and tokens against the
+    oracle on those same accumulators."""
+    import torch
+    from test_gpu_lmhead import bits, gemm_bound, gpu_logits, inputs
+
+    B, L, H, V, variant, bn, frac = draw_lmhead_case(seed)
+    if variant == "auto":
+        monkeypatch.delenv("FDLLM_LMHEAD_GEMM", raising=False)
+    else:
+        monkeypatch.setenv("FDLLM_LMHEAD_GEMM", variant)  # slab only where B * L <= 32
+    monkeypatch.setenv("FDLLM_LMHEAD_BN", str(bn))
+    h, w, mask_np = inputs(B, L, H, V, seed=40_000 + seed, frac=frac)
+    conf, tok = fd.fdllm_lmhead_confidence(h, w, torch.from_numpy(mask_np).cuda())
+    torch.cuda.synchronize()
+    x32 = gpu_logits(fd, h, w, mask_np)
+    mk = mask_np.astype(bool)
+    rc, rt, bad = orc.confidence(x32, mask_np)
+    assert bad == 0
+    g_conf, g_tok = conf.cpu().numpy().astype(np.float64), tok.cpu().numpy()
+    assert np.array_equal(g_tok[mk], rt[mk])
+    if mk.any():
+        assert (np.abs(g_conf[mk] - rc[mk]) / rc[mk]).max() <= CONF_RTOL
+    ref, mag = orc.lmhead_logits(bits(h), bits(w), mask=mask_np, with_abs=True)
+    err = np.abs(x32[mk].astype(np.float64) - ref[mk])
+    assert (err <= gemm_bound(mag[mk], ref[mk], H)).all()
+    assert fd.fdllm_device_status() == 0
