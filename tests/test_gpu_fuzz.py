@@ -105,3 +105,20 @@ def test_random_lmhead_case_matches_oracle(fd, orc, monkeypatch, seed):
     err = np.abs(x32[mk].astype(np.float64) - ref[mk])
     assert (err <= gemm_bound(mag[mk], ref[mk], H)).all()
     assert fd.fdllm_device_status() == 0
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("seed", range(12))
+def test_random_robust_case_matches_oracle(fd, orc, seed):
+    """The calibration-robust rule on the drawn cases, with a drawn uniform allowance or a
+    drawn per-position one (App. C), against the oracle's robust selector."""
+    from test_gpu_robust import _check
+
+    w, mask, _, _ = draw_case(100 + seed)
+    rng = np.random.default_rng(50_000 + seed)
+    param = float(rng.choice([0.5, 0.75, 1.0]))
+    logits = syn.make_logits(w, seed=100 + seed, device="cuda")
+    if rng.random() < 0.5:
+        _check(fd, orc, logits, mask, param, float(rng.uniform(0.0, 0.3)))
+    else:
+        _check(fd, orc, logits, mask, param, 0.0, rng.uniform(0.0, 0.3, (w.B, w.L)))
