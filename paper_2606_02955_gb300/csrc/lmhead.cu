@@ -935,7 +935,7 @@ fdllm_status check_lmhead(const void *hidden, const void *w, int B, int L, int H
 }
 
 int sm_count();
-int choose_bn(int64_t rows, int V);
+int choose_bn(int64_t rows, int V, bool pair);
 
 // Rows of W per CTA on the longest-running SM: for the slab variant ceil(G / P) groups of 64;
 // for the tile variants (one row tile) whole waves of vocabulary tiles times their width.
@@ -947,7 +947,7 @@ bool slab_preferred(int V)
     const int64_t sms = sm_count();
     const int64_t groups = ((int64_t)V + kGroup - 1) / kGroup;
     const int64_t per_cta = (groups + sms - 1) / sms;
-    const int bn = choose_bn(1, V);
+    const int bn = choose_bn(1, V, false);
     const int64_t tile_rows = ((V + bn - 1) / bn + sms - 1) / sms * bn;
     return per_cta % 2 == 0 && per_cta * kGroup <= tile_rows;
 }
@@ -991,9 +991,11 @@ int sm_count()
 }
 
 // The vocabulary tile width with the least estimated time: whole waves of tiles over the
-// SMs (row tiles estimated from B * L, the most the mask can hold) times the tile width;
-// ties go to the wider tile.  FDLLM_LMHEAD_BN = 256 or 208 forces one.
-int choose_bn(int64_t rows, int V)
+// SMs (row tiles estimated from B * L, the most the mask can hold) times the tile width.
+// Ties go to 208 for one CTA per tile (measured 1.3-1.4 % faster at 4 estimated row tiles,
+// B = 14 and 16 of 32 positions) and to 256 for the CTA pair (208 is slower there at every
+// size).  FDLLM_LMHEAD_BN = 256 or 208 forces one.
+int choose_bn(int64_t rows, int V, bool pair)
 {
     if (const char *e = std::getenv("FDLLM_LMHEAD_BN")) {
         const int f = std::atoi(e);
@@ -1001,9 +1003,10 @@ int choose_bn(int64_t rows, int V)
             return f;
     }
     const int64_t m_tiles = (rows + BM - 1) / BM, sms = sm_count();
-    int best = 256;
+    const int order[2] = {pair ? 256 : 208, pair ? 208 : 256};  // the first wins ties
+    int best = order[0];
     int64_t best_cost = -1;
-    for (int bn : {256, 208}) {
+    for (int bn : order) {
         const int64_t tiles = (V + bn - 1) / bn * m_tiles;
         const int64_t cost = (tiles + sms - 1) / sms * bn;
         if (best_cost < 0 || cost < best_cost) {
@@ -1121,7 +1124,7 @@ fdllm_status run_lmhead(const void *hidden, const void *w, int B, int L, int H, 
 {
     const int64_t rows = (int64_t)B * L;
     const int mode = gemm_mode(rows, V);
-    const int bn = mode == kSlab ? kGroup : choose_bn(rows, V);
+    const int bn = mode == kSlab ? kGroup : choose_bn(rows, V, mode == kPair);
     // partials per row: one per vocabulary tile, or one per CTA of the slab variant
     const int n_tiles = mode == kSlab ? slab_grid(V) : (V + bn - 1) / bn;
     const LmLayout lay = lm_layout(rows, H, n_tiles);
