@@ -210,7 +210,7 @@ fdllm_status fdllm_gather_masked_rows(const void *src, void *dst, int dtype, int
  * bytes and a header), allocated outside the step as for fdllm_select.  Asynchronous on
  * `stream`.  The GEMM's tiling (row tiles of 128, CTA pairs, or vocabulary slabs for at most
  * 32 rows) is chosen from B*L and V; the environment variables FDLLM_LMHEAD_GEMM (solo,
- * multicast, pair, slab) and FDLLM_LMHEAD_BN (256, 208) force one, for measurements.
+ * pair, slab) and FDLLM_LMHEAD_BN (256, 208) force one, for measurements.
  * Results agree with fdllm_select applied to the fp32 logits fdllm_lmhead_logits writes
  * under the same tiling (the same tensor-core accumulation): tokens bit-exact, confidences
  * within 1e-5. */

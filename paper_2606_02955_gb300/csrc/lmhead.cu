@@ -11,8 +11,8 @@
 //   2. gather_rows_kernel    the masked rows' hidden states, packed [R, H] (TMA-friendly)
 //   3. lmhead_gemm_kernel    persistent tcgen05 GEMM: warp 0 issues TMA loads into a ring of
 //                            stages, warp 1 issues tcgen05.mma into one of two TMEM
-//                            accumulators, warps 2-5 reduce (or store) the other one; solo,
-//                            W-multicast or CTA-pair (cta_group::2) variants
+//                            accumulators, warps 2-5 reduce (or store) the other one; solo
+//                            or CTA-pair (cta_group::2) variants
 //      lmhead_slab_kernel    (at most 32 rows) the operands swapped, W as the M = 128 side:
 //                            each CTA streams one vocabulary slab, one partial per row
 //   4. combine_rows_kernel   four warps per row fold its tile (or slab) partials in a fixed
@@ -48,8 +48,6 @@ constexpr uint64_t kDrainLimitNs = 100000000ull;  // waits for own copies after 
 // How the CTAs of a cluster share a W tile.
 enum Mode {
     kSolo = 0,       // one CTA per work item; it loads the whole W tile
-    kMulticast = 1,  // 2-CTA cluster, two row tiles: each CTA loads half of the W tile and
-                     // multicasts it into both CTAs
     kPair = 2,       // 2-CTA pair MMA (tcgen05 cta_group::2, M = 256): each CTA holds its 128
                      // rows and half of the W tile; the even CTA issues the MMAs for both
     kSlab = 3,       // at most 32 rows: W as the M = 128 operand, each CTA a vocabulary slab
@@ -110,11 +108,9 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity, ui
     }
 }
 
-// MODE kSolo: every CTA loads its own W tile.  kMulticast: the two CTAs of a cluster take
-// row tiles 2j and 2j + 1 of the same vocabulary tile; each loads half of the W tile and
-// multicasts it into both CTAs' shared memory (half the L2 -> SM traffic for W), and each
-// MMA releases a stage in both CTAs, since either producer overwrites it in both.  kPair:
-// the same two row tiles form one M = 256 MMA issued by the even CTA (tcgen05 cta_group::2):
+// MODE kSolo: every CTA loads its own W tile.  kPair: the two CTAs of a cluster take row
+// tiles 2j and 2j + 1 of the same vocabulary tile, which form one M = 256 MMA issued by the
+// even CTA (tcgen05 cta_group::2):
 // each CTA loads its 128 rows and half of the W tile into its own shared memory and
 // signals the even CTA's stage barrier, so each CTA's shared memory supplies half the
 // operand bytes per MMA; the accumulators live in both CTAs' tensor memory.
@@ -146,7 +142,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             mbar_init(&full[s], 1);
-            mbar_init(&empty[s], MODE == kMulticast ? 2 : 1);  // one release per MMA issuer
+            mbar_init(&empty[s], 1);  // released by the MMA issuer's commit
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&tfull[i], 1);
@@ -167,7 +163,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::fence_before_sync();
     __syncthreads();
     if (CL > 1)
-        tc::cluster_sync();  // the peer's barriers are initialised before any multicast
+        tc::cluster_sync();  // the peer's barriers are initialised before any remote signal
     tc::fence_after_sync();
     const uint32_t tmem_base = *tmem_slot;
 
@@ -226,13 +222,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     } else {
                         mbar_arrive_expect_tx(&full[s], kStageBytes);
                         tc::tma_load_2d(sA + s * kABytes, &map_h, kb * BK, m * BM, &full[s]);
-                        if (CL == 1)
-                            tc::tma_load_2d_hint(sB + s * kBBytes, &map_w, kb * BK, n * BN,
-                                                 &full[s], pol);
-                        else
-                            tc::tma_load_2d_multicast(sB + s * kBBytes + rank * (kBBytes / CL),
-                                                      &map_w, kb * BK, n * BN + rank * (BN / CL),
-                                                      &full[s], (uint16_t)((1u << CL) - 1u));
+                        tc::tma_load_2d_hint(sB + s * kBBytes, &map_w, kb * BK, n * BN,
+                                             &full[s], pol);
                     }
                     used[s] = true;
                     last_ph[s] = ph;
@@ -279,15 +270,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                         else
                             tc::mma_bf16(d, ad + 2u * k, bd + 2u * k, idesc, (kb | k) != 0);
                     }
-                    // The stage is free once these MMAs have read it (in every CTA of the
-                    // cluster: either producer overwrites it in both, or each refills its own
-                    // half of the pair's operands).
+                    // The stage is free once these MMAs have read it (in a pair, in both
+                    // CTAs: each refills its own half of the pair's operands).
                     if constexpr (PAIR)
                         tc::commit_pair_multicast(&empty[s]);
-                    else if (CL == 1)
-                        tc::commit(&empty[s]);
                     else
-                        tc::commit_multicast(&empty[s], (uint16_t)((1u << CL) - 1u));
+                        tc::commit(&empty[s]);
                     if (++s == kStages) {
                         s = 0;
                         ph ^= 1u;
@@ -955,16 +943,14 @@ bool slab_preferred(int V)
 // The GEMM variant: for at most kSlabRows rows the slab variant where slab_preferred; else
 // kPair (cta_group::2) when at least 8 row tiles can share every W tile, kSolo below that
 // (the pair pads to an even number of row tiles, and W streaming from HBM, not
-// shared-memory bandwidth, is the limit there).  FDLLM_LMHEAD_GEMM = solo, multicast, pair
-// or slab forces one (slab only where B * L <= kSlabRows).
+// shared-memory bandwidth, is the limit there).  FDLLM_LMHEAD_GEMM = solo, pair or slab
+// forces one (slab only where B * L <= kSlabRows).
 int gemm_mode(int64_t rows, int V)
 {
     if (const char *e = std::getenv("FDLLM_LMHEAD_GEMM")) {
         const std::string v(e);
         if (v == "solo")
             return kSolo;
-        if (v == "multicast")
-            return kMulticast;
         if (v == "pair")
             return kPair;
         if (v == "slab" && rows <= kSlabRows)
@@ -1112,7 +1098,6 @@ cudaError_t launch_gemm(const CUtensorMap &mh, const CUtensorMap &mw, const Gemm
         return launch_slab<EPI>(mh, mw, g, stream);
     switch (mode) {
     case kPair: return launch_gemm_mode<EPI, kPair>(mh, mw, g, bn, stream);
-    case kMulticast: return launch_gemm_mode<EPI, kMulticast>(mh, mw, g, bn, stream);
     default: return launch_gemm_mode<EPI, kSolo>(mh, mw, g, bn, stream);
     }
 }

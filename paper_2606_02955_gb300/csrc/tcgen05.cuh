@@ -37,19 +37,6 @@ __device__ __forceinline__ void tma_load_2d_hint(void *dst, const CUtensorMap *m
         : "memory");
 }
 
-// The same load delivered to the same shared-memory offset, and signalled on the mbarrier at
-// the same offset, in every CTA of the cluster whose bit is set in cta_mask.
-__device__ __forceinline__ void tma_load_2d_multicast(void *dst, const CUtensorMap *map,
-                                                      int32_t x, int32_t y, uint64_t *bar,
-                                                      uint16_t cta_mask)
-{
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-        ".multicast::cluster [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(smem_addr(dst)),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar)), "h"(cta_mask)
-        : "memory");
-}
-
 // The CTA-pair form: the box lands in this CTA's shared memory and completes its bytes on
 // the mbarrier at `bar_cluster` (a shared::cluster address, here the even CTA's barrier).
 __device__ __forceinline__ void tma_load_2d_pair(void *dst, const CUtensorMap *map, int32_t x,
@@ -144,16 +131,6 @@ __device__ __forceinline__ void commit(uint64_t *bar)
     asm volatile(
         "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
             smem_addr(bar))
-        : "memory");
-}
-
-// commit() arriving on the mbarrier at the same offset in every CTA of cta_mask.
-__device__ __forceinline__ void commit_multicast(uint64_t *bar, uint16_t cta_mask)
-{
-    asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
-        " [%0], %1;" ::"r"(smem_addr(bar)),
-        "h"(cta_mask)
         : "memory");
 }
 

@@ -68,7 +68,7 @@ def draw_lmhead_case(seed):
     L = int(rng.integers(1, 65))
     H = int(rng.choice([8, 40, 72, 256, 520, 1024]))
     V = int(rng.choice([40, 300, 1000, 2050, 5000, 20000]))
-    variant = ("auto", "solo", "multicast", "pair", "slab")[rng.integers(5)]
+    variant = ("auto", "solo", "pair", "slab")[rng.integers(4)]
     bn = int(rng.choice([256, 208]))
     frac = float(rng.uniform(0.2, 1.0))
     return B, L, H, V, variant, bn, frac

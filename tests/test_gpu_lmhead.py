@@ -28,11 +28,11 @@ pytestmark = pytest.mark.gpu
 U = 2.0 ** -23
 
 
-@pytest.fixture(params=[(g, bn) for bn in (256, 208) for g in ("solo", "multicast", "pair")],
+@pytest.fixture(params=[(g, bn) for bn in (256, 208) for g in ("solo", "pair")],
                 ids=lambda p: "%s-n%d" % p)
 def cluster(request, monkeypatch):
-    """Every GEMM variant: one CTA per W tile, W halves multicast across a 2-CTA cluster, or
-    a CTA-pair MMA (M = 256), with vocabulary tiles of 256 or 208 entries."""
+    """Every tile GEMM variant: one CTA per W tile, or a CTA-pair MMA (M = 256), with
+    vocabulary tiles of 256 or 208 entries."""
     mode, bn = request.param
     monkeypatch.setenv("FDLLM_LMHEAD_GEMM", mode)
     monkeypatch.setenv("FDLLM_LMHEAD_BN", str(bn))
