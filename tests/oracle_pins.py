@@ -549,6 +549,109 @@ def pin_bonus_terms(o):
     assert np.isnan(t["G"][0, 4]) and np.isnan(t["B"][0, 4])
 
 
+
+MARGINS = os.path.join(os.path.dirname(GOLDEN), "decision_margins.json")
+
+
+def _select_any(o, conf, mask, rule, param, eta=None, eta_pos=None):
+    tok = np.arange(conf.size, dtype=np.int32).reshape(conf.shape)
+    if rule == "robust":
+        return o.select_robust_from_conf(conf, tok, mask, param, 0.0 if eta is None else eta,
+                                         eta_pos)
+    mode = {"profile": PROFILE, "factor": FACTOR, "threshold": THRESHOLD}[rule]
+    return o.select_from_conf(conf, tok, mask, mode, param)
+
+
+def pin_decision_margin_hand_worked(o):
+    """The decision margin (the distance that decides which rows parity may excuse) on
+    profiles whose margin is worked out by hand (tests/golden/decision_margins.json): the
+    rule quantity at n* and n* + 1, the rank gap, a tie block straddling n* with its
+    neighbour above or below closest, the progress fallback, n* = m, and the robust rule's
+    distance to a clipping point.  Every value is a multiple of 1/64, so the comparison is
+    exact."""
+    with open(MARGINS) as fh:
+        cases = json.load(fh)["cases"]
+    for case in cases:
+        conf = np.array([case["conf_by_pos"]], np.float64)
+        mask = (conf > 0).astype(np.uint8)
+        r = _select_any(o, conf, mask, case["rule"], case["param"], case.get("eta"))
+        assert r["n"][0] == case["nstar"], (case["name"], r["n"][0])
+        assert np.nonzero(r["commit"][0])[0].tolist() == case["commit_pos"], case["name"]
+        assert r["margin"][0] == case["margin"], (case["name"], r["margin"][0], case["margin"])
+
+
+def _tie_profile(rng, m, grid=256):
+    """m dyadic confidences in [8, 248] / grid with planted equal groups (ties across
+    positions), so that tie blocks often straddle the boundary."""
+    k = int(rng.integers(1, m + 1))
+    levels = rng.choice(np.arange(8, grid - 7), size=k, replace=False) / grid
+    c = levels[rng.integers(0, k, m)]
+    return c
+
+
+def pin_decision_margin_stability(o):
+    """What the margin means: no perturbation that moves every confidence by less than
+    margin / (n* + 2), and moves equal confidences together (bit-identical inputs give
+    bit-identical confidences on both sides), can change n* or the committed set.  The rule
+    quantity at rank n moves by at most (n + 1) times the perturbation (sorting is
+    1-Lipschitz in the largest change; L_n sums n confidences, U_n one), so the decisions at
+    n* and n* + 1 keep their sides, the rules' monotonicity in n carries them to every other
+    n, and gaps above twice the perturbation keep the committed ranks (whole tie blocks
+    move as one) in place.  For the robust rule the groups are equal lower confidences and
+    the perturbation is applied to c_hat, which stays on its side of its clipping point.
+    Checked on random dyadic profiles with planted ties, for every rule, with the
+    perturbations that push every group up, every group down, or neighbouring groups apart
+    and together."""
+    rng = np.random.default_rng(61)
+    rules = [("profile", (1.0, 0.875, 0.75, 0.5)), ("factor", (0.5, 1.0, 1.5, 2.0)),
+             ("threshold", (0.5, 0.75, 0.875)), ("robust", (1.0, 0.75))]
+    checked = 0
+    for trial in range(600):
+        rule, params = rules[trial % len(rules)]
+        param = float(params[rng.integers(len(params))])
+        m = int(rng.integers(1, 9))
+        L = m + int(rng.integers(0, 3))
+        c_hat = _tie_profile(rng, m)
+        pos = rng.permutation(L)[:m]
+        conf = np.zeros((1, L))
+        conf[0, pos] = c_hat
+        mask = (conf > 0).astype(np.uint8)
+        eta_pos = None
+        if rule == "robust":
+            eta_pos = np.zeros((1, L))
+            eta_pos[0, pos] = rng.integers(0, 9, m) / 256 if trial % 8 < 4 else 6 / 256
+            if trial % 3 == 0:  # some allowances just above or below their confidence
+                near = rng.random(m) < 0.5
+                eta_pos[0, pos[near]] = c_hat[near] + rng.integers(-2, 3, near.sum()) / 256
+        r0 = _select_any(o, conf, mask, rule, param, eta_pos=eta_pos)
+        M, nstar = float(r0["margin"][0]), int(r0["n"][0])
+        if not M > 0:
+            continue
+        eps = min(0.999 * M / (nstar + 2), 4 / 256)
+        low = conf[0] if eta_pos is None else np.maximum(conf[0] - eta_pos[0], 0.0)
+        # groups: equal (lower) confidences move together; clipped positions stay clipped
+        keys = {}
+        group = np.full(L, -1)
+        for l in pos:
+            key = low[l] if low[l] > 0 else ("clip", int(l))
+            group[l] = keys.setdefault(key, len(keys))
+        order = sorted(keys.items(), key=lambda kv: -(kv[0] if not isinstance(kv[0], tuple)
+                                                       else 0.0))
+        rank_of = {g: i for i, (_, g) in enumerate(order)}
+        signs = [np.ones(len(keys)), -np.ones(len(keys)),
+                 np.array([(-1.0) ** rank_of[g] for g in range(len(keys))]),
+                 np.array([-((-1.0) ** rank_of[g]) for g in range(len(keys))]),
+                 rng.choice([-1.0, 1.0], len(keys))]
+        for sg in signs:
+            pert = conf.copy()
+            pert[0, pos] += eps * sg[group[pos]]
+            r1 = _select_any(o, pert, mask, rule, param, eta_pos=eta_pos)
+            assert r1["n"][0] == nstar, (rule, param, c_hat, eps, M)
+            assert np.array_equal(r1["commit"], r0["commit"]), (rule, param, c_hat, eps, M)
+        checked += 1
+    assert checked > 400
+
+
 ALL_PINS = [
     pin_confidence_vs_torch, pin_confidence_closed_forms, pin_nonfinite, pin_hand_worked,
     pin_bruteforce_subsets, pin_equal_confidence_reduction, pin_heterogeneity_bonus,
@@ -556,4 +659,5 @@ ALL_PINS = [
     pin_reveal_and_ties, pin_end_to_end, pin_robust_zero_eta_is_profile,
     pin_robust_calibration_penalty, pin_robust_bruteforce, pin_robust_monotone_and_clipped,
     pin_bonus_terms, pin_half_widening, pin_extreme_magnitudes,
+    pin_decision_margin_hand_worked, pin_decision_margin_stability,
 ]

@@ -62,6 +62,20 @@ MUTANTS = {
     "robust_margin_not_strict": ("if (Gn[n - 1] > delta)", "if (Gn[n - 1] >= delta)"),
     "robust_delta_not_matched": ("const double delta = 1.0 - param;", "const double delta = param;",
                                  1),
+    # the decision margin: each term dropped or mis-measured
+    "margin_drops_next_rank": ("if (nstar < m && fabs(q[nstar]) < mg)\n                mg = fabs(q[nstar]);",
+                               ""),
+    "margin_at_n_star_only_from_rank": ("double mg = fabs(q[nstar - 1]);", "double mg = INFINITY;"),
+    "margin_drops_rank_gap": ("if (gap < mg)\n                mg = gap;", ""),
+    "margin_ignores_tie_block": ("if (cs[nstar] != v) {", "if (1) {"),
+    "margin_tie_block_ignores_above": ("if (a > 1 && cs[a - 2] - v < mg)\n        mg = cs[a - 2] - v;",
+                                       ""),
+    "margin_tie_block_ignores_below": ("if (b < m && v - cs[b] < mg)\n        mg = v - cs[b];", ""),
+    "robust_margin_drops_clip_gap": ("if (clip_gap < mg)\n                mg = clip_gap;", ""),
+    "robust_margin_drops_next_rank": (
+        "if (nstar < m && fabs(Gn[nstar] - delta) < mg)\n                mg = fabs(Gn[nstar] - delta);",
+        ""),
+    "robust_margin_drops_rank_gap": ("if (gap < mg)\n                mg = gap;", "", 1),
 }
 
 
