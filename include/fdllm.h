@@ -158,6 +158,14 @@ fdllm_status fdllm_select_static(const void *logits, int dtype, int B, int L, in
                                  uint8_t *mask, double param, int mode, int32_t *out_tokens,
                                  uint8_t *out_commit, int32_t *out_n, void *stream);
 
+/* The sticky device error of fdllm_select_static's array on the current device, as
+ * fdllm_device_status reports the library workspace's: synchronises `stream`, returns
+ * FDLLM_ERR_DEVICE if a kernel of a static call gave up a bounded wait (every row of that
+ * call also reports out_n = -2), FDLLM_OK otherwise, and clears the error.  Call it after a
+ * static call and before the next one, which clears the array's status word itself.
+ * Allocates nothing. */
+fdllm_status fdllm_static_status(void *stream);
+
 /* Step a1 alone (Sec. 3 "Notation"; Alg. 1 confidence loop): for every masked position,
  * out_conf = c = max softmax probability (fp32) and out_argmax = x_hat (int32, lowest index
  * among equal maxima).  Both [B, L] device arrays, written only at masked positions; a
@@ -313,7 +321,9 @@ fdllm_status fdllm_check_bounded_wait(double seconds, void *stream);
 /* Synchronises `stream`, then reports (and clears) the sticky device error of the library
  * workspace on the current device: FDLLM_ERR_DEVICE if a kernel gave up a bounded wait
  * since the last call, FDLLM_OK otherwise.  For fdllm_select_ws, pass the workspace to
- * fdllm_workspace_status instead. */
+ * fdllm_workspace_status instead.  Clearing an error also resets the workspace's work
+ * counter, which a launch that gave up may have left mid-queue, so that the next call
+ * starts from a clean header. */
 fdllm_status fdllm_device_status(void *stream);
 fdllm_status fdllm_workspace_status(void *workspace, void *stream);
 

@@ -20,7 +20,8 @@ __all__ = [
     "BF16", "FP32", "FP16", "PROFILE", "FACTOR", "THRESHOLD", "ROW_NONFINITE", "ROW_DEVICE_ERROR",
     "FdllmError", "fdllm_select", "fdllm_select_ws", "fdllm_workspace_bytes",
     "fdllm_confidence", "fdllm_select_from_conf", "fdllm_device_status",
-    "fdllm_workspace_status", "fdllm_release_workspace", "fdllm_status_string",
+    "fdllm_workspace_status", "fdllm_static_status", "fdllm_release_workspace",
+    "fdllm_status_string",
     "fdllm_version", "library_path", "fdllm_select_static", "fdllm_select_robust",
     "fdllm_profile_terms", "fdllm_check_bounded_wait", "fdllm_decode_loop", "FORWARD_FN",
     "fdllm_lmhead_select", "fdllm_lmhead_confidence", "fdllm_lmhead_logits",
@@ -89,6 +90,8 @@ def _load():
     lib.fdllm_device_status.restype = i
     lib.fdllm_workspace_status.argtypes = [p, p]
     lib.fdllm_workspace_status.restype = i
+    lib.fdllm_static_status.argtypes = [p]
+    lib.fdllm_static_status.restype = i
     lib.fdllm_release_workspace.argtypes = []
     lib.fdllm_release_workspace.restype = None
     lib.fdllm_status_string.argtypes = [i]
@@ -533,6 +536,12 @@ def fdllm_device_status(stream=None) -> int:
 @_on_device
 def fdllm_workspace_status(workspace: torch.Tensor, stream=None) -> int:
     return _load().fdllm_workspace_status(_dev(workspace, "workspace", torch.uint8), _stream(stream))
+
+
+def fdllm_static_status(stream=None) -> int:
+    """Synchronises and returns (clearing it) the sticky device status of
+    fdllm_select_static's fixed array on the current device."""
+    return _load().fdllm_static_status(_stream(stream))
 
 
 def fdllm_release_workspace() -> None:

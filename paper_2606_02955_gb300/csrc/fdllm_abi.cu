@@ -175,7 +175,11 @@ fdllm_status check_select_args(const void *logits, int dtype, int B, int L, int 
     return plan_fits((int64_t)B * L, (int64_t)V * esize_of(dtype)) ? FDLLM_OK : FDLLM_ERR_ARG;
 }
 
-fdllm_status read_and_clear_status(uint32_t *status, cudaStream_t stream)
+// Reads the sticky status word and, when it is set, zeroes `clear_bytes` from it: for a
+// workspace header the status word and the vocab reduction's work counter, which a launch
+// that gave up a wait may leave mid-queue (it stops fetching before its last unit).
+fdllm_status read_and_clear_status(uint32_t *status, cudaStream_t stream,
+                                   size_t clear_bytes = sizeof(uint32_t))
 {
     uint32_t host = 0;
     if (cudaMemcpyAsync(&host, status, sizeof host, cudaMemcpyDeviceToHost, stream) !=
@@ -185,11 +189,14 @@ fdllm_status read_and_clear_status(uint32_t *status, cudaStream_t stream)
         return FDLLM_ERR_CUDA;
     if (host == 0)
         return FDLLM_OK;
-    if (cudaMemsetAsync(status, 0, sizeof(uint32_t), stream) != cudaSuccess ||
+    if (cudaMemsetAsync(status, 0, clear_bytes, stream) != cudaSuccess ||
         cudaStreamSynchronize(stream) != cudaSuccess)
         return FDLLM_ERR_CUDA;
     return FDLLM_ERR_DEVICE;
 }
+
+// Status word and work counter at the head of every workspace.
+constexpr size_t kHeaderClearBytes = 2 * sizeof(uint32_t);
 
 // Scratch for fdllm_select_static: a fixed array in device memory that every GPU loading
 // this library holds until the process exits, so that a selection step needs no
@@ -467,7 +474,8 @@ fdllm_status fdllm_device_status(void *stream)
     }
     if (!ptr)
         return FDLLM_OK;
-    return read_and_clear_status(static_cast<uint32_t *>(ptr), static_cast<cudaStream_t>(stream));
+    return read_and_clear_status(static_cast<uint32_t *>(ptr), static_cast<cudaStream_t>(stream),
+                                 kHeaderClearBytes);
 }
 
 fdllm_status fdllm_workspace_status(void *workspace, void *stream)
@@ -475,7 +483,17 @@ fdllm_status fdllm_workspace_status(void *workspace, void *stream)
     if (!workspace || (reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0)
         return FDLLM_ERR_WORKSPACE;
     return read_and_clear_status(static_cast<uint32_t *>(workspace),
-                                 static_cast<cudaStream_t>(stream));
+                                 static_cast<cudaStream_t>(stream), kHeaderClearBytes);
+}
+
+fdllm_status fdllm_static_status(void *stream)
+{
+    void *ws = nullptr;
+    fdllm_status st = static_scratch_address(&ws);
+    if (st != FDLLM_OK)
+        return st;
+    return read_and_clear_status(static_cast<uint32_t *>(ws), static_cast<cudaStream_t>(stream),
+                                 kHeaderClearBytes);
 }
 
 void fdllm_release_workspace(void)

@@ -43,7 +43,6 @@ constexpr uint32_t kAccStride = 256;  // TMEM columns between the two accumulato
 constexpr uint32_t kTmemCols = 512;
 constexpr size_t kBarrierBytes = 256;
 constexpr size_t kRingBudget = 220 * 1024;
-constexpr uint64_t kDrainLimitNs = 100000000ull;  // waits for own copies after an abort
 
 // How the CTAs of a cluster share a W tile.
 enum Mode {

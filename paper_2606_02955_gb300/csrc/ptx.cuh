@@ -8,6 +8,9 @@ namespace fdllm {
 
 // A wait on an mbarrier gives up after this long and records FDLLM_DEVSTAT_TIMEOUT.
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s
+// After a wait gave up, how long a CTA waits for its own asynchronous copies still in
+// flight (they write its shared memory) before it exits.
+constexpr uint64_t kDrainLimitNs = 100000000ull;  // 100 ms
 constexpr uint32_t kDevStatTimeout = 1u;
 
 __device__ __forceinline__ uint32_t smem_addr(const void *p)

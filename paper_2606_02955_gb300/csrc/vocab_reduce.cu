@@ -346,7 +346,7 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
             const uint32_t n = (uint32_t)min((int64_t)kChunkVecs, v1 - v);
             const uint32_t s = k % kStages;
             if (k >= kStages && !mbar_wait(&sm.empty[s], ((k / kStages) - 1) & 1, a.status))
-                return false;  // math warps stopped; issued copies complete on their own
+                return false;  // the math warps stopped consuming; the caller drains
             ChunkMeta cm;
             cm.n = n;
             cm.vec_base = (uint32_t)v;
@@ -466,34 +466,51 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
                 *a.next_unit = 0;
             return u;
         };
+        bool alive = true;  // false once a bounded wait has given up
         if (first_tried) {
             fetched(u_next);
+            alive = first_issued;
         } else if (blockIdx.x < total) {
             // the first unit was not within the producer's scan
             u_next = fetched(G + atomicAdd(a.next_unit, 1u));
             first_issued = issue_unit(blockIdx.x,
                                       masked_row(blockIdx.x / upr, sm.bits, sm.pref, nwords));
+            alive = first_issued;
         }
         if (first_issued) {
             // Then the work queue, which hands out units gridDim.x, gridDim.x + 1, ...
             uint32_t u = u_next;
             while (u < total) {
                 const uint32_t un = fetched(G + atomicAdd(a.next_unit, 1u));
-                if (!issue_unit(u, masked_row(u / upr, sm.bits, sm.pref, nwords)))
-                    return;
+                if (!issue_unit(u, masked_row(u / upr, sm.bits, sm.pref, nwords))) {
+                    alive = false;
+                    break;
+                }
                 u = un;
             }
         }
-        const uint32_t s = k % kStages;
-        if (k >= kStages && !mbar_wait(&sm.empty[s], ((k / kStages) - 1) & 1, a.status))
-            return;
-        ChunkMeta end;
-        end.n = 0;
-        end.vec_base = 0;
-        end.last = 1;
-        end.pidx = kEndMarker;
-        sm.meta[s] = end;
-        mbar_arrive(&sm.full[s]);
+        if (alive) {
+            const uint32_t s = k % kStages;
+            if (k < kStages || mbar_wait(&sm.empty[s], ((k / kStages) - 1) & 1, a.status)) {
+                ChunkMeta end;
+                end.n = 0;
+                end.vec_base = 0;
+                end.last = 1;
+                end.pidx = kEndMarker;
+                sm.meta[s] = end;
+                mbar_arrive(&sm.full[s]);
+            } else {
+                alive = false;
+            }
+        }
+        if (!alive) {
+            // A bounded wait gave up.  Copies already issued still write this CTA's shared
+            // memory, so before the producer lets the CTA exit it waits (bounded again) for
+            // the last chunk issued into each stage; every earlier chunk of a stage completed
+            // before the stage was reused.
+            for (uint32_t c = k > (uint32_t)kStages ? k - (uint32_t)kStages : 0u; c < k; ++c)
+                mbar_wait(&sm.full[c % kStages], (c / kStages) & 1u, a.status, kDrainLimitNs);
+        }
     } else if (warp <= NW) {
         // ------------------------------------------------------------ math warps
         const int mw = warp - 1;

@@ -34,3 +34,29 @@ def test_bounded_wait_runs_out_and_device_stays_usable(fd, orc):
 def test_bounded_wait_rejects_bad_limits(fd):
     assert fd.fdllm_check_bounded_wait(0.0) == 1
     assert fd.fdllm_check_bounded_wait(60.0) == 1
+
+
+def test_clearing_an_error_resets_the_work_counter(fd, orc):
+    """A launch that gave up a wait may stop fetching from its work queue before its last
+    unit and so leave the counter mid-queue; the status read that reports the error clears
+    both words, so that the next call on the workspace processes every unit.  The left-over
+    state is written into a caller workspace from the host: no kernel is made to fail."""
+    w = syn.WORKLOADS["target_b8_l32_bf16"]
+    logits = syn.make_logits(w, seed=13, device="cuda")
+    mask_np = syn.make_mask(w, seed=13)
+    ws = torch.zeros(fd.fdllm_workspace_bytes(w.B, w.L, w.V, fd.BF16), dtype=torch.uint8,
+                     device="cuda")
+    header = ws[:8].view(torch.int32)
+    header.copy_(torch.tensor([1, 37], dtype=torch.int32))
+    assert fd.fdllm_workspace_status(ws) == ERR_DEVICE
+    assert header.cpu().tolist() == [0, 0]
+    assert fd.fdllm_workspace_status(ws) == 0
+    mask = torch.from_numpy(mask_np.copy()).cuda()
+    tok, commit, n = fd.fdllm_select_ws(logits, mask, 0.75, fd.PROFILE, ws)
+    torch.cuda.synchronize()
+    assert fd.fdllm_workspace_status(ws) == 0 and header.cpu().tolist() == [0, 0]
+    ref = orc.select(syn.host_bits(logits), mask_np, 0, 0.75)
+    ok = ref["margin"] >= 1e-5
+    assert ok.sum() >= w.B // 2
+    assert np.array_equal(n.cpu().numpy()[ok], ref["n"][ok])
+    assert np.array_equal(commit.cpu().numpy()[ok], ref["commit"][ok])

@@ -24,6 +24,8 @@ def _c_entry(path):
     p, i, d = ctypes.c_void_p, ctypes.c_int, ctypes.c_double
     lib.fdllm_select_static.argtypes = [p, i, i, i, i, p, d, i, p, p, p, p]
     lib.fdllm_select_static.restype = i
+    lib.fdllm_static_status.argtypes = [p]
+    lib.fdllm_static_status.restype = i
     lib.fdllm_workspace_bytes.argtypes = [i, i, i, i]
     lib.fdllm_workspace_bytes.restype = ctypes.c_size_t
     return lib
@@ -59,6 +61,7 @@ def test_static_scratch_matches_select_on_two_calls(fd, name, mode, param):
                                      param, mode, tok.data_ptr(), commit.data_ptr(),
                                      n.data_ptr(), stream)
         assert st == OK, "call %d returned %d" % (call, st)
+        assert lib.fdllm_static_status(stream) == OK, "call %d: device error" % call
         torch.cuda.synchronize()
         got = [tok.cpu().numpy(), commit.cpu().numpy(), n.cpu().numpy(), mask.cpu().numpy()]
         for a, b, what in zip(ref, got, ("tokens", "commit", "n", "mask")):
