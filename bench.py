@@ -9,12 +9,17 @@ profile rule with f = 1 (delta = 0).
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
                   [--workload NAME] [--no-graph]
 
-Prints one JSON line (rank 0).  Under torchrun (N > 1) every rank runs its own batch on its
-own GPU (weak scaling, no data exchange); the time is the max over ranks.  The roofline
+Prints one JSON line (rank 0).  With N > 1 every rank runs its own batch on its own GPU
+(weak scaling, no data exchange); the time is the max over ranks.  Started without
+torchrun's environment, --gpus N > 1 launches the N ranks itself (torch.distributed.run on
+127.0.0.1).  The main timed region covers at least --min-steps steps (1000).  The roofline
 object times the vocabulary reduction by itself (fdllm_vocab_reduce) against the measured
-copy bandwidth.  At N = 1 the line also carries `evolving`: the serving workload with masks
-evolving from step to step until every row has finished, measured after the timed region
-(--skip-evolving leaves it out).  Other measurements, each one JSON line:
+copy bandwidth.  At N = 1 the line also carries, measured after the timed region:
+`evolving` (the serving workload with masks evolving from step to step until every row has
+finished), `per_config` (the single-block, mixed-mask, tie-group and full-sequence
+workloads, each beside the oracle on a bounded sample) and `lmhead` (the LM-head-fused step
+at B = 64 and 16); --skip-evolving, --skip-per-config and --skip-lmhead leave them out.
+Other measurements, each one JSON line:
   --evolving      masks evolving from step to step until every row has finished
   --loop          the full-sequence workload (B = 16, L = 1024) selected until no mask remains
   --lmhead        the LM-head-fused step against cuBLAS logits + selection
@@ -112,28 +117,76 @@ _REASON_BITS = {
 
 
 class ClockSampler:
-    """nvidia-smi sampling of SM clocks and throttle reasons while work runs."""
+    """SM clock and clock-event reasons sampled while work runs.  NVML is read through
+    ctypes every `period_ms` milliseconds (read-only queries: nothing is set), so that even
+    a timed region of some tens of milliseconds holds several samples; without NVML,
+    nvidia-smi's own loop."""
 
-    def __init__(self, gpu_index: int, period_ms: int = 50):
+    def __init__(self, gpu_index: int, period_ms: float = 4.0, pci_bus_id: str | None = None):
         self.gpu = gpu_index
+        self.pci = pci_bus_id
         self.period = period_ms
         self.samples = []  # (t, sm_mhz, max_mhz, reasons_bitmask)
+        self.source = None
         self.proc = None
         self.thread = None
+        self._stop = threading.Event()
+
+    def _nvml_handle(self):
+        import ctypes
+        try:
+            lib = ctypes.CDLL("libnvidia-ml.so.1")
+        except OSError:
+            return None, None
+        if lib.nvmlInit_v2() != 0:
+            return None, None
+        h = ctypes.c_void_p()
+        ok = False
+        if self.pci:
+            ok = lib.nvmlDeviceGetHandleByPciBusId_v2(self.pci.encode(), ctypes.byref(h)) == 0
+        if not ok:
+            ok = lib.nvmlDeviceGetHandleByIndex_v2(ctypes.c_uint(self.gpu), ctypes.byref(h)) == 0
+        if not ok:
+            lib.nvmlShutdown()
+            return None, None
+        return lib, h
 
     def start(self):
+        lib, h = self._nvml_handle()
+        if lib is not None:
+            self.source = "nvml"
+            self.thread = threading.Thread(target=self._poll_nvml, args=(lib, h), daemon=True)
+            self.thread.start()
+            return self
         cmd = ["nvidia-smi", "-i", str(self.gpu),
                "--query-gpu=clocks.sm,clocks.max.sm,clocks_event_reasons.active",
-               "--format=csv,noheader,nounits", "-lms", str(self.period)]
+               "--format=csv,noheader,nounits", "-lms", str(max(20, int(self.period)))]
         try:
             self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL,
                                          text=True)
         except OSError:
             self.proc = None
             return self
+        self.source = "nvidia-smi"
         self.thread = threading.Thread(target=self._read, daemon=True)
         self.thread.start()
         return self
+
+    def _poll_nvml(self, lib, h):
+        import ctypes
+        sm, mx, rs = ctypes.c_uint(), ctypes.c_uint(), ctypes.c_ulonglong()
+        reasons_fn = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            getattr(lib, "nvmlDeviceGetCurrentClocksThrottleReasons")
+        try:
+            while not self._stop.is_set():
+                if (lib.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(sm)) == 0
+                        and lib.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0
+                        and reasons_fn(h, ctypes.byref(rs)) == 0):
+                    self.samples.append((time.time(), float(sm.value), float(mx.value),
+                                         int(rs.value)))
+                self._stop.wait(self.period / 1e3)
+        finally:
+            lib.nvmlShutdown()
 
     def _read(self):
         for line in self.proc.stdout:
@@ -147,6 +200,7 @@ class ClockSampler:
                 continue
 
     def stop(self):
+        self._stop.set()
         if self.proc is not None:
             self.proc.terminate()
             try:
@@ -161,17 +215,161 @@ class ClockSampler:
         used = inside if inside else self.samples
         if not used:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"],
-                    "samples_in_timed_region": 0}
+                    "samples_in_timed_region": 0, "source": self.source}
         mask = 0
         for s in used:
             mask |= s[3]
         reasons = [name for bit, name in _REASON_BITS.items() if mask & bit and bit != 0x1]
         return {"sm_mhz": statistics.median(s[1] for s in used),
                 "sm_max_mhz": max(s[2] for s in used), "reasons": reasons,
-                "samples_in_timed_region": len(inside)}
+                "samples_in_timed_region": len(inside), "source": self.source,
+                "period_ms": self.period}
+
+
+def pci_bus_id(torch, dev) -> str | None:
+    """The device's PCI address in NVML's form, so that the sampler watches the GPU this
+    process runs on whatever CUDA_VISIBLE_DEVICES says."""
+    p = torch.cuda.get_device_properties(dev)
+    if not all(hasattr(p, k) for k in ("pci_domain_id", "pci_bus_id", "pci_device_id")):
+        return None
+    return "%08X:%02X:%02X.0" % (p.pci_domain_id, p.pci_bus_id, p.pci_device_id)
+
+
+# ----------------------------------------------------------------------------- ranks
+def free_port() -> int:
+    import socket
+    with socket.socket() as sk:
+        sk.bind(("127.0.0.1", 0))
+        return sk.getsockname()[1]
+
+
+def launch_ranks(n: int, argv: list[str], script: str | None = None) -> int:
+    """Run `script` (this file by default) as n ranks on this node through
+    torch.distributed.run, rendezvous on 127.0.0.1; returns the launcher's exit code.  Each
+    rank reads RANK / LOCAL_RANK / WORLD_SIZE from its environment."""
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1",
+           "--nproc-per-node", str(n), "--master-addr", "127.0.0.1",
+           "--master-port", str(free_port()), script or os.path.abspath(__file__), *argv]
+    return subprocess.call(cmd)
+
+
+def init_dist(world: int, device):
+    """The process group of a multi-rank run (None for one rank): NCCL between GPUs, gloo for
+    CPU ranks.  The only collectives are the timing gather and barriers."""
+    if world <= 1:
+        return None
+    import torch.distributed as dist
+    if getattr(device, "type", str(device)) == "cuda":
+        dist.init_process_group("nccl", device_id=device)
+    else:
+        dist.init_process_group("gloo")
+    return dist
 
 
 # ----------------------------------------------------------------------------- our arm
+def graph_runner(torch, stream, fn, per_replay: int, no_graph: bool = False):
+    """A callable run(r) that issues `per_replay` consecutive calls fn(i) on `stream`: one
+    CUDA graph replay (or eager launches with no_graph).  fn is called a few times first so
+    that one-time set-up (kernel attributes, workspaces) stays out of the graph."""
+    with torch.cuda.stream(stream):
+        for i in range(max(3, per_replay)):
+            fn(i)
+    stream.synchronize()
+    if no_graph:
+        def run(r):
+            with torch.cuda.stream(stream):
+                for i in range(per_replay):
+                    fn(r * per_replay + i)
+        return run
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for i in range(per_replay):
+            fn(i)
+
+    def run(_r):
+        g.replay()
+    return run
+
+
+def time_runner(torch, stream, run, n_rep: int, warm_rep: int, dist=None):
+    """Seconds of n_rep runs on `stream` by CUDA events, after warm_rep untimed runs, with a
+    synchronize (and a barrier across ranks) on both sides; also the wall-clock bounds."""
+    for r in range(warm_rep):
+        with torch.cuda.stream(stream):
+            run(r)
+    stream.synchronize()
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    t_wall0 = time.time()
+    e0.record(stream)
+    with torch.cuda.stream(stream):
+        for r in range(n_rep):
+            run(r)
+    e1.record(stream)
+    e1.synchronize()
+    t_wall1 = time.time()
+    torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    return e0.elapsed_time(e1) / 1e3, t_wall0, t_wall1
+
+
+class SelectionBench:
+    """One workload's selection step over `n_buf` rotating logits buffers (each with its own
+    copy of the initial mask, all restored by one copy per graph replay), so that a replay of
+    n_buf steps reads more than the 129 MB L2 when n_buf * buffer size does."""
+
+    def __init__(self, torch, fd, syn, w, seed: int, n_buf: int, dev, stream):
+        self.torch, self.fd, self.w, self.dev, self.stream = torch, fd, w, dev, stream
+        self.n_buf = max(1, n_buf)
+        self.bufs = [syn.make_logits(w, seed=seed + i, device=dev) for i in range(self.n_buf)]
+        self.mask0_np = syn.make_mask(w, seed=seed)
+        self.mask0 = torch.from_numpy(self.mask0_np).to(dev)
+        self.masked_rows = int(self.mask0_np.sum())
+        self.alg_bytes = self.masked_rows * w.V * w.elem_bytes
+        self.masks = self.mask0.unsqueeze(0).repeat(self.n_buf, 1, 1).contiguous()
+        self.masks0 = self.masks.clone()
+        self.tok = torch.full((w.B, w.L), -1, dtype=torch.int32, device=dev)
+        self.commit = torch.empty((w.B, w.L), dtype=torch.uint8, device=dev)
+        self.n_out = torch.empty((w.B,), dtype=torch.int32, device=dev)
+
+    @property
+    def buffer_bytes(self) -> int:
+        return self.bufs[0].numel() * self.bufs[0].element_size()
+
+    def l2_policy(self) -> str:
+        return ("inputs larger than L2: %d rotating logits buffers of %.1f MB (%.2f GB > "
+                "129 MB L2)" % (self.n_buf, self.buffer_bytes / 1e6,
+                                self.n_buf * self.buffer_bytes / 1e9))
+
+    def step_fn(self, rule: str, param: float, eta: float = 0.0):
+        fd, n_buf = self.fd, self.n_buf
+        mode = fd.MODES["profile" if rule == "robust" else rule]
+
+        def step(i):
+            if i % n_buf == 0:  # steady state: the same masked rows every step
+                self.masks.copy_(self.masks0, non_blocking=True)
+            j = i % n_buf
+            if rule == "robust":
+                fd.fdllm_select_robust(self.bufs[j], self.masks[j], param, eta, None, self.tok,
+                                       self.commit, self.n_out, stream=self.stream)
+            else:
+                fd.fdllm_select(self.bufs[j], self.masks[j], param, mode, self.tok,
+                                self.commit, self.n_out, stream=self.stream)
+        return step
+
+    def time_steps(self, fn, steps: int, warmup: int, no_graph=False, dist=None):
+        """(seconds, steps timed, wall bounds, runner) for at least `steps` calls of fn."""
+        run = graph_runner(self.torch, self.stream, fn, self.n_buf, no_graph)
+        replays = max(1, -(-steps // self.n_buf))
+        warm = max(1, -(-warmup // self.n_buf))
+        sec, t0, t1 = time_runner(self.torch, self.stream, run, replays, warm, dist)
+        return sec, replays * self.n_buf, (t0, t1), run
+
+
 def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
     import numpy as np
     import torch
@@ -181,107 +379,34 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
 
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
-    dist = None
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl", device_id=dev)
+    dist = init_dist(world, dev)
 
     w = syn.WORKLOADS[args.workload]
-    seed = rank_seed(1234, rank)
-    n_buf = max(1, args.buffers)
-    bufs = [syn.make_logits(w, seed=seed + i, device=dev) for i in range(n_buf)]
-    mask0_np = syn.make_mask(w, seed=seed)
-    mask0 = torch.from_numpy(mask0_np).to(dev)
-    masked_rows = int(mask0_np.sum())
-    alg_bytes = masked_rows * w.V * w.elem_bytes
-    mode = {"profile": fd.PROFILE, "factor": fd.FACTOR, "threshold": fd.THRESHOLD,
-            "robust": fd.PROFILE}[args.mode]
-
-    # one mask buffer per logits buffer, all restored by a single copy per replay
-    masks = mask0.unsqueeze(0).repeat(n_buf, 1, 1).contiguous()
-    masks0 = masks.clone()
-    tok = torch.full((w.B, w.L), -1, dtype=torch.int32, device=dev)
-    commit = torch.empty((w.B, w.L), dtype=torch.uint8, device=dev)
-    n_out = torch.empty((w.B,), dtype=torch.int32, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+    sb = SelectionBench(torch, fd, syn, w, rank_seed(1234, rank), args.buffers, dev, stream)
     conf = torch.empty((w.B, w.L), dtype=torch.float32, device=dev)
     amax = torch.empty((w.B, w.L), dtype=torch.int32, device=dev)
-    stream = torch.cuda.Stream(device=dev)
-
-    def step(i):
-        if i % n_buf == 0:  # steady state: the same masked rows every step
-            masks.copy_(masks0, non_blocking=True)
-        if args.mode == "robust":
-            fd.fdllm_select_robust(bufs[i % n_buf], masks[i % n_buf], args.param, args.eta,
-                                   None, tok, commit, n_out, stream=stream)
-        else:
-            fd.fdllm_select(bufs[i % n_buf], masks[i % n_buf], args.param, mode, tok, commit,
-                            n_out, stream=stream)
+    step = sb.step_fn(args.mode, args.param, args.eta)
 
     def k1_only(i):
-        fd.fdllm_confidence(bufs[i % n_buf], mask0, conf, amax, stream=stream)
+        fd.fdllm_confidence(sb.bufs[i % sb.n_buf], sb.mask0, conf, amax, stream=stream)
 
     def k1_alone(i):  # the reduction kernel by itself
-        fd.fdllm_vocab_reduce(bufs[i % n_buf], mask0, stream=stream)
+        fd.fdllm_vocab_reduce(sb.bufs[i % sb.n_buf], sb.mask0, stream=stream)
 
-    def make_runner(fn, per_replay):
-        """A callable running `per_replay` consecutive steps (one CUDA graph replay)."""
-        with torch.cuda.stream(stream):
-            for i in range(max(3, per_replay)):  # warm: allocations, attributes
-                fn(i)
-        stream.synchronize()
-        if args.no_graph:
-            def run(r):
-                with torch.cuda.stream(stream):
-                    for i in range(per_replay):
-                        fn(r * per_replay + i)
-            return run
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, stream=stream):
-            for i in range(per_replay):
-                fn(i)
-
-        def run(_r):
-            g.replay()
-        return run
-
-    per_replay = n_buf
-    replays = max(1, -(-args.steps // per_replay))
-    steps = replays * per_replay
-    warm_replays = max(1, -(-args.warmup // per_replay))
-
-    def timed(run, n_rep):
-        for r in range(warm_replays):
-            with torch.cuda.stream(stream):
-                run(r)
-        stream.synchronize()
-        if dist is not None:
-            dist.barrier()
-        torch.cuda.synchronize()
-        e0 = torch.cuda.Event(enable_timing=True)
-        e1 = torch.cuda.Event(enable_timing=True)
-        t_wall0 = time.time()
-        e0.record(stream)
-        with torch.cuda.stream(stream):
-            for r in range(n_rep):
-                run(r)
-        e1.record(stream)
-        e1.synchronize()
-        t_wall1 = time.time()
-        torch.cuda.synchronize()
-        if dist is not None:
-            dist.barrier()
-        return e0.elapsed_time(e1) / 1e3, t_wall0, t_wall1
-
-    sampler = ClockSampler(local_rank).start() if rank == 0 else None
-    step_run = make_runner(step, per_replay)
-    t_step, tw0, tw1 = timed(step_run, replays)
-    k1_run = make_runner(k1_only, per_replay)
-    t_k1, _, _ = timed(k1_run, replays)
-    k1a_run = make_runner(k1_alone, per_replay)
-    t_k1a, _, _ = timed(k1a_run, replays)
+    # at least min_steps timed steps whatever --steps says (the serving workload is quoted
+    # over 1000 steps), so that the region holds several clock samples and >= 100 replays
+    want = max(args.steps, args.min_steps)
+    sampler = None
+    if rank == 0:
+        sampler = ClockSampler(local_rank, pci_bus_id=pci_bus_id(torch, dev)).start()
+    t_step, steps, (tw0, tw1), step_run = sb.time_steps(step, want, args.warmup, args.no_graph,
+                                                        dist)
+    t_k1, _, _, _ = sb.time_steps(k1_only, want, args.warmup, args.no_graph, dist)
+    t_k1a, _, _, _ = sb.time_steps(k1_alone, want, args.warmup, args.no_graph, dist)
     # distribution of the step time: replays timed one by one (outside the timed region)
     per_step_us = []
-    for r in range(min(200, replays)):
+    for r in range(min(200, steps // sb.n_buf)):
         a0 = torch.cuda.Event(enable_timing=True)
         a1 = torch.cuda.Event(enable_timing=True)
         a0.record(stream)
@@ -289,73 +414,46 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
             step_run(r)
         a1.record(stream)
         a1.synchronize()
-        per_step_us.append(a0.elapsed_time(a1) * 1e3 / per_replay)
+        per_step_us.append(a0.elapsed_time(a1) * 1e3 / sb.n_buf)
     if sampler is not None:
-        time.sleep(0.12)
+        time.sleep(0.02)
         sampler.stop()
 
     times = gather_times(dist, t_step, dev) if dist is not None else [t_step]
     agg = aggregate(w.B, steps, times)
     ms_per_step = agg["seconds"] / steps * 1e3
+    warm_steps = max(1, -(-args.warmup // sb.n_buf)) * sb.n_buf
 
     # end to end: the public call with pinned host buffers, copies inside the timed region
     e2e = None
     if not args.skip_e2e:
-        h_logits = torch.empty(bufs[0].shape, dtype=bufs[0].dtype, pin_memory=True)
-        h_logits.copy_(bufs[0])
-        h_mask = torch.from_numpy(mask0_np.copy()).pin_memory()
-        h_tok = torch.full((w.B, w.L), -1, dtype=torch.int32).pin_memory()
-        h_commit = torch.empty((w.B, w.L), dtype=torch.uint8).pin_memory()
-        h_n = torch.empty((w.B,), dtype=torch.int32).pin_memory()
-        for _ in range(2):
-            h_mask.copy_(torch.from_numpy(mask0_np))
-            fd.fdllm_select(h_logits, h_mask, args.param, mode, h_tok, h_commit, h_n)
-        e2e_steps = max(3, min(20, args.steps // 50))
-        torch.cuda.synchronize()
-        t0 = time.perf_counter()
-        for _ in range(e2e_steps):
-            h_mask.copy_(torch.from_numpy(mask0_np))
-            fd.fdllm_select(h_logits, h_mask, args.param, mode, h_tok, h_commit, h_n)
-        t_e2e = time.perf_counter() - t0
-        e2e = {"value": w.B * e2e_steps / t_e2e, "unit": UNIT,
-               # only the masked rows cross the host link (read by the GPU from pinned memory)
-               "h2d_bytes_per_step": masked_rows * w.V * w.elem_bytes
-               + h_mask.numel() + h_tok.numel() * 4,
-               "path": "pinned host logits; masked rows read over the host link by "
-                       "fdllm_gather_masked_rows, then fdllm_select; results copied back",
-               "d2h_bytes_per_step": h_tok.numel() * 4 + h_commit.numel() + h_n.numel() * 4
-               + h_mask.numel(),
-               "steps": e2e_steps}
-        del h_logits
+        e2e = run_e2e(args, torch, fd, w, sb)
 
     result = None
     if rank == 0:
         peak, peak_kind = peak_hbm_gbs()
         k1_s = t_k1a / steps
-        achieved = alg_bytes / k1_s / 1e9
+        achieved = sb.alg_bytes / k1_s / 1e9
         traffic = ncu_traffic()
         clocks = sampler.summary(tw0, tw1) if sampler is not None else None
         result = {
             "metric": METRIC, "value": agg["value"], "unit": UNIT, "n_gpus": world,
-            "steps": steps, "warmup": warm_replays * per_replay,
+            "steps": steps, "warmup": warm_steps,
             "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
             "config": {
                 "workload": w.name, "description": w.description, "B": w.B, "L": w.L,
                 "V": w.V, "rule": args.mode, "param": args.param,
-                "masked_rows_per_step": masked_rows,
-                "logits_bytes_per_step": alg_bytes,
-                "logits_gbs_per_step": alg_bytes / (ms_per_step * 1e-3) / 1e9,
-                "positions_per_s": masked_rows * world / (ms_per_step * 1e-3),
+                "masked_rows_per_step": sb.masked_rows,
+                "logits_bytes_per_step": sb.alg_bytes,
+                "logits_gbs_per_step": sb.alg_bytes / (ms_per_step * 1e-3) / 1e9,
+                "positions_per_s": sb.masked_rows * world / (ms_per_step * 1e-3),
+                "steps_requested": args.steps,
                 "step_us_distribution": {
                     "median": float(np.median(per_step_us)), "min": float(min(per_step_us)),
                     "max": float(max(per_step_us)), "replays": len(per_step_us),
-                    "steps_per_replay": per_replay},
-                "l2_policy": "inputs larger than L2: %d rotating logits buffers of %.0f MB "
-                             "(%.2f GB > 129 MB L2)" % (n_buf, bufs[0].numel() *
-                                                        bufs[0].element_size() / 1e6,
-                                                        n_buf * bufs[0].numel() *
-                                                        bufs[0].element_size() / 1e9),
+                    "steps_per_replay": sb.n_buf},
+                "l2_policy": sb.l2_policy(),
                 "cuda_graph": not args.no_graph,
                 "parallelism": "dp%d (independent batches, no collective)" % world,
             },
@@ -367,16 +465,215 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
                           "reduction kernel alone",
                 "kernel_us": k1_s * 1e6, "peak_source": peak_kind,
                 "kernel_us_with_finalize": t_k1 / steps * 1e6,
-                "algorithmic_bytes_per_launch": alg_bytes,
+                "algorithmic_bytes_per_launch": sb.alg_bytes,
             },
             "clocks": clocks,
             "gpu_launches": 2 * steps,
             "e2e": e2e,
         }
+    del sb
     if dist is not None:
         dist.barrier()
         dist.destroy_process_group()
     return result
+
+
+def run_e2e(args, torch, fd, w, sb) -> dict:
+    """The public call with page-locked host buffers: the host copies of the step's inputs
+    and results are inside the timed region (the masked rows are read by the GPU over the
+    host link, the rest copied)."""
+    h_logits = torch.empty(sb.bufs[0].shape, dtype=sb.bufs[0].dtype, pin_memory=True)
+    h_logits.copy_(sb.bufs[0])
+    h_mask = torch.from_numpy(sb.mask0_np.copy()).pin_memory()
+    h_tok = torch.full((w.B, w.L), -1, dtype=torch.int32).pin_memory()
+    h_commit = torch.empty((w.B, w.L), dtype=torch.uint8).pin_memory()
+    h_n = torch.empty((w.B,), dtype=torch.int32).pin_memory()
+    mode = fd.MODES["profile" if args.mode == "robust" else args.mode]
+    for _ in range(2):
+        h_mask.copy_(torch.from_numpy(sb.mask0_np))
+        fd.fdllm_select(h_logits, h_mask, args.param, mode, h_tok, h_commit, h_n)
+    e2e_steps = max(3, min(20, args.steps // 50))
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        h_mask.copy_(torch.from_numpy(sb.mask0_np))
+        fd.fdllm_select(h_logits, h_mask, args.param, mode, h_tok, h_commit, h_n)
+    t_e2e = time.perf_counter() - t0
+    out = {"value": w.B * e2e_steps / t_e2e, "unit": UNIT,
+           # only the masked rows cross the host link (read by the GPU from pinned memory)
+           "h2d_bytes_per_step": sb.masked_rows * w.V * w.elem_bytes
+           + h_mask.numel() + h_tok.numel() * 4,
+           "path": "pinned host logits; masked rows read over the host link by "
+                   "fdllm_gather_masked_rows, then fdllm_select; results copied back",
+           "d2h_bytes_per_step": h_tok.numel() * 4 + h_commit.numel() + h_n.numel() * 4
+           + h_mask.numel(),
+           "steps": e2e_steps}
+    del h_logits
+    return out
+
+
+# Rules timed on each small config: the ones its recipe names.
+CONFIG_RULES = {
+    "single_block_b1_l32_bf16": [("profile", 1.0)],
+    "mixed_mask_b8_l32_bf16": [("profile", 0.5), ("profile", 1.0), ("profile", 2.0),
+                               ("factor", 0.5), ("factor", 1.0), ("factor", 2.0),
+                               ("threshold", 0.9)],
+    "tie_groups_b16_l64_fp32": [("profile", 1.0), ("factor", 1.0)],
+}
+CONFIG_BUFFERS = {"single_block_b1_l32_bf16": 32, "mixed_mask_b8_l32_bf16": 8,
+                  "tie_groups_b16_l64_fp32": 4}
+
+
+def run_per_config(args, torch, fd, syn, dev, peak_gbs: float) -> dict:
+    """The other workloads of the metric at N = 1, each as CUDA-graph replays over rotating
+    buffers larger than L2: per rule the time per step, selections/s (batch rows decided per
+    second) and the algorithmic logits GB/s (masked rows x V x element size per step) with
+    its fraction of the measured copy peak; the tie-group workload also reports whether the
+    profile and factor rules took identical decisions (they must, Cor. factor-reduction);
+    the full-sequence workload its step count and per-step latency for both rules; beside
+    each, the CPU oracle on a bounded sample of the same recipe."""
+    stream = torch.cuda.Stream(device=dev)
+    out = {}
+    for name, rules in CONFIG_RULES.items():
+        w = syn.WORKLOADS[name]
+        sb = SelectionBench(torch, fd, syn, w, 1234, CONFIG_BUFFERS[name], dev, stream)
+        per_rule = {}
+        decisions = {}
+        for rule, param in rules:
+            sec, steps, _, _ = sb.time_steps(sb.step_fn(rule, param), args.config_steps, 32)
+            us = sec / steps * 1e6
+            per_rule["%s f=%g" % (rule, param) if rule != "threshold" else
+                     "threshold tau=%g" % param] = {
+                "us_per_step": us, "selections_per_s": w.B / (us * 1e-6),
+                "logits_gbs": sb.alg_bytes / (us * 1e-6) / 1e9,
+                "frac_of_measured_hbm": sb.alg_bytes / (us * 1e-6) / 1e9 / peak_gbs,
+                "steps": steps}
+            m = sb.mask0.clone()
+            with torch.cuda.stream(stream):
+                fd.fdllm_select(sb.bufs[0], m, param, fd.MODES[rule], sb.tok, sb.commit,
+                                sb.n_out, stream=stream)
+            stream.synchronize()
+            decisions[(rule, param)] = (sb.n_out.cpu().clone(), sb.commit.cpu().clone())
+        entry = {"description": w.description, "B": w.B, "L": w.L, "V": w.V,
+                 "dtype": w.dtype, "masked_rows_per_step": sb.masked_rows,
+                 "logits_bytes_per_step": sb.alg_bytes, "l2_policy": sb.l2_policy(),
+                 "rules": per_rule}
+        if name == "tie_groups_b16_l64_fp32":
+            (n_p, c_p), (n_f, c_f) = decisions[("profile", 1.0)], decisions[("factor", 1.0)]
+            entry["identical_decisions_profile_factor"] = bool(torch.equal(n_p, n_f) and
+                                                               torch.equal(c_p, c_f))
+        if not args.skip_cpu_baseline:
+            rule, param = rules[0]
+            entry["cpu_baseline"] = oracle_bounded(name, rule, param, args.config_cpu_s,
+                                                   rows=min(w.B, 2))
+        out[name] = entry
+        del sb
+        torch.cuda.empty_cache()
+    out["full_seq_b16_l1024_fp32"] = run_full_sequence(args, torch, fd, syn, dev, stream)
+    if not args.skip_cpu_baseline:
+        out["full_seq_b16_l1024_fp32"]["cpu_baseline"] = oracle_bounded(
+            "full_seq_b16_l1024_fp32", "profile", 1.0, args.config_cpu_s, rows=1)
+    return out
+
+
+def run_full_sequence(args, torch, fd, syn, dev, stream) -> dict:
+    """The full-sequence workload (B = 16, L = 1024, fp32): selection + commit until no
+    mask remains, profile against factor (f = 1), logits regenerated from (seed, step)
+    before every step outside the timing; each step timed with events on its stream."""
+    import numpy as np
+    w = syn.WORKLOADS["full_seq_b16_l1024_fp32"]
+    res = {"description": w.description, "B": w.B, "L": w.L, "V": w.V, "dtype": w.dtype}
+    logits = syn.make_logits(w, seed=4321, device=dev, step=0)
+    for mode in (fd.PROFILE, fd.FACTOR):  # one untimed call per rule: one-time set-up
+        m0 = torch.from_numpy(syn.make_mask(w, seed=4321)).to(dev)
+        fd.fdllm_select(logits, m0, 1.0, mode, stream=stream)
+    stream.synchronize()
+    del logits
+    for rule in ("profile", "factor"):
+        mask = torch.from_numpy(syn.make_mask(w, seed=4321)).to(dev)
+        tok = torch.full((w.B, w.L), -1, dtype=torch.int32, device=dev)
+        commit = torch.empty((w.B, w.L), dtype=torch.uint8, device=dev)
+        n = torch.empty((w.B,), dtype=torch.int32, device=dev)
+        times, masked = [], []
+        remaining = int(mask.sum().item())
+        while remaining and len(times) < min(w.L + 1, args.full_seq_max_steps):
+            logits = syn.make_logits(w, seed=4321, device=dev, step=len(times))
+            torch.cuda.synchronize()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            fd.fdllm_select(logits, mask, 1.0, fd.MODES[rule], tok, commit, n, stream=stream)
+            e1.record(stream)
+            e1.synchronize()
+            times.append(e0.elapsed_time(e1))
+            masked.append(remaining)
+            del logits
+            remaining = int(mask.sum().item())
+        t = np.array(times)
+        res[rule + " f=1"] = {
+            "steps": len(times), "finished": remaining == 0,
+            "tokens_per_step": float((w.B * w.L - remaining) / max(len(times), 1)),
+            "per_step_ms_median": float(np.median(t)), "per_step_ms_mean": float(t.mean()),
+            "first_step_ms": float(t[0]),
+            "first_step_logits_gbs": masked[0] * w.V * w.elem_bytes / (t[0] * 1e-3) / 1e9,
+            "selections_per_s_median_step": w.B / (float(np.median(t)) * 1e-3)}
+    return res
+
+
+def oracle_bounded(name: str, rule: str, param: float, budget_s: float, rows: int,
+                   step: int = 0) -> dict:
+    """The CPU oracle on `rows` batch rows of a workload's recipe, on all host cores, for
+    about budget_s seconds (at least one step)."""
+    import fdllm_synth as syn
+    import oracle
+    w = syn.WORKLOADS[name]
+    ws = dataclasses.replace(w, B=rows)
+    host = syn.host_bits(syn.make_logits(ws, seed=1234, device="cpu", step=step))
+    mask = syn.make_mask(ws, seed=1234)
+    threads = os.cpu_count() or 1
+    orc = oracle.default()
+    mode = {"profile": oracle.PROFILE, "factor": oracle.FACTOR,
+            "threshold": oracle.THRESHOLD}[rule]
+    t0 = time.perf_counter()
+    done = 0
+    while done == 0 or time.perf_counter() - t0 < budget_s:
+        orc.select(host, mask, mode, param, nthreads=threads)
+        done += 1
+    t = time.perf_counter() - t0
+    return {"value": rows * done / t, "unit": UNIT, "cores": threads, "kind": "oracle",
+            "ms_per_step_of_sample": t / done * 1e3,
+            "sample": "%d batch row(s) of %s (%d masked positions of V=%d), %d steps"
+                      % (rows, name, int(mask.sum()), w.V, done)}
+
+
+def run_lmhead_key(args, torch) -> dict:
+    """The LM-head-fused step at B = 64 and B = 16 for the default line: fused ms per step,
+    the a1 path's PFLOP/s (2 R H V over the fdllm_lmhead_confidence time) against the
+    measured sustained bf16 peak, and cuBLAS's GEMM on the same masked rows alone."""
+    out = {}
+    for b in (64, 16):
+        a = argparse.Namespace(**vars(args))
+        a.lmhead_batch, a.lmhead_vocab = b, 126464
+        a.lmhead_variants = "fused,gemm,cublas_masked"
+        a.lmhead_steps = 20
+        r = run_lmhead(a)
+        sustained = None
+        try:
+            with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as fh:
+                sustained = float(json.load(fh)["bf16_tflops_sustained"])
+        except (OSError, KeyError, ValueError):
+            pass
+        ach = r["roofline"]["achieved"]
+        out["B=%d" % b] = {
+            "masked_rows": r["masked_rows"], "fused_ms": r["ms_per_step"]["fused"],
+            "a1_path_ms": r["ms_per_step"]["fused_confidence_only"],
+            "a1_path_pflops": ach / 1e3 if ach else None,
+            "frac_of_sustained_bf16": ach / sustained if ach and sustained else None,
+            "cublas_gemm_masked_rows_ms": r["ms_per_step"]["cublas_gemm_masked_rows_only"],
+            "selections_per_s_fused": r["selections_per_s_fused"],
+            "clocks": r["clocks"]}
+        torch.cuda.empty_cache()
+    return out
 
 
 # ----------------------------------------------------------------------------- loop mode
@@ -884,8 +1181,12 @@ def run_reference(args, rank: int, world: int) -> dict | None:
 # ----------------------------------------------------------------------------- main
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
-    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--gpus", type=int, default=1,
+                    help="ranks, one GPU each; without torchrun's environment, N > 1 starts "
+                         "them through torch.distributed.run")
     ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--min-steps", type=int, default=1000,
+                    help="the main timed region covers at least this many steps")
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="serving_b64_l32_bf16")
@@ -930,6 +1231,17 @@ def main(argv=None):
                     help="vocabulary size of the LM head (LLaDA-8B: 126464)")
     ap.add_argument("--lmhead-variants", default="fused,gemm,ours,cublas,cublas_masked",
                     help="comma list of: fused, gemm, ours, cublas, cublas_masked")
+    ap.add_argument("--skip-per-config", action="store_true",
+                    help="leave out the other workloads' figures (`per_config`)")
+    ap.add_argument("--skip-lmhead", action="store_true",
+                    help="leave out the LM-head-fused figures (`lmhead`)")
+    ap.add_argument("--config-steps", type=int, default=512,
+                    help="timed steps per rule of each small workload in `per_config`")
+    ap.add_argument("--config-cpu-s", type=float, default=2.0,
+                    help="seconds of oracle time per workload in `per_config`")
+    ap.add_argument("--full-seq-max-steps", type=int, default=1025,
+                    help="bound on the full-sequence loop's steps per rule in `per_config`")
+    argv = sys.argv[1:] if argv is None else list(argv)
     args = ap.parse_args(argv)
     if args.evolving:
         print(json.dumps(run_evolving(args)), flush=True)
@@ -954,9 +1266,14 @@ def main(argv=None):
         print(json.dumps(run_loop(args)), flush=True)
         return
 
+    if "WORLD_SIZE" not in os.environ and args.gpus > 1:
+        # one rank per GPU: start them here, each re-entering this file under torchrun
+        sys.exit(launch_ranks(args.gpus, argv))
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if world != args.gpus:
+        ap.error("--gpus %d but the launcher started %d ranks" % (args.gpus, world))
 
     if args.impl == "reference":
         out = run_reference(args, rank, world)
@@ -970,6 +1287,18 @@ def main(argv=None):
             out["evolving"] = {k: ev[k] for k in ("us_per_step", "selections_per_s",
                                                   "logits_gbs", "period_steps",
                                                   "masked_rows_per_step")}
+        if (out is not None and world == 1 and not args.skip_per_config
+                and args.workload == "serving_b64_l32_bf16"):
+            import torch
+
+            import fdllm_synth as syn
+            import paper_2606_02955_gb300 as fd
+            out["per_config"] = run_per_config(args, torch, fd, syn, torch.device("cuda", 0),
+                                               peak_hbm_gbs()[0])
+        if (out is not None and world == 1 and not args.skip_lmhead
+                and args.workload == "serving_b64_l32_bf16"):
+            import torch
+            out["lmhead"] = run_lmhead_key(args, torch)
         if out is not None and world == 1 and not args.skip_cpu_baseline:
             out["cpu_baseline"] = run_oracle_timed(args, 1, 1, args.cpu_budget_s)
     if out is not None:
