@@ -503,8 +503,9 @@ def run_e2e(args, torch, fd, w, sb) -> dict:
            # only the masked rows cross the host link (read by the GPU from pinned memory)
            "h2d_bytes_per_step": sb.masked_rows * w.V * w.elem_bytes
            + h_mask.numel() + h_tok.numel() * 4,
-           "path": "pinned host logits; masked rows read over the host link by "
-                   "fdllm_gather_masked_rows, then fdllm_select; results copied back",
+           "path": "fdllm_select_host (one C call): pinned host logits, the masked rows "
+                   "read by the GPU over the host link, mask and tokens copied in, the step, "
+                   "results and mask copied back",
            "d2h_bytes_per_step": h_tok.numel() * 4 + h_commit.numel() + h_n.numel() * 4
            + h_mask.numel(),
            "steps": e2e_steps}

@@ -203,6 +203,27 @@ fdllm_status fdllm_select_from_conf(const float *conf, const int32_t *argmax, in
 fdllm_status fdllm_gather_masked_rows(const void *src, void *dst, int dtype, int B, int L, int V,
                                       const uint8_t *mask, void *stream);
 
+/* One selection step end to end on host buffers (Alg. 1's step as fdllm_select computes it;
+ * this entry only moves data around it): the call a host program makes when its logits
+ * are in host memory.  Arguments as in fdllm_select, except:
+ *   logits  [B, L, V] in page-locked host memory (cudaHostAlloc / cudaHostRegister / torch
+ *           pin_memory): the GPU reads the rows of masked positions over the host link and
+ *           nothing else; pageable host memory is copied whole first (slower); device
+ *           memory is read in place.  16-byte aligned.
+ *   mask, out_tokens, out_commit, out_n  host (or device) arrays of fdllm_select's shapes;
+ *           mask is updated in place and out_tokens keeps its values at positions not
+ *           committed, as in fdllm_select.
+ * The library copies mask and out_tokens to a device staging buffer of its own (per device,
+ * grown on demand with cudaMalloc, released by fdllm_release_workspace), runs the step on
+ * `stream` with the library workspace, copies out_tokens, out_commit, out_n and the mask
+ * back and synchronises `stream` before it returns: the results are in place when the call
+ * returns.  Argument errors are reported before anything is enqueued; the same device
+ * errors as fdllm_select (fdllm_device_status).  Not for stream capture (it synchronises).
+ * The paper has no counterpart. */
+fdllm_status fdllm_select_host(const void *logits, int dtype, int B, int L, int V,
+                               uint8_t *mask, double param, int mode, int32_t *out_tokens,
+                               uint8_t *out_commit, int32_t *out_n, void *stream);
+
 /* Step a1 fused with the LM head (the projection that produces the logits, Sec. 3
  * "Notation": p_i = softmax of the logits of position i), then steps a2-a5 as in
  * fdllm_select.  For every masked position the logits x = W h are computed on the tensor

@@ -26,6 +26,7 @@ __all__ = [
     "fdllm_profile_terms", "fdllm_check_bounded_wait", "fdllm_decode_loop", "FORWARD_FN",
     "fdllm_lmhead_select", "fdllm_lmhead_confidence", "fdllm_lmhead_logits",
     "fdllm_gather_masked_rows", "fdllm_decode_loop_lmhead", "fdllm_vocab_reduce",
+    "fdllm_select_host",
 ]
 
 BF16, FP32, FP16 = 0, 1, 2
@@ -92,6 +93,8 @@ def _load():
     lib.fdllm_workspace_status.restype = i
     lib.fdllm_static_status.argtypes = [p]
     lib.fdllm_static_status.restype = i
+    lib.fdllm_select_host.argtypes = [p, i, i, i, i, p, d, i, p, p, p, p]
+    lib.fdllm_select_host.restype = i
     lib.fdllm_release_workspace.argtypes = []
     lib.fdllm_release_workspace.restype = None
     lib.fdllm_status_string.argtypes = [i]
@@ -212,32 +215,32 @@ def fdllm_select(logits: torch.Tensor, mask: torch.Tensor, param: float, mode=PR
 
 
 def _select_from_host(logits, mask, param, mode, out_tokens, out_commit, out_n):
-    dev = torch.device("cuda", torch.cuda.current_device())
-    d_mask = mask.to(dev, non_blocking=True)
-    if logits.is_pinned() and logits.is_contiguous():
-        # Page-locked logits: the GPU reads only the masked rows, straight from host memory.
-        B, L, V = logits.shape
-        d_logits = torch.empty(logits.shape, dtype=logits.dtype, device=dev)
-        _check(_load().fdllm_gather_masked_rows(logits.data_ptr(), d_logits.data_ptr(),
-                                                _dtype_code(logits), B, L, V, d_mask.data_ptr(),
-                                                _stream(None)), "fdllm_gather_masked_rows")
-    else:
-        d_logits = logits.to(dev, non_blocking=True)
-    B, L, _ = logits.shape
-    d_tok = (torch.full((B, L), -1, dtype=torch.int32, device=dev) if out_tokens is None
-             else out_tokens.to(dev, non_blocking=True))
-    t, c, n = fdllm_select(d_logits, d_mask, param, mode, d_tok)
+    """fdllm_select_host: the whole step on host tensors in one library call (the GPU reads
+    only the masked rows of page-locked logits; results and mask copied back)."""
+    B, L, V = logits.shape
+    if not logits.is_contiguous():
+        raise FdllmError(1, "fdllm_select_host: contiguous logits required")
     pin = logits.is_pinned()
-    host = lambda x: torch.empty(x.shape, dtype=x.dtype, pin_memory=pin)
-    h_tok = out_tokens if out_tokens is not None else host(t)
-    h_commit = out_commit if out_commit is not None else host(c)
-    h_n = out_n if out_n is not None else host(n)
-    h_tok.copy_(t, non_blocking=True)
-    h_commit.copy_(c, non_blocking=True)
-    h_n.copy_(n, non_blocking=True)
-    mask.copy_(d_mask, non_blocking=True)
-    torch.cuda.current_stream().synchronize()
-    return h_tok, h_commit, h_n
+
+    def host(t, name, dtype, shape, fill=None):
+        if t is None:
+            t = torch.empty(shape, dtype=dtype, pin_memory=pin)
+            if fill is not None:
+                t.fill_(fill)
+        if t.is_cuda or t.dtype != dtype or tuple(t.shape) != shape or not t.is_contiguous():
+            raise FdllmError(1, "%s: contiguous host %s %s required" % (name, dtype, shape))
+        return t
+
+    mask = host(mask, "mask", torch.uint8, (B, L))
+    out_tokens = host(out_tokens, "out_tokens", torch.int32, (B, L), -1)
+    out_commit = host(out_commit, "out_commit", torch.uint8, (B, L))
+    out_n = host(out_n, "out_n", torch.int32, (B,))
+    st = _load().fdllm_select_host(logits.data_ptr(), _dtype_code(logits), B, L, V,
+                                   mask.data_ptr(), float(param), _mode(mode),
+                                   out_tokens.data_ptr(), out_commit.data_ptr(),
+                                   out_n.data_ptr(), _stream(None))
+    _check(st, "fdllm_select_host")
+    return out_tokens, out_commit, out_n
 
 
 @_on_device

@@ -158,6 +158,8 @@ fdllm_status run_select(const void *logits, int dtype, int B, int L, int V, uint
     return FDLLM_OK;
 }
 
+}  // namespace
+
 fdllm_status check_select_args(const void *logits, int dtype, int B, int L, int V,
                                const uint8_t *mask, double param, int mode,
                                const int32_t *out_tokens, const uint8_t *out_commit,
@@ -174,6 +176,8 @@ fdllm_status check_select_args(const void *logits, int dtype, int B, int L, int 
         return st;
     return plan_fits((int64_t)B * L, (int64_t)V * esize_of(dtype)) ? FDLLM_OK : FDLLM_ERR_ARG;
 }
+
+namespace {
 
 // Reads the sticky status word and, when it is set, zeroes `clear_bytes` from it: for a
 // workspace header the status word and the vocab reduction's work counter, which a launch
@@ -508,6 +512,7 @@ void fdllm_release_workspace(void)
         g_ws[dev].ptr = nullptr;
         g_ws[dev].bytes = 0;
     }
+    release_host_staging(dev);
 }
 
 const char *fdllm_status_string(int status)

@@ -137,6 +137,16 @@ fdllm_status lmhead_select_owned(const void *hidden, const void *w_vocab, int B,
 // compact row count at 8.
 fdllm_status owned_workspace(size_t need, cudaStream_t stream, void **out);
 
+// fdllm_select's argument checks (shape, pointers, mode, param, logits alignment and the
+// unit plan's index range), done before anything is enqueued.
+fdllm_status check_select_args(const void *logits, int dtype, int B, int L, int V,
+                               const uint8_t *mask, double param, int mode,
+                               const int32_t *out_tokens, const uint8_t *out_commit,
+                               const int32_t *out_n);
+
+// Frees fdllm_select_host's device staging buffer of device `dev` (the caller synchronises).
+void release_host_staging(int dev);
+
 // fdllm_select on the library-owned workspace, with programmatic dependent launches
 // switched on or off (the decode loop's graph body falls back to plain stream order where
 // the driver does not accept programmatic edges inside a conditional node).

@@ -81,6 +81,24 @@ def test_select_rejects_bad_shapes(lib, args, want):
     assert st == want
 
 
+@pytest.mark.parametrize("args,want", [
+    ((A16, 0, 0, 32, 1024), ERR_ARG),          # B = 0
+    ((A16, 0, 2, 1025, 1024), ERR_ARG),        # L > 1024
+    ((None, 0, 2, 32, 1024), ERR_ARG),         # null logits
+    ((A2, 0, 2, 32, 1024), ERR_ALIGN),         # logits not 16-byte aligned
+    ((A16, 0, 2, 32, 1001), ERR_ALIGN),        # V * 2 not a multiple of 16
+])
+def test_select_host_rejects_bad_arguments_before_any_copy(lib, args, want):
+    logits, dtype, B, L, V = args
+    lib.fdllm_select_host.argtypes = lib.fdllm_select.argtypes
+    assert lib.fdllm_select_host(logits, dtype, B, L, V, A16, 1.0, 0, A16, A16, A16,
+                                 None) == want
+    assert lib.fdllm_select_host(A16, 0, 2, 32, 1024, None, 1.0, 0, A16, A16, A16,
+                                 None) == ERR_ARG
+    assert lib.fdllm_select_host(A16, 0, 2, 32, 1024, A16, 1.0, 5, A16, A16, A16,
+                                 None) == ERR_ARG
+
+
 def test_select_rejects_bad_mode_param_and_outputs(lib):
     call = lambda mode, param, out=A16, mask=A16: lib.fdllm_select(
         A16, 0, 2, 32, 1024, mask, param, mode, out, A16, A16, None)

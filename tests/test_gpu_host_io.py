@@ -48,3 +48,49 @@ def test_host_select_through_pinned_path_matches_oracle(fd, orc):
     assert np.array_equal(h_mask.numpy()[ok], ref["mask"][ok])
     c = ref["commit"].astype(bool) & ok[:, None]
     assert np.array_equal(tok.numpy()[c], ref["tokens"][c])
+
+
+def _c_select_host(path):
+    import ctypes
+    lib = ctypes.CDLL(path)
+    p, i, d = ctypes.c_void_p, ctypes.c_int, ctypes.c_double
+    lib.fdllm_select_host.argtypes = [p, i, i, i, i, p, d, i, p, p, p, p]
+    lib.fdllm_select_host.restype = i
+    return lib
+
+
+@pytest.mark.parametrize("where", ["pinned", "pageable", "device"])
+@pytest.mark.parametrize("name,mode,param", [("mixed_mask_b8_l32_bf16", 0, 1.0),
+                                             ("target_ties_b16_l64_fp32", 1, 1.0),
+                                             ("target_b8_l32_fp16", 2, 0.9)])
+def test_select_host_through_c_abi_equals_device_select(fd, orc, where, name, mode, param):
+    """fdllm_select_host called through the C interface with host mask and outputs equals
+    fdllm_select on device copies of the same inputs, bit for bit, wherever the logits
+    live; positions it does not commit keep the caller's token values."""
+    lib = _c_select_host(fd.library_path())
+    w = syn.WORKLOADS[name]
+    V = 4096 if where == "pageable" else w.V
+    x = syn.make_logits(w, seed=21, device="cpu", V=V)
+    mask_np = syn.make_mask(w, seed=21)
+    dmask = torch.from_numpy(mask_np.copy()).cuda()
+    ref = fd.fdllm_select(x.cuda(), dmask, param, mode)
+    torch.cuda.synchronize()
+    src = {"pinned": x.pin_memory(), "pageable": x, "device": x.cuda()}[where]
+    dtype = {"bf16": 0, "fp32": 1, "fp16": 2}[w.dtype]
+    h_mask = torch.from_numpy(mask_np.copy()).pin_memory()
+    h_tok = torch.full((w.B, w.L), -7, dtype=torch.int32)
+    h_commit = torch.full((w.B, w.L), 9, dtype=torch.uint8)
+    h_n = torch.full((w.B,), -9, dtype=torch.int32)
+    st = lib.fdllm_select_host(src.data_ptr(), dtype, w.B, w.L, V, h_mask.data_ptr(), param,
+                               mode, h_tok.data_ptr(), h_commit.data_ptr(), h_n.data_ptr(),
+                               torch.cuda.current_stream().cuda_stream)
+    assert st == 0
+    assert np.array_equal(h_n.numpy(), ref[2].cpu().numpy())
+    assert np.array_equal(h_commit.numpy(), ref[1].cpu().numpy())
+    assert np.array_equal(h_mask.numpy(), dmask.cpu().numpy())
+    c = h_commit.numpy().astype(bool)
+    assert np.array_equal(h_tok.numpy()[c], ref[0].cpu().numpy()[c])
+    assert (h_tok.numpy()[~c] == -7).all()
+    oref = orc.select(syn.host_bits(x), mask_np, mode, param)
+    ok = oref["margin"] >= 1e-5
+    assert np.array_equal(h_n.numpy()[ok], oref["n"][ok])
