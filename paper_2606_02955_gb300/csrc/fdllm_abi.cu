@@ -29,7 +29,7 @@ struct Layout {
 Layout layout_for(int64_t rows, int64_t row_bytes)
 {
     Layout l;
-    l.plan = plan_units(row_bytes);
+    l.plan = plan_units(row_bytes, rows);
     l.status = 0;
     l.next_unit = 4;
     l.partials = kAlign;
@@ -53,7 +53,7 @@ fdllm_status check_shape(int B, int L, int V)
 // Unit partial slots are indexed with 32 bits.
 bool plan_fits(int64_t rows, int64_t row_bytes)
 {
-    return rows * (int64_t)plan_units(row_bytes).units_per_row < ((int64_t)1 << 31);
+    return rows * (int64_t)plan_units(row_bytes, rows).units_per_row < ((int64_t)1 << 31);
 }
 
 fdllm_status check_logits(const void *logits, int dtype, int V)

@@ -13,11 +13,19 @@ namespace fdllm {
 
 // ------------------------------------------------------------------ vocab reduction (a1)
 // Each row of logits is cut into units_per_row units of unit_vecs 16-byte vectors (the last
-// unit may be shorter), with units_per_row = ceil(row_bytes / kUnitTargetBytes).  A unit is
-// reduced by one CTA in a fixed order, so a row's result depends only on its bytes.  The
-// CTA streams a unit through a ring of shared-memory chunk buffers.
+// unit may be shorter), with units_per_row = ceil(row_bytes / target).  A unit is reduced by
+// one CTA in a fixed order, so a row's result depends only on its bytes and the call's
+// shape (B * L, V, dtype), which fixes the plan.  The CTA streams a unit through a ring of
+// shared-memory chunk buffers.  The target is 128 KB; a step whose logits, all B * L rows
+// counted, fit in about one wave of such units over the SMs (kSmallStepBytes) takes 64 KB
+// units instead, so that twice as many SMs share its reduction: there the per-SM exp
+// throughput and the first copy's latency, not HBM, set the time.  Smaller units pay for
+// themselves nowhere: a unit must fill the ring (192 KB in flight per SM) to stream at
+// full bandwidth.
 constexpr int kSegQueue = 8;  // unit results queued from math warps to the epilogue warp
 constexpr int64_t kUnitTargetBytes = 131072;
+constexpr int64_t kSmallUnitTargetBytes = 65536;
+constexpr int64_t kSmallStepBytes = 20ll << 20;
 constexpr int kMaxGrid = 1024;
 constexpr int kMaxRows = 65536;
 constexpr int kMaskWords = kMaxRows / 32;
@@ -60,10 +68,12 @@ struct UnitPlan {
 // no unit is empty.
 constexpr int64_t kUnitAlignVecs = 512;
 
-inline UnitPlan plan_units(int64_t row_bytes)
+inline UnitPlan plan_units(int64_t row_bytes, int64_t rows)
 {
     const int64_t vpr = row_bytes / 16;
-    int64_t upr = (row_bytes + kUnitTargetBytes - 1) / kUnitTargetBytes;
+    const int64_t target =
+        rows * row_bytes <= kSmallStepBytes ? kSmallUnitTargetBytes : kUnitTargetBytes;
+    int64_t upr = (row_bytes + target - 1) / target;
     if (upr < 1)
         upr = 1;
     int64_t uv = (vpr + upr - 1) / upr;

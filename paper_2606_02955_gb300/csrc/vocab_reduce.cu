@@ -5,11 +5,13 @@
 // Design (an HBM-bound streaming reduction; no tensor cores):
 //  * Work = the masked rows only.  Every CTA compacts the mask into a bitmap plus word prefix
 //    counts in shared memory and maps the r-th masked row to its global row.
-//  * Each row is cut into fixed units (about 64 KB, see plan_units); the units of all masked
-//    rows form one queue served by an atomic counter, so CTAs that run faster take more
-//    units and the tail is at most one unit.  A unit is reduced by one CTA in a fixed order,
-//    so a row's result depends only on its bytes (identical rows give identical bits, for any
-//    batch composition).
+//  * Each row is cut into fixed units (128 KB, or 64 KB for small steps, see plan_units);
+//    the units of all masked rows form one queue served by an atomic counter, so CTAs that
+//    run faster take more units and the tail is at most one unit.  A producer requests its
+//    next unit before it issues the current one's copies and reads the answer after, so
+//    the counter's round trip overlaps the copies.  A unit is reduced by one CTA in a fixed
+//    order, so a row's result depends only on its bytes and the call's shape (identical rows
+//    give identical bits, for any mask).
 //  * Warp 0 (one lane) streams each unit through a kStages-deep ring of kChunkBytes buffers
 //    with 1-D bulk copies (cp.async.bulk, completion on mbarriers); chunk metadata travels
 //    with the stage.
@@ -395,9 +397,10 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
         if (grow >= 0) {
             first_tried = true;
             if (lane == 0) {
-                // the next unit's request is in flight while the first one streams
-                u_next = gridDim.x + atomicAdd(a.next_unit, 1u);
+                // the first unit's copies go out first; the queue request for the next unit
+                // is then in flight while they stream (its value is read only later)
                 first_issued = issue_unit(blockIdx.x, grow);
+                u_next = gridDim.x + atomicAdd(a.next_unit, 1u);
             }
         }
     } else {
@@ -468,7 +471,7 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
         };
         bool alive = true;  // false once a bounded wait has given up
         if (first_tried) {
-            fetched(u_next);
+            u_next = fetched(u_next);
             alive = first_issued;
         } else if (blockIdx.x < total) {
             // the first unit was not within the producer's scan
@@ -481,12 +484,13 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
             // Then the work queue, which hands out units gridDim.x, gridDim.x + 1, ...
             uint32_t u = u_next;
             while (u < total) {
-                const uint32_t un = fetched(G + atomicAdd(a.next_unit, 1u));
+                // the request for the unit after u is in flight while u's copies are issued
+                const uint32_t raw = atomicAdd(a.next_unit, 1u);
                 if (!issue_unit(u, masked_row(u / upr, sm.bits, sm.pref, nwords))) {
                     alive = false;
                     break;
                 }
-                u = un;
+                u = fetched(G + raw);
             }
         }
         if (alive) {

@@ -197,3 +197,27 @@ def test_masked_rows_only_far_into_the_batch(fd, orc, first_masked):
     flat[rows] = 1
     check_confidence(fd, orc, logits, mask)
     assert check_select(fd, orc, logits, mask, 0, 0.75) <= 2
+
+
+@pytest.mark.parametrize("dtype,L", [("bf16", 8), ("fp32", 96)])
+def test_argmax_ties_on_unit_boundaries(fd, orc, dtype, L):
+    """Equal maxima on both sides of a unit boundary, under both unit plans: a small step
+    (8 bf16 rows, 2 MB: 64 KB units of 32768 logits) and a large one (96 fp32 rows, 48 MB:
+    128 KB units of 32768 logits).  The boundary's left neighbour must win, and the rows'
+    confidences match the oracle."""
+    V = 126464
+    per_unit = 32768  # logits per unit in both plans (64 KB of bf16, 128 KB of fp32)
+    rng = np.random.default_rng(17)
+    x = rng.normal(0, 1, (1, L, V)).astype(np.float32)
+    for j in range(min(L, 3)):
+        edge = per_unit * (j + 1)
+        x[0, j, [edge - 1, edge]] = 25.0            # straddles unit j | j + 1
+        x[0, j, edge + 5] = 25.0
+    x[0, 3, [per_unit, 2 * per_unit - 1]] = 30.0    # both ends of one unit
+    logits = _bf16(x) if dtype == "bf16" else torch.from_numpy(x).cuda()
+    mask_np = np.ones((1, L), np.uint8)
+    conf, tok, rc, rt = check_confidence(fd, orc, logits, mask_np)
+    for j in range(min(L, 3)):
+        assert tok[0, j] == per_unit * (j + 1) - 1
+    assert tok[0, 3] == per_unit
+    check_select(fd, orc, logits, mask_np, PROFILE, 0.75)
