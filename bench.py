@@ -369,9 +369,25 @@ class SelectionBench:
         sec, t0, t1 = time_runner(self.torch, self.stream, run, replays, warm, dist)
         return sec, replays * self.n_buf, (t0, t1), run
 
+    def step_distribution(self, run, replays: int) -> dict:
+        """Per-step µs of `replays` graph replays timed one by one (median, min, max)."""
+        import numpy as np
+        torch, stream = self.torch, self.stream
+        per = []
+        for r in range(replays):
+            a0 = torch.cuda.Event(enable_timing=True)
+            a1 = torch.cuda.Event(enable_timing=True)
+            a0.record(stream)
+            with torch.cuda.stream(stream):
+                run(r)
+            a1.record(stream)
+            a1.synchronize()
+            per.append(a0.elapsed_time(a1) * 1e3 / self.n_buf)
+        return {"median": float(np.median(per)), "min": float(min(per)),
+                "max": float(max(per)), "replays": len(per), "steps_per_replay": self.n_buf}
+
 
 def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
-    import numpy as np
     import torch
 
     import fdllm_synth as syn
@@ -405,16 +421,7 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
     t_k1, _, _, _ = sb.time_steps(k1_only, want, args.warmup, args.no_graph, dist)
     t_k1a, _, _, _ = sb.time_steps(k1_alone, want, args.warmup, args.no_graph, dist)
     # distribution of the step time: replays timed one by one (outside the timed region)
-    per_step_us = []
-    for r in range(min(200, steps // sb.n_buf)):
-        a0 = torch.cuda.Event(enable_timing=True)
-        a1 = torch.cuda.Event(enable_timing=True)
-        a0.record(stream)
-        with torch.cuda.stream(stream):
-            step_run(r)
-        a1.record(stream)
-        a1.synchronize()
-        per_step_us.append(a0.elapsed_time(a1) * 1e3 / sb.n_buf)
+    dist_us = sb.step_distribution(step_run, min(200, steps // sb.n_buf))
     if sampler is not None:
         time.sleep(0.02)
         sampler.stop()
@@ -426,7 +433,7 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
 
     # end to end: the public call with pinned host buffers, copies inside the timed region
     e2e = None
-    if not args.skip_e2e:
+    if not args.skip_e2e and rank == 0:  # the host link is the node's: rank 0 alone
         e2e = run_e2e(args, torch, fd, w, sb)
 
     result = None
@@ -449,10 +456,7 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
                 "logits_gbs_per_step": sb.alg_bytes / (ms_per_step * 1e-3) / 1e9,
                 "positions_per_s": sb.masked_rows * world / (ms_per_step * 1e-3),
                 "steps_requested": args.steps,
-                "step_us_distribution": {
-                    "median": float(np.median(per_step_us)), "min": float(min(per_step_us)),
-                    "max": float(max(per_step_us)), "replays": len(per_step_us),
-                    "steps_per_replay": sb.n_buf},
+                "step_us_distribution": dist_us,
                 "l2_policy": sb.l2_policy(),
                 "cuda_graph": not args.no_graph,
                 "parallelism": "dp%d (independent batches, no collective)" % world,
@@ -541,14 +545,15 @@ def run_per_config(args, torch, fd, syn, dev, peak_gbs: float) -> dict:
         per_rule = {}
         decisions = {}
         for rule, param in rules:
-            sec, steps, _, _ = sb.time_steps(sb.step_fn(rule, param), args.config_steps, 32)
+            sec, steps, _, run = sb.time_steps(sb.step_fn(rule, param), args.config_steps, 32)
             us = sec / steps * 1e6
             per_rule["%s f=%g" % (rule, param) if rule != "threshold" else
                      "threshold tau=%g" % param] = {
                 "us_per_step": us, "selections_per_s": w.B / (us * 1e-6),
                 "logits_gbs": sb.alg_bytes / (us * 1e-6) / 1e9,
                 "frac_of_measured_hbm": sb.alg_bytes / (us * 1e-6) / 1e9 / peak_gbs,
-                "steps": steps}
+                "steps": steps,
+                "step_us_distribution": sb.step_distribution(run, max(8, min(100, steps // sb.n_buf)))}
             m = sb.mask0.clone()
             with torch.cuda.stream(stream):
                 fd.fdllm_select(sb.bufs[0], m, param, fd.MODES[rule], sb.tok, sb.commit,
