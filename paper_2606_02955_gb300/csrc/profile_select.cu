@@ -159,20 +159,30 @@ __global__ void __launch_bounds__(T) profile_select_kernel(const ProfileSelectAr
     // partials, or read from the given arrays.
     // Launched as a programmatic dependent: whatever produced the unit partials or the
     // confidences (and the mask) has completed and its writes are visible past this wait.
+    // As in the warp kernel: after the vocab reduction, the mask byte and the allowance are
+    // loaded before the launch wait (their writers completed before the reduction passed
+    // its own wait); the unit partials or confidences and the status word after it, all
+    // issued before any is used.
+    const bool in_row = t < L;
+    const bool early = a.partials != nullptr;
+    uint8_t mask_byte = 0;
+    float eta = (float)a.eta;
+    auto load_row_inputs = [&]() {
+        mask_byte = in_row ? __ldcg(a.mask + base + t) : (uint8_t)0;
+        if (a.mode == kModeRobust && a.eta_pos != nullptr && in_row)
+            eta = __ldcg(a.eta_pos + base + t);
+    };
+    if (early)
+        load_row_inputs();
     pdl_wait();
     if (threadIdx.x == 0)
         pdl_launch_dependents();  // a following vocab reduction may start its prologue
-    // The mask byte, the position's (c, x_hat), its allowance and the status word are loaded
-    // together (one memory round trip on the critical path of a decode step instead of
-    // three); an unmasked position's values are in-bounds leftovers and are discarded.
-    const bool dev_err = a.status != nullptr && *((volatile const uint32_t *)a.status) != 0;
-    const bool in_row = t < L;
-    const bool masked = in_row && a.mask[base + t] != 0;
+    if (!early)
+        load_row_inputs();
+    const bool dev_err = a.status != nullptr && __ldcg(a.status) != 0;
+    const bool masked = mask_byte != 0;
     float c = 0.0f;
     int32_t tok = -1;
-    const float eta = a.mode == kModeRobust && a.eta_pos != nullptr && in_row
-                          ? a.eta_pos[base + t]
-                          : (float)a.eta;
     if (in_row) {
         if (a.partials != nullptr) {
             combine_position(a.partials + (base + t) * a.units_per_row, a.units_per_row, c,
@@ -242,17 +252,31 @@ __global__ void __launch_bounds__(32) profile_select_warp_kernel(const ProfileSe
     const int L = a.L;
     const int64_t base = (int64_t)blockIdx.x * L;
 
-    pdl_wait();  // the producer of the partials or confidences (and the mask) has completed
+    // After the vocab reduction (partials given), the mask byte and the allowance are loaded
+    // before the launch wait: this kernel starts only once the reduction has passed its own
+    // launch wait, so whatever wrote them has completed, and the reduction writes neither.
+    // The unit partials and the status word are the reduction's output: loaded after it.
+    // Otherwise (confidences given) everything is loaded after the wait.
+    const bool in_row = t < L;
+    const bool early = a.partials != nullptr;
+    uint8_t mask_byte = 0;
+    float eta = (float)a.eta;
+    auto load_row_inputs = [&]() {
+        mask_byte = in_row ? __ldcg(a.mask + base + t) : (uint8_t)0;
+        if (a.mode == kModeRobust && a.eta_pos != nullptr && in_row)
+            eta = __ldcg(a.eta_pos + base + t);
+    };
+    if (early)
+        load_row_inputs();
+    pdl_wait();  // the producer of the partials or confidences has completed
     if (t == 0)
         pdl_launch_dependents();  // a following vocab reduction may start its prologue
-    // Every load of the row is issued here, before any of them is used (one memory round
-    // trip): status word, mask byte, allowance, and the position's unit partials or (c, x_hat).
-    const bool in_row = t < L;
+    if (!early)
+        load_row_inputs();
+    // The rest of the row's loads are issued here, before any of them is used (one memory
+    // round trip): status word and the position's unit partials or (c, x_hat).
     const uint32_t status = a.status != nullptr ? __ldcg(a.status) : 0u;
-    const bool masked = in_row && __ldcg(a.mask + base + t) != 0;
-    const float eta = a.mode == kModeRobust && a.eta_pos != nullptr && in_row
-                          ? __ldcg(a.eta_pos + base + t)
-                          : (float)a.eta;
+    const bool masked = mask_byte != 0;
     float c = 0.0f;
     int32_t tok = -1;
     if (in_row) {
