@@ -17,8 +17,11 @@ object times the vocabulary reduction by itself (fdllm_vocab_reduce) against the
 copy bandwidth.  At N = 1 the line also carries, measured after the timed region:
 `evolving` (the serving workload with masks evolving from step to step until every row has
 finished), `per_config` (the single-block, mixed-mask, tie-group and full-sequence
-workloads, each beside the oracle on a bounded sample) and `lmhead` (the LM-head-fused step
-at B = 64 and 16); --skip-evolving, --skip-per-config and --skip-lmhead leave them out.
+workloads, each beside the oracle on a bounded sample, and the calibration-robust rule on
+the serving workload), `lmhead` (the LM-head-fused step at B = 64 and 16) and `decode_loop`
+(a 256-token generation of 8 sequences in blocks of 32 through the device-resident loop and
+a host-driven one: NFE per block, tokens per step, tokens/s); --skip-evolving,
+--skip-per-config, --skip-lmhead and --skip-decode-loop leave them out.
 Other measurements, each one JSON line:
   --evolving      masks evolving from step to step until every row has finished
   --loop          the full-sequence workload (B = 16, L = 1024) selected until no mask remains
@@ -575,6 +578,22 @@ def run_per_config(args, torch, fd, syn, dev, peak_gbs: float) -> dict:
         out[name] = entry
         del sb
         torch.cuda.empty_cache()
+    # the calibration-robust rule (App. C) on the serving workload, uniform allowance
+    w = syn.WORKLOADS["serving_b64_l32_bf16"]
+    sb = SelectionBench(torch, fd, syn, w, 1234, 8, dev, stream)
+    timed_rules = {}
+    for rule in ("profile", "robust"):
+        sec, steps, _, _ = sb.time_steps(sb.step_fn(rule, 1.0, args.eta), 1000, 32)
+        timed_rules[rule] = sec / steps * 1e6
+    out["serving_b64_l32_bf16_robust"] = {
+        "description": "the serving workload under the calibration-robust profile rule "
+                       "(lower confidences max(0, c - eta), eta = %g) beside the plain rule, "
+                       "same buffers, 1000 steps each" % args.eta,
+        "robust_us_per_step": timed_rules["robust"],
+        "profile_us_per_step": timed_rules["profile"],
+        "robust_selections_per_s": w.B / (timed_rules["robust"] * 1e-6)}
+    del sb
+    torch.cuda.empty_cache()
     out["full_seq_b16_l1024_fp32"] = run_full_sequence(args, torch, fd, syn, dev, stream)
     if not args.skip_cpu_baseline:
         out["full_seq_b16_l1024_fp32"]["cpu_baseline"] = oracle_bounded(
@@ -1246,6 +1265,8 @@ def main(argv=None):
                     help="leave out the other workloads' figures (`per_config`)")
     ap.add_argument("--skip-lmhead", action="store_true",
                     help="leave out the LM-head-fused figures (`lmhead`)")
+    ap.add_argument("--skip-decode-loop", action="store_true",
+                    help="leave out the device-resident decode loop's figures (`decode_loop`)")
     ap.add_argument("--config-steps", type=int, default=512,
                     help="timed steps per rule of each small workload in `per_config`")
     ap.add_argument("--config-cpu-s", type=float, default=2.0,
@@ -1310,6 +1331,15 @@ def main(argv=None):
                 and args.workload == "serving_b64_l32_bf16"):
             import torch
             out["lmhead"] = run_lmhead_key(args, torch)
+        if (out is not None and world == 1 and not args.skip_decode_loop
+                and args.workload == "serving_b64_l32_bf16"):
+            a = argparse.Namespace(**vars(args))
+            a.gen_len, a.loop_lmhead, a.repeats, a.warmup_loops = 256, False, 3, 1
+            a.mode, a.param = "profile", 1.0
+            dl = run_decode_loop(a)
+            out["decode_loop"] = {k: dl[k] for k in (
+                "workload", "steps", "nfe_per_block", "tokens_per_step", "device_loop",
+                "host_loop", "host_round_trip_us_per_step", "identical_decisions")}
         if out is not None and world == 1 and not args.skip_cpu_baseline:
             out["cpu_baseline"] = run_oracle_timed(args, 1, 1, args.cpu_budget_s)
     if out is not None:

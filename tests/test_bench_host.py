@@ -131,6 +131,11 @@ def test_main_arm_prints_one_contract_line():
     assert pc["tie_groups_b16_l64_fp32"]["identical_decisions_profile_factor"] is True
     fs = pc["full_seq_b16_l1024_fp32"]
     assert fs["profile f=1"]["steps"] == 3 and fs["factor f=1"]["per_step_ms_median"] > 0
+    rb = pc["serving_b64_l32_bf16_robust"]
+    assert rb["robust_us_per_step"] > 0 and rb["profile_us_per_step"] > 0
+    dl = d["decode_loop"]
+    assert dl["identical_decisions"] is True and dl["steps"] == sum(dl["nfe_per_block"])
+    assert dl["device_loop"]["tokens_per_s"] > 0
     for b in ("B=64", "B=16"):
         lm = d["lmhead"][b]
         assert lm["fused_ms"] > 0 and 0 < lm["frac_of_burst_bf16"] < 1.3
