@@ -221,3 +221,38 @@ def test_argmax_ties_on_unit_boundaries(fd, orc, dtype, L):
         assert tok[0, j] == per_unit * (j + 1) - 1
     assert tok[0, 3] == per_unit
     check_select(fd, orc, logits, mask_np, PROFILE, 0.75)
+
+
+@pytest.mark.parametrize("B,L,offset,density", [
+    (5, 7, 1, 0.6),       # 35 rows: a partial mask word, mask pointer not 16-byte aligned
+    (5, 7, 0, 0.6),
+    (128, 32, 0, 0.05),   # 4096 rows, sparse: most first units lie beyond the producer's scan
+    (128, 32, 3, 0.5),
+    (4097, 1, 0, 0.1),
+    (64, 64, 0, 1.0),
+])
+def test_mask_reading_unaligned_and_partial_words(fd, orc, B, L, offset, density):
+    """Masks at any byte offset (the reduction and the selection read them byte by byte),
+    row counts that are not a multiple of 32, and sparse masks whose masked rows lie beyond
+    the producer's first-unit scan, against the oracle."""
+    V = 1024
+    w = syn.Workload("mask_edge", B, L, V, "bf16", 1.0, "target", 0.3, 4.0)
+    logits = syn.make_logits(w, seed=B * 7 + L + offset, device="cuda")
+    rng = np.random.default_rng(B + L + offset)
+    mask_np = (rng.random((B, L)) < density).astype(np.uint8)
+    store = torch.zeros(B * L + 64, dtype=torch.uint8, device="cuda")
+    mask = store[offset:offset + B * L].view(B, L)
+    mask.copy_(torch.from_numpy(mask_np))
+    assert (mask.data_ptr() % 16 == 0) == (offset == 0)
+    conf, tok = fd.fdllm_confidence(logits, mask)
+    torch.cuda.synchronize()
+    rc, rt, _ = orc.confidence(syn.host_bits(logits), mask_np)
+    mk = mask_np.astype(bool)
+    assert np.array_equal(tok.cpu().numpy()[mk], rt[mk])
+    assert (np.abs(conf.cpu().numpy()[mk] - rc[mk]) / rc[mk]).max() <= 1e-5
+    out = fd.fdllm_select(logits, mask, 0.75, PROFILE)
+    torch.cuda.synchronize()
+    ref = orc.select(syn.host_bits(logits), mask_np, PROFILE, 0.75)
+    ok = ref["margin"] >= 1e-5
+    assert np.array_equal(out[2].cpu().numpy()[ok], ref["n"][ok])
+    assert np.array_equal(mask.cpu().numpy()[ok], ref["mask"][ok])
