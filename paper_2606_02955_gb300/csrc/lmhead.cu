@@ -78,7 +78,8 @@ struct GemmArgs {
     int32_t V;
     int32_t n_tiles;           // partials per row: ceil(V / BN), or the slab variant's grid
     int32_t k_blocks;          // ceil(H / BK)
-    int32_t n_groups;          // slab variant: ceil(V / 64)
+    int32_t slab_tiles;        // slab variant: vocabulary tiles, ceil(V / slab_h)
+    int32_t slab_h;            // slab variant: W rows per tile (a multiple of 8, <= 128)
     UnitPartial *partials;     // kReduce: [R][n_tiles]
     float *logits;             // kStore: [B * L][V] fp32, written at masked rows
     uint32_t *status;          // sticky device error bits
@@ -406,21 +407,21 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // ----------------------------------------------------------------------------- slab variant
 // For at most kSlabRows masked rows the operands swap roles: W is the MMA's A operand (M =
-// 128 vocabulary entries, TMEM lane = entry) and the packed rows are its B operand (N = 32,
-// TMEM column = row).  CTA c of P owns the 64-entry groups c, c + P, c + 2P, ... of the G
-// groups (LLaDA's 1976 groups are 13 per SM on 152 SMs, an even split) and streams them as
-// tiles of two groups, groups c + 2jP and c + (2j + 1)P, the last tile possibly one; so the
-// CTAs read W in a window that moves through it, as a grid of one tile per CTA would.
-// The padded row tile costs 4 KB per stage instead of 16 KB, so 10 stages (160 KB of W)
-// are in flight per SM.  Each epilogue thread keeps, for every row, a running maximum, sum
+// 128 TMEM lanes, lane = vocabulary entry) and the packed rows are its B operand (N = 32,
+// TMEM column = row).  The vocabulary is cut into tiles of h entries (one TMA box of h W
+// rows, h a multiple of 8 up to 128, chosen by the host so that the busiest CTA streams as
+// few W rows as possible: LLaDA's V = 126464 is 1216 tiles of 104, eight per SM on 152
+// SMs); CTA c of P owns the tiles c, c + P, c + 2P, ..., so the CTAs read W in a window that
+// moves through it.  The MMA always spans 128 lanes; lanes h..127 hold sums of stale shared
+// memory that the epilogue skips.  The padded row tile costs 4 KB per stage instead of
+// 16 KB, so 11 stages (143 KB of W at h = 104) are in flight per SM.  Each epilogue thread keeps, for every row, a running maximum, sum
 // of exp relative to it and first index over its own entry of each tile; after the last
 // tile the 128 threads' states are folded per row (a transposing butterfly in each warp,
 // then the four warps in order) into one partial per (row, CTA).
 constexpr int kSlabRows = 32;
-constexpr int kGroup = 64;                               // W rows per TMA box
-constexpr int kSlabABytes = BM * BK * 2;                 // two groups
+constexpr int kSlabABytes = BM * BK * 2;                 // 128 lanes; a tile fills h rows
 constexpr int kSlabBBytes = kSlabRows * BK * 2;
-constexpr int kSlabStages = 10;
+constexpr int kSlabStages = 11;
 constexpr int kSlabAccs = 4;                             // accumulators of 32 columns
 constexpr uint32_t kSlabTmemCols = 128;
 constexpr size_t kSlabSmemBytes =
@@ -487,9 +488,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     pdl_wait();  // the packed rows and their count are complete
 
     const int R = *a.row_count;  // <= kSlabRows: the host takes this variant only then
-    const int64_t G = a.n_groups, P = gridDim.x, c = blockIdx.x;
-    const int64_t n_g = c < G ? (G - c + P - 1) / P : 0;   // groups of this CTA
-    const int n_t = R > 0 ? (int)((n_g + 1) / 2) : 0;      // tiles of (up to) two groups
+    const int64_t NT = a.slab_tiles, P = gridDim.x, c = blockIdx.x;
+    const int h = a.slab_h;
+    const int n_t = R > 0 && c < NT ? (int)((NT - c + P - 1) / P) : 0;  // tiles of this CTA
 
     if (warp == 0) {
         if (lane == 0) {
@@ -501,22 +502,18 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int i = 0; i < kSlabStages; ++i)
                 used[i] = false;
             bool ok = true;
+            // a box's bytes count in full, the part beyond V zero-filled
+            const uint32_t bytes = (uint32_t)(h * BK * 2) + kSlabBBytes;
             for (int t = 0; ok && t < n_t; ++t) {
-                const int64_t ga = c + 2 * t * P, gb = ga + P;
-                const bool two = 2 * t + 1 < n_g;
-                const uint32_t bytes = (two ? 2u : 1u) * (kGroup * BK * 2) + kSlabBBytes;
+                const int64_t T = c + (int64_t)t * P;
                 for (int kb = 0; kb < a.k_blocks; ++kb) {
                     if (!wait_or_abort(&empty[s], ph ^ 1u, a.status, abort_flag)) {
                         ok = false;
                         break;
                     }
                     mbar_arrive_expect_tx(&full[s], bytes);
-                    uint8_t *dst = sA + s * kSlabABytes;
-                    tc::tma_load_2d_hint(dst, &map_w, kb * BK, (int32_t)(ga * kGroup),
+                    tc::tma_load_2d_hint(sA + s * kSlabABytes, &map_w, kb * BK, (int32_t)(T * h),
                                          &full[s], pol);
-                    if (two)
-                        tc::tma_load_2d_hint(dst + kGroup * BK * 2, &map_w, kb * BK,
-                                             (int32_t)(gb * kGroup), &full[s], pol);
                     tc::tma_load_2d(sB + s * kSlabBBytes, &map_h, kb * BK, 0, &full[s]);
                     used[s] = true;
                     last_ph[s] = ph;
@@ -549,8 +546,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                         break;
                     }
                     tc::fence_after_sync();
-                    // A single-group tile leaves the second half of the A stage stale: those
-                    // 64 TMEM lanes hold meaningless sums that the epilogue skips.
+                    // Rows h..127 of the A stage are stale: those TMEM lanes hold
+                    // meaningless sums that the epilogue skips.
                     const uint64_t ad = tc::sw128_kmajor_desc(sA + s * kSlabABytes);
                     const uint64_t bd = tc::sw128_kmajor_desc(sB + s * kSlabBBytes);
 #pragma unroll
@@ -599,10 +596,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             __syncwarp();
             if (lane == 0)
                 mbar_arrive(&tempty[acc]);
-            // lanes 0-63 of the tile: group c + 2tP; lanes 64-127: group c + (2t + 1)P
-            const int64_t g = c + (2 * t + (q >> 1)) * P;
-            const int64_t ent = g * kGroup + (q & 1) * 32 + lane;
-            if (2 * t + (q >> 1) >= n_g || ent >= a.V)
+            // lane q * 32 + lane of tile c + tP: vocabulary entry (c + tP) * h + q * 32 + lane
+            const int in_tile = q * 32 + lane;
+            const int64_t ent = (c + (int64_t)t * P) * h + in_tile;
+            if (in_tile >= h || ent >= a.V)
                 continue;
             if (EPI == kStore) {
 #pragma unroll
@@ -924,19 +921,50 @@ fdllm_status check_lmhead(const void *hidden, const void *w, int B, int L, int H
 int sm_count();
 int choose_bn(int64_t rows, int V, bool pair);
 
-// Rows of W per CTA on the longest-running SM: for the slab variant ceil(G / P) groups of 64;
-// for the tile variants (one row tile) whole waves of vocabulary tiles times their width.
-// Measured on LLaDA-sized heads, the slab variant is faster when each CTA's group count is
-// even and its rows do not exceed the tile variant's; with an odd count every CTA ends on a
-// one-group tile, half as many W bytes in flight, and the tile variant is faster.
+// The slab variant's tile height: the multiple of 8 in [96, 128] that minimises the W rows
+// of the busiest CTA, ceil(ceil(V / h) / P) * h with P = min(tiles, SMs); ties go to the
+// taller tile (fewer, larger copies).  Heights below 96 would put too few W bytes in each
+// stage to keep the stream going.
+int slab_height(int V)
+{
+    const int64_t sms = sm_count();
+    int best = 128;
+    int64_t best_rows = -1;
+    for (int h = 128; h >= 96; h -= 8) {
+        const int64_t tiles = ((int64_t)V + h - 1) / h;
+        const int64_t P = tiles < sms ? tiles : sms;
+        const int64_t rows = (tiles + P - 1) / P * h;
+        if (best_rows < 0 || rows < best_rows) {
+            best = h;
+            best_rows = rows;
+        }
+    }
+    return best;
+}
+
+// The slab variant's grid: one CTA per SM, or one per tile if there are fewer.
+int slab_grid(int V)
+{
+    const int64_t h = slab_height(V);
+    const int64_t tiles = ((int64_t)V + h - 1) / h;
+    return (int)(tiles < sm_count() ? tiles : sm_count());
+}
+
+// Rows of W per CTA on the longest-running SM, for the slab variant (whole tiles of its
+// height) against the tile variant (one row tile: whole waves of vocabulary tiles times
+// their width).  The slab variant keeps more W in flight per SM (11 stages of h rows against
+// the tile variant's 5 of its width); measured on LLaDA-sized heads, it is faster when its
+// busiest CTA streams no more rows.
 bool slab_preferred(int V)
 {
     const int64_t sms = sm_count();
-    const int64_t groups = ((int64_t)V + kGroup - 1) / kGroup;
-    const int64_t per_cta = (groups + sms - 1) / sms;
+    const int64_t h = slab_height(V);
+    const int64_t tiles = ((int64_t)V + h - 1) / h;
+    const int64_t P = tiles < sms ? tiles : sms;
+    const int64_t slab_rows = (tiles + P - 1) / P * h;
     const int bn = choose_bn(1, V, false);
     const int64_t tile_rows = ((V + bn - 1) / bn + sms - 1) / sms * bn;
-    return per_cta % 2 == 0 && per_cta * kGroup <= tile_rows;
+    return slab_rows <= tile_rows;
 }
 
 // The GEMM variant: for at most kSlabRows rows the slab variant where slab_preferred; else
@@ -1053,13 +1081,6 @@ cudaError_t launch_gemm_mode(const CUtensorMap &mh, const CUtensorMap &mw, const
                      : launch_gemm_cfg<EPI, MODE, 256>(mh, mw, g, stream);
 }
 
-// The slab variant's grid: one CTA per SM, or one per 64-entry group if there are fewer.
-int slab_grid(int V)
-{
-    const int64_t groups = ((int64_t)V + kGroup - 1) / kGroup;
-    return (int)(groups < sm_count() ? groups : sm_count());
-}
-
 template <int EPI>
 cudaError_t launch_slab(const CUtensorMap &mh, const CUtensorMap &mw, const GemmArgs &g,
                         cudaStream_t stream)
@@ -1108,7 +1129,7 @@ fdllm_status run_lmhead(const void *hidden, const void *w, int B, int L, int H, 
 {
     const int64_t rows = (int64_t)B * L;
     const int mode = gemm_mode(rows, V);
-    const int bn = mode == kSlab ? kGroup : choose_bn(rows, V, mode == kPair);
+    const int bn = mode == kSlab ? slab_height(V) : choose_bn(rows, V, mode == kPair);
     // partials per row: one per vocabulary tile, or one per CTA of the slab variant
     const int n_tiles = mode == kSlab ? slab_grid(V) : (V + bn - 1) / bn;
     const LmLayout lay = lm_layout(rows, H, n_tiles);
@@ -1139,7 +1160,8 @@ fdllm_status run_lmhead(const void *hidden, const void *w, int B, int L, int H, 
     g.V = V;
     g.n_tiles = n_tiles;
     g.k_blocks = (H + BK - 1) / BK;
-    g.n_groups = (V + kGroup - 1) / kGroup;
+    g.slab_h = mode == kSlab ? bn : 0;
+    g.slab_tiles = mode == kSlab ? (V + bn - 1) / bn : 0;
     g.partials = reinterpret_cast<UnitPartial *>(ws + lay.partials);
     g.logits = out_logits;
     g.status = reinterpret_cast<uint32_t *>(ws);

@@ -231,20 +231,24 @@ def test_hidden_sizes_below_one_stage(fd, orc, H):
 
 # ----------------------------------------------------------------------------- slab variant
 SLAB_SHAPES = [
-    # (B, L, H, V) with B * L <= 32: ragged 64-entry groups, CTAs with an odd number of
-    # groups (a single-group last tile), V below one group, LLaDA's head.
+    # (B, L, H, V) with B * L <= 32: a ragged last tile, V below one tile, tiles of every
+    # height the host picks on 152 SMs (96 for small V, 112 at V = 34048, 120 at 36480, 104
+    # for LLaDA's head: 1216 tiles, eight per CTA), and the head itself.
     (1, 32, 256, 5000),
     (1, 3, 72, 40),
     (2, 8, 128, 300),
     (1, 17, 512, 20000),
     (4, 8, 64, 129),
+    (1, 20, 128, 34048),
+    (2, 7, 192, 36480),
     (1, 32, 4096, syn.LLADA_VOCAB),
 ]
 
 
 @pytest.fixture
 def slab(monkeypatch):
-    """The swapped-operand variant (W as the M = 128 side, one vocabulary slab per CTA)."""
+    """The swapped-operand variant (W as the M = 128 side, vocabulary tiles of up to 128
+    entries dealt round-robin over the CTAs)."""
     monkeypatch.setenv("FDLLM_LMHEAD_GEMM", "slab")
 
 
@@ -355,8 +359,8 @@ def test_slab_agrees_with_the_tile_variant(fd, orc, monkeypatch):
 
 
 def test_automatic_tiling_small_batch(fd, orc, monkeypatch):
-    """No variant forced: at most 32 rows with V = 19456 (304 groups of 64, two per CTA on
-    152 SMs) is where the host takes the slab variant by itself; any other SM count takes
+    """No variant forced: at most 32 rows with V = 19456 (152 tiles of 128, one per CTA on
+    152 SMs) is where the host takes the slab variant by itself; any other SM count may take
     another variant, which must agree with the oracle all the same."""
     monkeypatch.delenv("FDLLM_LMHEAD_GEMM", raising=False)
     monkeypatch.delenv("FDLLM_LMHEAD_BN", raising=False)
