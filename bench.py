@@ -672,12 +672,12 @@ def oracle_bounded(name: str, rule: str, param: float, budget_s: float, rows: in
 
 
 def run_lmhead_key(args, torch) -> dict:
-    """The LM-head-fused step at B = 64 and B = 16 for the default line: fused ms per step,
+    """The LM-head-fused step at B = 64, 16 and 1 for the default line: fused ms per step,
     the a1 path's PFLOP/s (2 R H V over the fdllm_lmhead_confidence time) against the
     measured bf16 burst peak (and the sustained one), and cuBLAS's GEMM on the same masked
     rows alone."""
     out = {}
-    for b in (64, 16):
+    for b in (64, 16, 1):
         a = argparse.Namespace(**vars(args))
         a.lmhead_batch, a.lmhead_vocab = b, 126464
         a.lmhead_variants = "fused,gemm,cublas_masked"
