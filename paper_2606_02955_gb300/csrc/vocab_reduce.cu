@@ -268,6 +268,18 @@ __device__ __forceinline__ int64_t masked_row(uint32_t r, const uint32_t *bits,
     return (int64_t)lo * 32 + bit;
 }
 
+// Bit j of the result = byte j of x is nonzero (j = 0..3): each byte folded onto its bit 0,
+// then the four bits gathered by one multiply (the partial products land on distinct bits
+// below 24, so bits 24-27 carry no interference).
+__device__ __forceinline__ uint32_t nonzero_bytes4(uint32_t x)
+{
+    uint32_t t = x | (x >> 4);
+    t |= t >> 2;
+    t |= t >> 1;
+    t &= 0x01010101u;
+    return ((t * 0x01020408u) >> 24) & 0xFu;
+}
+
 struct ChunkMeta {
     uint32_t n;         // vectors in the chunk; 0 marks the end of the CTA's work
     uint32_t vec_base;  // row-relative index of the chunk's first vector
@@ -372,28 +384,38 @@ __global__ void __launch_bounds__((NW + 2) * 32, 1) vocab_reduce_kernel(const Vo
         if (EVICT)
             policy = make_evict_first_policy();
         const uint32_t kth = blockIdx.x / upr;
-        uint32_t seen = 0;
         int64_t grow = -1;
-        // A bounded scan (two memory round trips at most): with few masked rows among the
-        // first kScanRows, the first unit is issued after the compaction instead (below),
-        // which the other warps finish in about the same time.
+        // A bounded scan of the first kScanRows rows in one memory round trip: lane l reads
+        // rows [16 l, 16 l + 16) (one 16-byte load where the mask allows, byte loads at a
+        // ragged end or an unaligned mask), then a warp scan of the per-lane counts finds the
+        // kth masked row.  With fewer masked rows there, the first unit is issued after the
+        // compaction instead (below), which the other warps finish in about the same time.
         constexpr int64_t kScanRows = 512;
         const int64_t scan_end = a.rows < kScanRows ? a.rows : kScanRows;
-        for (int64_t base = 0; base < scan_end && grow < 0; base += 8 * 32) {
-            uint32_t ball[8];
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                const int64_t r = base + i * 32 + lane;
-                ball[i] = __ballot_sync(0xFFFFFFFFu, r < scan_end && a.mask[r] != 0);
-            }
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                const uint32_t c = (uint32_t)__popc(ball[i]);
-                if (grow < 0 && seen + c > kth)
-                    grow = base + i * 32 + (int64_t)__fns(ball[i], 0, (int)(kth - seen) + 1);
-                seen += c;
-            }
+        const int64_t r0 = (int64_t)lane * 16;
+        uint32_t bits16 = 0;
+        if ((reinterpret_cast<uintptr_t>(a.mask) & 15u) == 0 && r0 + 16 <= scan_end) {
+            const uint4 v = __ldcg(reinterpret_cast<const uint4 *>(a.mask + r0));
+            bits16 = nonzero_bytes4(v.x) | (nonzero_bytes4(v.y) << 4) |
+                     (nonzero_bytes4(v.z) << 8) | (nonzero_bytes4(v.w) << 12);
+        } else {
+            for (int j = 0; j < 16 && r0 + j < scan_end; ++j)
+                bits16 |= (a.mask[r0 + j] != 0 ? 1u : 0u) << j;
         }
+        const uint32_t cnt = (uint32_t)__popc(bits16);
+        uint32_t incl = cnt;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t t = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+            if (lane >= o)
+                incl += t;
+        }
+        const bool here = kth >= incl - cnt && kth < incl;
+        const uint32_t who = __ballot_sync(0xFFFFFFFFu, here);
+        const int64_t cand =
+            here ? r0 + (int64_t)__fns(bits16, 0, (int)(kth - (incl - cnt)) + 1) : (int64_t)-1;
+        if (who != 0u)
+            grow = __shfl_sync(0xFFFFFFFFu, cand, __ffs(who) - 1);
         if (grow >= 0) {
             first_tried = true;
             if (lane == 0) {
