@@ -601,17 +601,19 @@ def run_per_config(args, torch, fd, syn, dev, peak_gbs: float) -> dict:
     return out
 
 
-def run_full_sequence(args, torch, fd, syn, dev, stream) -> dict:
-    """The full-sequence workload (B = 16, L = 1024, fp32): selection + commit until no
-    mask remains, profile against factor (f = 1), logits regenerated from (seed, step)
-    before every step outside the timing; each step timed with events on its stream."""
+def run_full_sequence(args, torch, fd, syn, dev, stream,
+                      name: str = "full_seq_b16_l1024_fp32", param: float = 1.0) -> dict:
+    """A workload's selection + commit repeated until no mask remains (by default the
+    full-sequence workload, B = 16, L = 1024, fp32), profile against factor at f = param,
+    logits regenerated from (seed, step) before every step outside the timing; each step
+    timed with events on its stream."""
     import numpy as np
-    w = syn.WORKLOADS["full_seq_b16_l1024_fp32"]
+    w = syn.WORKLOADS[name]
     res = {"description": w.description, "B": w.B, "L": w.L, "V": w.V, "dtype": w.dtype}
     logits = syn.make_logits(w, seed=4321, device=dev, step=0)
     for mode in (fd.PROFILE, fd.FACTOR):  # one untimed call per rule: one-time set-up
         m0 = torch.from_numpy(syn.make_mask(w, seed=4321)).to(dev)
-        fd.fdllm_select(logits, m0, 1.0, mode, stream=stream)
+        fd.fdllm_select(logits, m0, param, mode, stream=stream)
     stream.synchronize()
     del logits
     for rule in ("profile", "factor"):
@@ -627,7 +629,7 @@ def run_full_sequence(args, torch, fd, syn, dev, stream) -> dict:
             e0 = torch.cuda.Event(enable_timing=True)
             e1 = torch.cuda.Event(enable_timing=True)
             e0.record(stream)
-            fd.fdllm_select(logits, mask, 1.0, fd.MODES[rule], tok, commit, n, stream=stream)
+            fd.fdllm_select(logits, mask, param, fd.MODES[rule], tok, commit, n, stream=stream)
             e1.record(stream)
             e1.synchronize()
             times.append(e0.elapsed_time(e1))
@@ -635,7 +637,7 @@ def run_full_sequence(args, torch, fd, syn, dev, stream) -> dict:
             del logits
             remaining = int(mask.sum().item())
         t = np.array(times)
-        res[rule + " f=1"] = {
+        res["%s f=%g" % (rule, param)] = {
             "steps": len(times), "finished": remaining == 0,
             "tokens_per_step": float((w.B * w.L - remaining) / max(len(times), 1)),
             "per_step_ms_median": float(np.median(t)), "per_step_ms_mean": float(t.mean()),
@@ -708,63 +710,21 @@ def run_lmhead_key(args, torch) -> dict:
 
 # ----------------------------------------------------------------------------- loop mode
 def run_loop(args) -> dict:
-    """Selection + commit repeated until no mask remains, for the profile and the factor
-    rule (f = args.param): steps taken and per-step selection latency.  Logits are
-    regenerated from (seed, step) before each step, outside the timed region; each step's
-    selection is timed with CUDA events on its stream."""
-    import numpy as np
+    """--loop: a workload's selection + commit until no mask remains, profile against factor
+    (f = args.param), as the default line's full-sequence figures (run_full_sequence)."""
     import torch
 
     import fdllm_synth as syn
     import paper_2606_02955_gb300 as fd
 
-    w = syn.WORKLOADS[args.workload]
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     stream = torch.cuda.Stream(device=dev)
-    out = {}
-    # One untimed call per rule first, so that the library's one-time set-up (kernel
-    # attributes, occupancy queries, its workspace) stays out of the first timed step.
-    logits = syn.make_logits(w, seed=4321, device=dev, step=0)
-    for mode in (fd.PROFILE, fd.FACTOR):
-        m0 = torch.from_numpy(syn.make_mask(w, seed=4321)).to(dev)
-        fd.fdllm_select(logits, m0, args.param, mode, stream=stream)
-    torch.cuda.synchronize()
-    del logits
-    for mode_name, mode in (("profile", fd.PROFILE), ("factor", fd.FACTOR)):
-        mask = torch.from_numpy(syn.make_mask(w, seed=4321)).to(dev)
-        tok = torch.full((w.B, w.L), -1, dtype=torch.int32, device=dev)
-        commit = torch.empty((w.B, w.L), dtype=torch.uint8, device=dev)
-        n = torch.empty((w.B,), dtype=torch.int32, device=dev)
-        times, masked, step = [], [], 0
-        while True:
-            remaining = int(mask.sum().item())
-            if remaining == 0 or step >= w.L + 1:
-                break
-            logits = syn.make_logits(w, seed=4321, device=dev, step=step)
-            torch.cuda.synchronize()
-            e0 = torch.cuda.Event(enable_timing=True)
-            e1 = torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-            fd.fdllm_select(logits, mask, args.param, mode, tok, commit, n, stream=stream)
-            e1.record(stream)
-            e1.synchronize()
-            times.append(e0.elapsed_time(e1))
-            masked.append(remaining)
-            del logits
-            step += 1
-        t = np.array(times)
-        first_bytes = masked[0] * w.V * w.elem_bytes
-        out[mode_name] = {
-            "steps": step, "finished": remaining == 0,
-            "per_step_ms_median": float(np.median(t)), "per_step_ms_mean": float(t.mean()),
-            "first_step_ms": float(t[0]), "total_selection_ms": float(t.sum()),
-            "first_step_logits_gbs": first_bytes / (t[0] * 1e-3) / 1e9,
-            "tokens_per_step": float(w.B * w.L / max(step, 1)),
-        }
+    args.full_seq_max_steps = max(args.full_seq_max_steps, syn.WORKLOADS[args.workload].L + 1)
+    res = run_full_sequence(args, torch, fd, syn, dev, stream, args.workload, args.param)
     return {"metric": "full-sequence loop: steps until no mask remains and per-step "
-                      "selection latency", "workload": w.name, "B": w.B, "L": w.L, "V": w.V,
-            "dtype": w.dtype, "param": args.param, "data": "synthetic", "results": out}
+                      "selection latency", "workload": args.workload, "data": "synthetic",
+            "param": args.param, "results": res}
 
 
 def run_decode_loop(args) -> dict:
