@@ -424,7 +424,7 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
     t_k1, _, _, _ = sb.time_steps(k1_only, want, args.warmup, args.no_graph, dist)
     t_k1a, _, _, _ = sb.time_steps(k1_alone, want, args.warmup, args.no_graph, dist)
     # distribution of the step time: replays timed one by one (outside the timed region)
-    dist_us = sb.step_distribution(step_run, min(200, steps // sb.n_buf))
+    dist_us = sb.step_distribution(step_run, 125)
     if sampler is not None:
         time.sleep(0.02)
         sampler.stop()
@@ -1185,7 +1185,9 @@ def main(argv=None):
     ap.add_argument("--eta", type=float, default=0.02,
                     help="calibration allowance of the robust rule (App. C)")
     ap.add_argument("--param", type=float, default=1.0)
-    ap.add_argument("--buffers", type=int, default=8)
+    ap.add_argument("--buffers", type=int, default=16,
+                    help="rotating logits buffers of the main workload (16: 8.3 GB); their "
+                         "masks are restored by one copy per graph replay of as many steps")
     ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--skip-e2e", action="store_true")
     ap.add_argument("--skip-cpu-baseline", action="store_true")
