@@ -156,13 +156,12 @@ __global__ void __launch_bounds__(T) profile_select_kernel(const ProfileSelectAr
     const int64_t base = (int64_t)blockIdx.x * L;
 
     // (c, x_hat) of this thread's position: folded from the vocab reduction's unit
-    // partials, or read from the given arrays.
-    // Launched as a programmatic dependent: whatever produced the unit partials or the
-    // confidences (and the mask) has completed and its writes are visible past this wait.
-    // As in the warp kernel: after the vocab reduction, the mask byte and the allowance are
-    // loaded before the launch wait (their writers completed before the reduction passed
-    // its own wait); the unit partials or confidences and the status word after it, all
-    // issued before any is used.
+    // partials, or read from the given arrays.  Launched as a programmatic dependent: the
+    // producer of the partials or confidences has completed past the launch wait.  As in the
+    // warp kernel, after the vocab reduction the mask byte and the allowance are loaded
+    // before that wait (their writers completed before the reduction passed its own wait,
+    // and the reduction writes neither); the partials or confidences and the status word
+    // after it, all issued before any is used.
     const bool in_row = t < L;
     const bool early = a.partials != nullptr;
     uint8_t mask_byte = 0;
@@ -188,8 +187,8 @@ __global__ void __launch_bounds__(T) profile_select_kernel(const ProfileSelectAr
             combine_position(a.partials + (base + t) * a.units_per_row, a.units_per_row, c,
                              tok);
         } else {
-            c = a.conf[base + t];
-            tok = a.tok[base + t];
+            c = __ldcg(a.conf + base + t);
+            tok = __ldcg(a.tok + base + t);
         }
     }
     if (!masked) {
