@@ -32,7 +32,14 @@
  *     and launch errors, detected on the host.  Per-row data errors are reported in out_n
  *     (see FDLLM_ROW_NONFINITE).
  *   - All kernels are deterministic: the same inputs on the same GPU model give
- *     bit-identical outputs.
+ *     bit-identical outputs.  A position's confidence depends only on its logits and the
+ *     call's shape (B * L, V, dtype), which fix how rows are cut into reduction units, so
+ *     identical rows of one call give identical confidences (exact ties stay ties).
+ *   - Arithmetic: confidences are reduced in fp32 (relative error within 1e-5 of the exact
+ *     value); the rules are evaluated on those fp32 confidences with exact 64-bit fixed-point
+ *     prefix sums of 1 - c in units of 2^-52 (delta = 1 - f formed from the same integer as
+ *     f, so a flat profile gives the factor rule's decision bit for bit), and the threshold
+ *     compares c with the smallest fp32 value >= tau, which decides c >= tau exactly.
  */
 #ifndef FDLLM_H
 #define FDLLM_H
