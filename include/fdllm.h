@@ -226,7 +226,9 @@ fdllm_status fdllm_gather_masked_rows(const void *src, void *dst, int dtype, int
  * back and synchronises `stream` before it returns: the results are in place when the call
  * returns.  Argument errors are reported before anything is enqueued; the same device
  * errors as fdllm_select (fdllm_device_status).  Not for stream capture (it synchronises).
- * The paper has no counterpart. */
+ * Calls share the staging buffer and the library workspace of their device: calls from
+ * several host threads at once must be serialised by the caller.  The paper has no
+ * counterpart. */
 fdllm_status fdllm_select_host(const void *logits, int dtype, int B, int L, int V,
                                uint8_t *mask, double param, int mode, int32_t *out_tokens,
                                uint8_t *out_commit, int32_t *out_n, void *stream);
