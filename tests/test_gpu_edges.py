@@ -256,3 +256,55 @@ def test_mask_reading_unaligned_and_partial_words(fd, orc, B, L, offset, density
     ok = ref["margin"] >= 1e-5
     assert np.array_equal(out[2].cpu().numpy()[ok], ref["n"][ok])
     assert np.array_equal(mask.cpu().numpy()[ok], ref["mask"][ok])
+
+
+def _select_from_conf_case(fd, orc, conf_np, mode, param):
+    B, L = conf_np.shape
+    mask_np = (conf_np > 0).astype(np.uint8)
+    tok_np = np.arange(B * L, dtype=np.int32).reshape(B, L)
+    mask = torch.from_numpy(mask_np.copy()).cuda()
+    t, c, n = fd.fdllm_select_from_conf(torch.from_numpy(conf_np).cuda(),
+                                        torch.from_numpy(tok_np).cuda(), mask, param, mode)
+    torch.cuda.synchronize()
+    ref = orc.select_from_conf(conf_np.astype(np.float64), tok_np, mask_np, mode, param)
+    return n.cpu().numpy(), c.cpu().numpy(), mask.cpu().numpy(), ref
+
+
+@pytest.mark.parametrize("tau", [0.3, 0.9, 0.1, 1.0 / 3.0, 0.875, 1.0, 1.0000001, 0.0, -1.0,
+                                 2.0])
+def test_threshold_decides_exactly_at_float_boundaries(fd, orc, tau):
+    """The threshold rule on fp32 confidences one ulp below, at and above the float nearest
+    tau (tau itself is rarely representable): c >= tau is decided exactly as the oracle
+    decides it on the same values in fp64, including tau at or beyond the ends of (0, 1]."""
+    t32 = np.float32(tau)
+    vals = [np.nextafter(t32, np.float32(-np.inf)), t32, np.nextafter(t32, np.float32(np.inf))]
+    vals = [v for v in vals if 0.0 < v <= 1.0] or [np.float32(0.5)]
+    rows = []
+    for v in vals:   # each row: the boundary value first, then fillers far below
+        rows.append([v, np.float32(0.01), np.float32(0.02), 0.0])
+        rows.append([np.float32(0.9999), v, 0.0, v])
+    conf_np = np.array(rows, np.float32)
+    n, c, m, ref = _select_from_conf_case(fd, orc, conf_np, THRESHOLD, tau)
+    assert np.array_equal(n, ref["n"]), (tau, conf_np, n, ref["n"])
+    assert np.array_equal(c, ref["commit"]) and np.array_equal(m, ref["mask"])
+
+
+@pytest.mark.parametrize("mode", [PROFILE, FACTOR])
+@pytest.mark.parametrize("f", [-1e30, -5.0, 0.0, 1e-12, 0.75, 1.0, 1.5, 1499.0, 2000.0, 1e30])
+def test_profile_and_factor_at_extreme_parameters(fd, orc, mode, f):
+    """Any finite f: far beyond the range where (n+1)(1 - c) <= 1025 can change a decision
+    (f clamped to +-1500 in the kernels' fixed point) every prefix is accepted or none is;
+    in between, the decisions equal the oracle's on the same fp32 confidences (dyadic
+    values, exact in both arithmetics)."""
+    rng = np.random.default_rng(int(abs(f)) % 1000 + mode)
+    conf_np = (rng.integers(1, 257, (6, 32)) / 256.0).astype(np.float32)
+    conf_np[rng.random((6, 32)) < 0.2] = 0.0   # unmasked
+    conf_np[0, :] = np.float32(1.0)            # all certain
+    conf_np[1, :5] = np.float32(0.5)           # flat
+    n, c, m, ref = _select_from_conf_case(fd, orc, conf_np, mode, f)
+    ok = ref["margin"] >= 1e-12
+    assert np.array_equal(n[ok], ref["n"][ok]), (f, n, ref["n"])
+    assert np.array_equal(c[ok], ref["commit"][ok])
+    if abs(f) >= 1500:
+        m_rows = (conf_np > 0).sum(axis=1)
+        assert np.array_equal(n, m_rows if f > 0 else np.minimum(m_rows, 1))
