@@ -30,7 +30,9 @@
  *   - Limits: 1 <= B, 1 <= L <= FDLLM_MAX_L, B * L <= FDLLM_MAX_ROWS, V >= 1.
  *   - Work is enqueued asynchronously on `stream`; the return value reports only argument
  *     and launch errors, detected on the host.  Per-row data errors are reported in out_n
- *     (see FDLLM_ROW_NONFINITE).
+ *     (see FDLLM_ROW_NONFINITE) and, for calls that use a workspace, in its sticky status
+ *     word, which fdllm_device_status / fdllm_workspace_status / fdllm_static_status read
+ *     as FDLLM_ERR_NONFINITE.
  *   - All kernels are deterministic: the same inputs on the same GPU model give
  *     bit-identical outputs.  A position's confidence depends only on its logits and the
  *     call's shape (B * L, V, dtype), which fix how rows are cut into reduction units, so
@@ -67,7 +69,7 @@ typedef enum {
     FDLLM_ERR_ARG = 1,       /* a null pointer, a size out of range, an unknown enum, a
                                 non-finite param                                         */
     FDLLM_ERR_ALIGN = 2,     /* logits base not 16-byte aligned or V*sizeof(dtype) % 16 */
-    FDLLM_ERR_NONFINITE = 3, /* reserved for callers mapping out_n == -1 to a status     */
+    FDLLM_ERR_NONFINITE = 3, /* a selection met a row of FDLLM_ROW_NONFINITE (status word) */
     FDLLM_ERR_CUDA = 4,      /* a CUDA runtime call or kernel launch failed             */
     FDLLM_ERR_WORKSPACE = 5, /* caller workspace too small or misaligned                */
     FDLLM_ERR_DEVICE = 6     /* a kernel's bounded wait gave up (see fdllm_device_status) */
@@ -168,7 +170,8 @@ fdllm_status fdllm_select_static(const void *logits, int dtype, int B, int L, in
 /* The sticky device error of fdllm_select_static's array on the current device, as
  * fdllm_device_status reports the library workspace's: synchronises `stream`, returns
  * FDLLM_ERR_DEVICE if a kernel of a static call gave up a bounded wait (every row of that
- * call also reports out_n = -2), FDLLM_OK otherwise, and clears the error.  Call it after a
+ * call also reports out_n = -2), else FDLLM_ERR_NONFINITE if its selection found a row of
+ * FDLLM_ROW_NONFINITE, FDLLM_OK otherwise, and clears the status.  Call it after a
  * static call and before the next one, which clears the array's status word itself.
  * Allocates nothing. */
 fdllm_status fdllm_static_status(void *stream);
@@ -293,6 +296,10 @@ typedef int (*fdllm_forward_fn)(void *user, const int32_t *loop_state,
  *   nfe_per_block   [gen_len / block_len] int32 device output: steps (NFE) per block.
  *   max_steps       bound on the total number of steps; reaching it ends the loop early
  *                   and returns FDLLM_ERR_DEVICE.
+ * A step whose selection reports a row as FDLLM_ROW_NONFINITE ends the loop after that
+ * step with FDLLM_ERR_NONFINITE (such a row commits nothing, so its block would never
+ * finish); a step that reports FDLLM_ROW_DEVICE_ERROR ends it with FDLLM_ERR_DEVICE.
+ * nfe_per_block then holds the steps of the blocks reached and out_steps the steps taken.
  *   out_steps       host int: total steps taken.
  * Synchronous: returns when the generation is finished.  Allocates its own small buffers
  * and the library workspace (outside the graph).  Limits as fdllm_select with L = block_len;
@@ -350,7 +357,8 @@ fdllm_status fdllm_check_bounded_wait(double seconds, void *stream);
 
 /* Synchronises `stream`, then reports (and clears) the sticky device error of the library
  * workspace on the current device: FDLLM_ERR_DEVICE if a kernel gave up a bounded wait
- * since the last call, FDLLM_OK otherwise.  For fdllm_select_ws, pass the workspace to
+ * since the last call, else FDLLM_ERR_NONFINITE if a selection since the last call found a
+ * row of FDLLM_ROW_NONFINITE, FDLLM_OK otherwise.  For fdllm_select_ws, pass the workspace to
  * fdllm_workspace_status instead.  Clearing an error also resets the workspace's work
  * counter, which a launch that gave up may have left mid-queue, so that the next call
  * starts from a clean header. */

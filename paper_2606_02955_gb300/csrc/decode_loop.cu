@@ -14,11 +14,17 @@
 namespace fdllm {
 namespace {
 
+// Why the loop stopped before the generation finished (LoopState::stop_reason).
+constexpr int32_t kStopNone = 0;
+constexpr int32_t kStopMaxSteps = 1;   // max_steps reached
+constexpr int32_t kStopNonfinite = 2;  // a row's logits were unusable (FDLLM_ROW_NONFINITE)
+constexpr int32_t kStopDevice = 3;     // a kernel gave up a bounded wait (FDLLM_ROW_DEVICE_ERROR)
+
 struct LoopState {
     int32_t step;         // global step (forward passes so far)
     int32_t block;        // current block
     int32_t block_steps;  // steps spent in the current block
-    int32_t overflow;     // nonzero: max_steps reached before the generation finished
+    int32_t stop_reason;  // kStop*: nonzero when the loop ended early
 };
 
 __global__ void loop_init_kernel(LoopState *st, uint8_t *block_mask, int64_t block_rows,
@@ -30,7 +36,7 @@ __global__ void loop_init_kernel(LoopState *st, uint8_t *block_mask, int64_t blo
         st->step = 0;
         st->block = 0;
         st->block_steps = 0;
-        st->overflow = 0;
+        st->stop_reason = kStopNone;
     }
     for (int64_t i = tid; i < block_rows; i += stride)
         block_mask[i] = 1;
@@ -41,17 +47,21 @@ __global__ void loop_init_kernel(LoopState *st, uint8_t *block_mask, int64_t blo
 }
 
 // One CTA.  Runs after the step's selection: reveal (Alg. 1) into the sequence, count the
-// step, and at the end of a block move on (re-mask the block buffer) or stop the loop.
+// step, and at the end of a block move on (re-mask the block buffer) or stop the loop.  A
+// step whose selection reported a row as unusable or failed ends the loop: such a row
+// commits nothing, so the block would never finish.
 __global__ void loop_control_kernel(LoopState *st, uint8_t *block_mask, const uint8_t *commit,
-                                    const int32_t *block_tokens, int32_t *seq, int32_t *nfe,
-                                    int B, int Lb, int gen_len, int nblocks, int max_steps,
-                                    cudaGraphConditionalHandle cond)
+                                    const int32_t *block_tokens, const int32_t *block_n,
+                                    int32_t *seq, int32_t *nfe, int B, int Lb, int gen_len,
+                                    int nblocks, int max_steps, cudaGraphConditionalHandle cond)
 {
     __shared__ int any_masked;
     __shared__ int advance;
+    __shared__ int worst_n;
     if (threadIdx.x == 0) {
         any_masked = 0;
         advance = 0;
+        worst_n = 0;
     }
     __syncthreads();
     const int blk = st->block;
@@ -63,12 +73,19 @@ __global__ void loop_control_kernel(LoopState *st, uint8_t *block_mask, const ui
         if (block_mask[i])
             any_masked = 1;
     }
+    for (int b = threadIdx.x; b < B; b += blockDim.x)
+        if (block_n[b] < 0)
+            atomicMin(&worst_n, block_n[b]);
     __syncthreads();
     if (threadIdx.x == 0) {
         st->step += 1;
         st->block_steps += 1;
         bool stop = false;
-        if (!any_masked) {
+        if (worst_n < 0) {
+            st->stop_reason = worst_n == FDLLM_ROW_DEVICE_ERROR ? kStopDevice : kStopNonfinite;
+            nfe[blk] = st->block_steps;
+            stop = true;
+        } else if (!any_masked) {
             nfe[blk] = st->block_steps;
             st->block = blk + 1;
             st->block_steps = 0;
@@ -76,7 +93,7 @@ __global__ void loop_control_kernel(LoopState *st, uint8_t *block_mask, const ui
             advance = !stop;
         }
         if (!stop && st->step >= max_steps) {
-            st->overflow = 1;
+            st->stop_reason = kStopMaxSteps;
             nfe[blk] = st->block_steps;
             stop = true;
             advance = 0;
@@ -156,8 +173,8 @@ fdllm_status build_loop_graph(const LoopArgs &a, cudaStream_t cs, bool pdl, Loop
         st = run_step_select(a, cs, pdl);
     if (st == FDLLM_OK) {
         loop_control_kernel<<<1, 256, 0, cs>>>(a.st, a.block_mask, a.commit, a.block_tokens,
-                                               a.seq, a.nfe, a.B, a.Lb, a.gen_len, a.nblocks,
-                                               a.max_steps, cond);
+                                               a.block_n, a.seq, a.nfe, a.B, a.Lb, a.gen_len,
+                                               a.nblocks, a.max_steps, cond);
         if (cudaGetLastError() != cudaSuccess)
             st = FDLLM_ERR_CUDA;
     }
@@ -240,7 +257,9 @@ fdllm_status run_decode_loop(LoopArgs a, int *out_steps, cudaStream_t s)
             cudaStreamSynchronize(s) != cudaSuccess)
             break;
         *out_steps = host.step;
-        result = host.overflow ? FDLLM_ERR_DEVICE : FDLLM_OK;
+        result = host.stop_reason == kStopNone        ? FDLLM_OK
+                 : host.stop_reason == kStopNonfinite ? FDLLM_ERR_NONFINITE
+                                                      : FDLLM_ERR_DEVICE;
     } while (false);
 
     if (cs)

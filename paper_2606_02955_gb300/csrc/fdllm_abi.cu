@@ -8,6 +8,7 @@
 
 #include "fdllm.h"
 #include "fdllm_internal.cuh"
+#include "ptx.cuh"
 
 namespace fdllm {
 namespace {
@@ -181,7 +182,8 @@ namespace {
 
 // Reads the sticky status word and, when it is set, zeroes `clear_bytes` from it: for a
 // workspace header the status word and the vocab reduction's work counter, which a launch
-// that gave up a wait may leave mid-queue (it stops fetching before its last unit).
+// that gave up a wait may leave mid-queue (it stops fetching before its last unit).  A
+// gave-up wait outranks a non-finite row.
 fdllm_status read_and_clear_status(uint32_t *status, cudaStream_t stream,
                                    size_t clear_bytes = sizeof(uint32_t))
 {
@@ -196,7 +198,7 @@ fdllm_status read_and_clear_status(uint32_t *status, cudaStream_t stream,
     if (cudaMemsetAsync(status, 0, clear_bytes, stream) != cudaSuccess ||
         cudaStreamSynchronize(stream) != cudaSuccess)
         return FDLLM_ERR_CUDA;
-    return FDLLM_ERR_DEVICE;
+    return (host & kDevStatTimeout) != 0 ? FDLLM_ERR_DEVICE : FDLLM_ERR_NONFINITE;
 }
 
 // Status word and work counter at the head of every workspace.

@@ -128,7 +128,8 @@ struct ProfileSelectArgs {
     int32_t *out_tokens;     // [B, L]
     uint8_t *out_commit;     // [B, L]
     int32_t *out_n;          // [B]
-    const uint32_t *status;  // nullable: nonzero -> every row reports a device error
+    uint32_t *status;        // nullable: the timeout bit set -> every row reports a device
+                             // error; a non-finite row sets the non-finite bit
     bool pdl = true;         // with partials: launch as a programmatic dependent
 };
 

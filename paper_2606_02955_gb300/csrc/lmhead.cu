@@ -1234,7 +1234,7 @@ fdllm_status lmhead_select_owned(const void *hidden, const void *w_vocab, int B,
     pa.out_tokens = out_tokens;
     pa.out_commit = out_commit;
     pa.out_n = out_n;
-    pa.status = reinterpret_cast<const uint32_t *>(ws);
+    pa.status = reinterpret_cast<uint32_t *>(ws);
     pa.pdl = pdl;
     return launch_profile_select(pa, s) == cudaSuccess ? FDLLM_OK : FDLLM_ERR_CUDA;
 }

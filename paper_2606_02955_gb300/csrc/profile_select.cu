@@ -18,6 +18,7 @@
 #include <cstdint>
 
 #include "fdllm_internal.cuh"
+#include "ptx.cuh"
 
 namespace fdllm {
 namespace {
@@ -178,7 +179,7 @@ __global__ void __launch_bounds__(T) profile_select_kernel(const ProfileSelectAr
         pdl_launch_dependents();  // a following vocab reduction may start its prologue
     if (!early)
         load_row_inputs();
-    const bool dev_err = a.status != nullptr && __ldcg(a.status) != 0;
+    const bool dev_err = a.status != nullptr && (__ldcg(a.status) & kDevStatTimeout) != 0;
     const bool masked = mask_byte != 0;
     float c = 0.0f;
     int32_t tok = -1;
@@ -220,8 +221,11 @@ __global__ void __launch_bounds__(T) profile_select_kernel(const ProfileSelectAr
     int nstar = block_max<T>(ok ? n : 0, warp_red);
     if (m > 0 && nstar == 0)
         nstar = 1;  // progress convention
-    if (any_bad)
+    if (any_bad) {
         nstar = -1;
+        if (t == 0 && a.status != nullptr)
+            atomicOr(a.status, kDevStatNonfinite);
+    }
     if (dev_err)
         nstar = -2;
 
@@ -326,9 +330,12 @@ __global__ void __launch_bounds__(32) profile_select_warp_kernel(const ProfileSe
     int nstar = __reduce_max_sync(kFull, ok ? n : 0);
     if (m > 0 && nstar == 0)
         nstar = 1;  // progress convention
-    if (any_bad)
+    if (any_bad) {
         nstar = -1;
-    if (status != 0)
+        if (t == 0 && a.status != nullptr)
+            atomicOr(a.status, kDevStatNonfinite);
+    }
+    if ((status & kDevStatTimeout) != 0)
         nstar = -2;
 
     if (t < L) {

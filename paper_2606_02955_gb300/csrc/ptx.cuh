@@ -6,12 +6,17 @@
 
 namespace fdllm {
 
-// A wait on an mbarrier gives up after this long and records FDLLM_DEVSTAT_TIMEOUT.
+// A wait on an mbarrier gives up after this long and records kDevStatTimeout.
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s
 // After a wait gave up, how long a CTA waits for its own asynchronous copies still in
 // flight (they write its shared memory) before it exits.
 constexpr uint64_t kDrainLimitNs = 100000000ull;  // 100 ms
+// Bits of a workspace's sticky status word.  kDevStatTimeout: a kernel gave up a bounded
+// wait (the step's rows report FDLLM_ROW_DEVICE_ERROR).  kDevStatNonfinite: a selection
+// found a batch row with unusable logits (FDLLM_ROW_NONFINITE); the kernels themselves
+// completed normally, so only the timeout bit makes later kernels treat the step as failed.
 constexpr uint32_t kDevStatTimeout = 1u;
+constexpr uint32_t kDevStatNonfinite = 2u;
 
 __device__ __forceinline__ uint32_t smem_addr(const void *p)
 {

@@ -19,6 +19,8 @@ import fdllm_synth
 
 CONF_RTOL = 1e-5
 MARGIN = 1e-5
+ERR_NONFINITE = 3   # fdllm_status FDLLM_ERR_NONFINITE
+ROW_NONFINITE = -1  # out_n of a row with unusable logits
 
 
 def oracle_threads() -> int:
@@ -55,13 +57,16 @@ def check_select(fd, orc, logits: torch.Tensor, mask_np: np.ndarray, mode: int, 
     """fdllm_select against the oracle; returns the number of low-margin rows."""
     B, L = mask_np.shape
     mask = torch.from_numpy(mask_np.copy()).cuda()
+    assert fd.fdllm_device_status() == 0, "status word already set before this call"
     tok, commit, n = fd.fdllm_select(logits, mask, param, mode)
-    torch.cuda.synchronize()
+    status = fd.fdllm_device_status()  # synchronises; reads and clears the status word
     g = dict(tokens=tok.cpu().numpy(), commit=commit.cpu().numpy(), n=n.cpu().numpy(),
              mask=mask.cpu().numpy())
     if ref is None:
         host = fdllm_synth.host_bits(logits)
         ref = orc.select(host, mask_np, mode, param, nthreads=oracle_threads())
+    # the status word reports non-finite rows exactly when the oracle has one
+    assert status == (ERR_NONFINITE if (ref["n"] == ROW_NONFINITE).any() else 0), status
     low = ref["margin"] < MARGIN
     ok = ~low
     assert np.array_equal(g["n"][ok], ref["n"][ok]), (

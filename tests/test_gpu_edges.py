@@ -6,7 +6,7 @@ import pytest
 import torch
 
 import fdllm_synth as syn
-from gpu_util import check_confidence, check_select
+from gpu_util import ERR_NONFINITE, check_confidence, check_select
 
 pytestmark = pytest.mark.gpu
 PROFILE, FACTOR, THRESHOLD = 0, 1, 2
@@ -73,6 +73,9 @@ def test_nonfinite_rows(fd, orc):
     tok, commit, n = fd.fdllm_select(logits, mask, 0.75, PROFILE)
     assert n.cpu().tolist() == [fd.ROW_NONFINITE] * 3
     assert commit.sum().item() == 0 and mask.sum().item() == 12
+    # the workspace's status word says so too, and reading it clears it
+    assert fd.fdllm_device_status() == ERR_NONFINITE
+    assert fd.fdllm_device_status() == 0
     # -inf entries alone are fine
     x[2, 3, 4000] = 0.0
     x[0, 1, 100] = 0.0
@@ -80,6 +83,51 @@ def test_nonfinite_rows(fd, orc):
     logits = torch.from_numpy(x).cuda()
     check_confidence(fd, orc, logits, mask_np)
     check_select(fd, orc, logits, mask_np, PROFILE, 0.75)
+
+
+def test_nonfinite_rows_reported_by_every_status_word(fd):
+    """A NaN in one masked row: the caller workspace's and the static array's status words
+    report FDLLM_ERR_NONFINITE after the step (the other row still commits), and a clean
+    step afterwards reads FDLLM_OK."""
+    B, L, V = 2, 8, 4096
+    x = np.random.default_rng(6).normal(0, 1, (B, L, V)).astype(np.float32)
+    x[1, 5, 7] = np.nan
+    mask_np = np.ones((B, L), np.uint8)
+    ws = torch.zeros(fd.fdllm_workspace_bytes(B, L, V, fd.FP32), dtype=torch.uint8,
+                     device="cuda")
+    for bad in (True, False):
+        logits = torch.from_numpy(x).cuda()
+        expect = ERR_NONFINITE if bad else 0
+        _, _, n = fd.fdllm_select_ws(logits, torch.from_numpy(mask_np.copy()).cuda(), 0.75,
+                                     PROFILE, ws)
+        assert fd.fdllm_workspace_status(ws) == expect
+        assert n[0].item() >= 1 and (n[1].item() == fd.ROW_NONFINITE) == bad
+        _, _, n = fd.fdllm_select_static(logits, torch.from_numpy(mask_np.copy()).cuda(), 0.75,
+                                         PROFILE)
+        assert fd.fdllm_static_status() == expect
+        assert n[0].item() >= 1 and (n[1].item() == fd.ROW_NONFINITE) == bad
+        assert fd.fdllm_static_status() == 0
+        x[1, 5, 7] = 0.0
+
+
+def test_decode_loop_stops_on_a_nonfinite_row(fd):
+    """A forward pass that leaves a NaN in a masked row: that row commits nothing, so the
+    loop ends after the step with FDLLM_ERR_NONFINITE instead of running to max_steps
+    (which would read as FDLLM_ERR_DEVICE)."""
+    B, gen, Lb, V = 2, 64, 32, 4096
+    logits = torch.empty((B, Lb, V), dtype=torch.bfloat16, device="cuda")
+
+    def forward(state, mask, out, stream):
+        syn.synth_block_logits_gpu(out, mask, B, Lb, V, 3, step_ptr=state, peak_max=16.0,
+                                   stream_ptr=stream)
+        with torch.cuda.stream(torch.cuda.ExternalStream(stream)):
+            logits[1, 4, 9].fill_(float("nan"))
+
+    with pytest.raises(fd.FdllmError) as err:
+        fd.fdllm_decode_loop(forward, logits, gen, 1.0, PROFILE, max_steps=10 * gen)
+    assert err.value.status == ERR_NONFINITE
+    assert fd.fdllm_device_status() == ERR_NONFINITE
+    assert fd.fdllm_device_status() == 0
 
 
 @pytest.mark.parametrize("dtype", ["bf16", "fp16", "fp32"])
