@@ -93,9 +93,10 @@ def peak_hbm_gbs():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def ncu_traffic():
-    """DRAM traffic per vocab-reduction launch from the committed ncu summary, only while
-    the kernel's sources (hashed in order) are the ones the counters were taken on."""
+def ncu_traffic(workload: str):
+    """DRAM traffic per vocab-reduction launch from the committed ncu summary, only for the
+    workload the summary was captured on and while the kernel's sources (hashed in order)
+    are the ones the counters were taken on."""
     try:
         text = open(PROFILE_SUMMARY).read()
         h = hashlib.sha256()
@@ -106,7 +107,8 @@ def ncu_traffic():
         return None
     m_sha = re.search(r"source_sha256:\s*([0-9a-f]{64})", text)
     m_t = re.search(r"traffic_bytes_per_launch:\s*([0-9]+)", text)
-    if not (m_sha and m_t) or m_sha.group(1) != sha:
+    m_w = re.search(r"workload:\s*(\S+)", text)
+    if not (m_sha and m_t and m_w) or m_sha.group(1) != sha or m_w.group(1) != workload:
         return None
     return int(m_t.group(1))
 
@@ -444,7 +446,7 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
         peak, peak_kind = peak_hbm_gbs()
         k1_s = t_k1a / steps
         achieved = sb.alg_bytes / k1_s / 1e9
-        traffic = ncu_traffic()
+        traffic = ncu_traffic(w.name)
         clocks = sampler.summary(tw0, tw1) if sampler is not None else None
         result = {
             "metric": METRIC, "value": agg["value"], "unit": UNIT, "n_gpus": world,

@@ -145,3 +145,18 @@ def test_main_arm_prints_one_contract_line():
     assert e["value"] > 0 and e["h2d_bytes_per_step"] > 0 and e["d2h_bytes_per_step"] > 0
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] > 0 and cb["sample"]
+
+
+def test_ncu_traffic_only_for_its_workload_and_sources(monkeypatch, tmp_path):
+    """The roofline's `traffic` comes from the committed ncu summary of the serving workload
+    only while the reduction's sources hash to the value recorded there (a kernel changed
+    since the capture reads as null), and never for another workload."""
+    sys.path.insert(0, ROOT)
+    import bench
+    t = bench.ncu_traffic("serving_b64_l32_bf16")
+    assert t is not None and t > 0, "profile summary is stale: re-capture it on these sources"
+    assert bench.ncu_traffic("single_block_b1_l32_bf16") is None
+    changed = tmp_path / "vocab_reduce.cu"
+    changed.write_text("// another kernel\n")
+    monkeypatch.setattr(bench, "KERNEL_SOURCES", [str(changed)])
+    assert bench.ncu_traffic("serving_b64_l32_bf16") is None
