@@ -56,9 +56,10 @@ METRIC = ("decode-step selections/sec and logits HBM GB/s (fraction of GB300 pea
 UNIT = "selections/s"
 FALLBACK_HBM_GBS = 6800.0
 PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "vocab_reduce_serving_b64_l32_bf16.md")
-# the vocab reduction's sources: the kernel and the unit plan it shares with the interface
+# the vocab reduction's sources: the kernel, the unit plan it shares with the interface and
+# the inline-PTX copies and waits it is built from
 KERNEL_SOURCES = [os.path.join(ROOT, "paper_2606_02955_gb300", "csrc", f)
-                  for f in ("vocab_reduce.cu", "fdllm_internal.cuh")]
+                  for f in ("vocab_reduce.cu", "fdllm_internal.cuh", "ptx.cuh")]
 
 
 # ----------------------------------------------------------------------------- host logic
