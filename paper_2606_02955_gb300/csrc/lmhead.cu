@@ -413,19 +413,22 @@ __global__ void __launch_bounds__(kThreads, 1)
 // few W rows as possible: LLaDA's V = 126464 is 1216 tiles of 104, eight per SM on 152
 // SMs); CTA c of P owns the tiles c, c + P, c + 2P, ..., so the CTAs read W in a window that
 // moves through it.  The MMA always spans 128 lanes; lanes h..127 hold sums of stale shared
-// memory that the epilogue skips.  The padded row tile costs 4 KB per stage instead of
-// 16 KB, so 11 stages (143 KB of W at h = 104) are in flight per SM.  Each epilogue thread keeps, for every row, a running maximum, sum
+// memory that the epilogue skips.  The padded row tile costs 4 KB per K-block instead of
+// 16 KB.  A stage holds two K-blocks (two W boxes and two row boxes), five stages in all
+// (130 KB of W at h = 104 in flight per SM): per-copy overhead, not the bytes in flight,
+// limits how fast W streams here, and two blocks per stage beat one, three or four.  Each epilogue thread keeps, for every row, a running maximum, sum
 // of exp relative to it and first index over its own entry of each tile; after the last
 // tile the 128 threads' states are folded per row (a transposing butterfly in each warp,
 // then the four warps in order) into one partial per (row, CTA).
 constexpr int kSlabRows = 32;
 constexpr int kSlabABytes = BM * BK * 2;                 // 128 lanes; a tile fills h rows
 constexpr int kSlabBBytes = kSlabRows * BK * 2;
-constexpr int kSlabStages = 11;
+constexpr int kSlabKB = 2;                               // K-blocks of BK per stage
+constexpr int kSlabStages = 5;
 constexpr int kSlabAccs = 4;                             // accumulators of 32 columns
 constexpr uint32_t kSlabTmemCols = 128;
 constexpr size_t kSlabSmemBytes =
-    1024 + (size_t)kSlabStages * (kSlabABytes + kSlabBBytes) + kBarrierBytes;
+    1024 + (size_t)kSlabStages * kSlabKB * (kSlabABytes + kSlabBBytes) + kBarrierBytes;
 static_assert(kSlabSmemBytes <= 227 * 1024, "slab ring");
 static_assert((2 * kSlabStages + 2 * kSlabAccs + 1) * 8 + 8 <= (int)kBarrierBytes, "barriers");
 
@@ -451,9 +454,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     __shared__ uint32_t s_I[4][kSlabRows];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint8_t *sA = smem;                              // kSlabStages x [128 W rows][128 B]
-    uint8_t *sB = smem + kSlabStages * kSlabABytes;  // kSlabStages x [32 rows][128 B]
-    uint64_t *bars = reinterpret_cast<uint64_t *>(sB + kSlabStages * kSlabBBytes);
+    // kSlabStages x kSlabKB x [128 W rows][128 B], then kSlabStages x kSlabKB x [32 rows][128 B]
+    uint8_t *sA = smem;
+    uint8_t *sB = smem + kSlabStages * kSlabKB * kSlabABytes;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sB + kSlabStages * kSlabKB * kSlabBBytes);
     uint64_t *full = bars;
     uint64_t *empty = bars + kSlabStages;
     uint64_t *tfull = bars + 2 * kSlabStages;
@@ -503,18 +507,25 @@ __global__ void __launch_bounds__(kThreads, 1)
                 used[i] = false;
             bool ok = true;
             // a box's bytes count in full, the part beyond V zero-filled
-            const uint32_t bytes = (uint32_t)(h * BK * 2) + kSlabBBytes;
+            // (K-blocks past H, in the last stage when k_blocks is odd, are zero-filled and
+            // count in full too)
+            const uint32_t bytes = kSlabKB * ((uint32_t)(h * BK * 2) + kSlabBBytes);
             for (int t = 0; ok && t < n_t; ++t) {
                 const int64_t T = c + (int64_t)t * P;
-                for (int kb = 0; kb < a.k_blocks; ++kb) {
+                for (int kb = 0; kb < a.k_blocks; kb += kSlabKB) {
                     if (!wait_or_abort(&empty[s], ph ^ 1u, a.status, abort_flag)) {
                         ok = false;
                         break;
                     }
                     mbar_arrive_expect_tx(&full[s], bytes);
-                    tc::tma_load_2d_hint(sA + s * kSlabABytes, &map_w, kb * BK, (int32_t)(T * h),
-                                         &full[s], pol);
-                    tc::tma_load_2d(sB + s * kSlabBBytes, &map_h, kb * BK, 0, &full[s]);
+#pragma unroll
+                    for (int q = 0; q < kSlabKB; ++q)
+                        tc::tma_load_2d_hint(sA + (s * kSlabKB + q) * kSlabABytes, &map_w,
+                                             (kb + q) * BK, (int32_t)(T * h), &full[s], pol);
+#pragma unroll
+                    for (int q = 0; q < kSlabKB; ++q)
+                        tc::tma_load_2d(sB + (s * kSlabKB + q) * kSlabBBytes, &map_h, (kb + q) * BK,
+                                        0, &full[s]);
                     used[s] = true;
                     last_ph[s] = ph;
                     if (++s == kSlabStages) {
@@ -540,7 +551,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     break;
                 tc::fence_after_sync();
                 const uint32_t d = tmem_base + (uint32_t)(acc * kSlabRows);
-                for (int kb = 0; kb < a.k_blocks; ++kb) {
+                for (int kb = 0; kb < a.k_blocks; kb += kSlabKB) {
                     if (!wait_or_abort(&full[s], ph, a.status, abort_flag)) {
                         ok = false;
                         break;
@@ -548,11 +559,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tc::fence_after_sync();
                     // Rows h..127 of the A stage are stale: those TMEM lanes hold
                     // meaningless sums that the epilogue skips.
-                    const uint64_t ad = tc::sw128_kmajor_desc(sA + s * kSlabABytes);
-                    const uint64_t bd = tc::sw128_kmajor_desc(sB + s * kSlabBBytes);
 #pragma unroll
-                    for (int k = 0; k < BK / 16; ++k)
-                        tc::mma_bf16(d, ad + 2u * k, bd + 2u * k, idesc, (kb | k) != 0);
+                    for (int q = 0; q < kSlabKB; ++q) {
+                        const uint64_t ad =
+                            tc::sw128_kmajor_desc(sA + (s * kSlabKB + q) * kSlabABytes);
+                        const uint64_t bd =
+                            tc::sw128_kmajor_desc(sB + (s * kSlabKB + q) * kSlabBBytes);
+#pragma unroll
+                        for (int k = 0; k < BK / 16; ++k)
+                            tc::mma_bf16(d, ad + 2u * k, bd + 2u * k, idesc, (kb | q | k) != 0);
+                    }
                     tc::commit(&empty[s]);
                     if (++s == kSlabStages) {
                         s = 0;
@@ -952,8 +968,8 @@ int slab_grid(int V)
 
 // Rows of W per CTA on the longest-running SM, for the slab variant (whole tiles of its
 // height) against the tile variant (one row tile: whole waves of vocabulary tiles times
-// their width).  The slab variant keeps more W in flight per SM (11 stages of h rows against
-// the tile variant's 5 of its width); measured on LLaDA-sized heads, it is faster when its
+// their width).  The slab variant's row operand is 4 KB per K-block where a row tile's is
+// 16 KB, so more of each stage is W; measured on LLaDA-sized heads, it is faster when its
 // busiest CTA streams no more rows.
 bool slab_preferred(int V)
 {
