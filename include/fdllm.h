@@ -77,7 +77,9 @@ typedef enum {
 
 /* out_n value of a batch row whose masked logits are unusable: a NaN anywhere in a masked
  * position's row, or a maximum of +inf or -inf.  Such a row commits nothing and its mask
- * is left unchanged.  (The paper defines confidences only for proper distributions.) */
+ * is left unchanged; a call with a workspace also records it in the workspace's status word
+ * (FDLLM_ERR_NONFINITE from the status calls).  (The paper defines confidences only for
+ * proper distributions.) */
 #define FDLLM_ROW_NONFINITE (-1)
 /* out_n value of every row when a kernel of the step gave up a bounded wait. */
 #define FDLLM_ROW_DEVICE_ERROR (-2)
