@@ -212,3 +212,25 @@ def test_decode_loop_lmhead_against_host_loop_and_oracle(fd, orc, mode, param):
     assert steps_d == step
     assert list(nfe_d.cpu().numpy()) == nfe
     assert np.array_equal(seq_d.cpu().numpy(), seq)
+
+
+def test_decode_loop_lmhead_stops_on_a_nonfinite_hidden_state(fd):
+    """A forward pass that leaves a NaN in a masked position's hidden state: its row commits
+    nothing, so the loop with the LM head ends after that step with FDLLM_ERR_NONFINITE
+    instead of running to max_steps."""
+    B, gen, Lb, H, V = 2, 32, 16, 256, 3000
+    w = lm_inputs(H, V)
+    hidden = torch.empty((B, Lb, H), dtype=torch.bfloat16, device="cuda")
+    synth = hidden_forward(B, Lb, H, V, w, 5, 20.0)
+
+    def forward(state, mask, out, stream):
+        synth(state, mask, out, stream)
+        with torch.cuda.stream(torch.cuda.ExternalStream(stream)):
+            hidden[0, 3, 11].fill_(float("nan"))
+
+    with pytest.raises(fd.FdllmError) as err:
+        fd.fdllm_decode_loop_lmhead(forward, hidden, w, gen, 1.0, oracle.PROFILE,
+                                    max_steps=10 * gen)
+    assert err.value.status == 3  # FDLLM_ERR_NONFINITE
+    assert fd.fdllm_device_status() == 3
+    assert fd.fdllm_device_status() == 0

@@ -375,3 +375,30 @@ def test_automatic_tiling_small_batch(fd, orc, monkeypatch):
     g_conf, g_tok = conf.cpu().numpy().astype(np.float64), tok.cpu().numpy()
     assert np.array_equal(g_tok[mk], rt[mk])
     assert (np.abs(g_conf[mk] - rc[mk]) / rc[mk]).max() <= CONF_RTOL
+
+
+@pytest.mark.parametrize("variant", ["solo", "pair", "slab"])
+@pytest.mark.parametrize("bad", [float("nan"), float("inf")])
+def test_nonfinite_hidden_state_flags_only_its_row(fd, monkeypatch, variant, bad):
+    """A NaN or an infinity in one masked position's hidden state makes that position's
+    logits unusable: its batch row reports FDLLM_ROW_NONFINITE, commits nothing and keeps its
+    mask, the status word reads FDLLM_ERR_NONFINITE, and every other batch row decides
+    exactly as on the clean input (a row's logits depend on its own hidden state only)."""
+    monkeypatch.setenv("FDLLM_LMHEAD_GEMM", variant)
+    B, L, H, V = 2, 16, 256, 3000
+    h, w, mask_np = inputs(B, L, H, V, seed=41, frac=1.0)
+    bad_h = h.clone()
+    bad_h[1, 5, 17] = bad
+    outs = []
+    for hid, expect in ((h, 0), (bad_h, 3)):
+        mask = torch.from_numpy(mask_np.copy()).cuda()
+        tok, commit, n = fd.fdllm_lmhead_select(hid, w, mask, 0.75)
+        assert fd.fdllm_device_status() == expect
+        outs.append((tok.cpu().numpy(), commit.cpu().numpy(), n.cpu().numpy(),
+                     mask.cpu().numpy()))
+    (t0, c0, n0, m0), (t1, c1, n1, m1) = outs
+    assert n1[1] == fd.ROW_NONFINITE and c1[1].sum() == 0
+    assert np.array_equal(m1[1], mask_np[1])
+    assert n0[1] >= 1 and n1[0] == n0[0] >= 1
+    assert np.array_equal(c1[0], c0[0]) and np.array_equal(m1[0], m0[0])
+    assert np.array_equal(t1[0][c1[0] == 1], t0[0][c0[0] == 1])
