@@ -53,16 +53,20 @@ enum Mode {
                      // (lmhead_slab_kernel)
 };
 
+constexpr int PAIR_KB = 2;  // pair mode: K-blocks per stage
+
 // Vocabulary entries per tile (the MMA's N and the fp32 accumulator's width): 256, or 208,
 // which splits LLaDA's V = 126464 into 608 = 4 x 152 tiles, whole waves over 152 SMs.  The
-// stage count fills the ring budget: solo 4 x 48 KB at 256, 5 x 42 KB at 208; pair 6 x 32 KB
-// at 256 (each CTA holds half the W tile).
+// stage count fills the ring budget: solo 4 x 48 KB at 256, 5 x 42 KB at 208; pair 3 x 64 KB
+// at 256 (each CTA holds half the W tile, and a stage two K-blocks: with the pair's two
+// cross-CTA signals per stage, fewer and larger stages measured faster than 6 x 32 KB).
 template <int BN_, int MODE>
 struct TileCfg {
     static constexpr int BN = BN_;
     static constexpr int kBRows = MODE == kPair ? BN / 2 : BN;  // W rows held per CTA
     static constexpr int kBBytes = kBRows * BK * 2;
-    static constexpr int kStageBytes = kABytes + kBBytes;
+    static constexpr int kKB = MODE == kPair ? PAIR_KB : 1;       // K-blocks of BK per stage
+    static constexpr int kStageBytes = kKB * (kABytes + kBBytes);
     static constexpr int kStages =
         (int)(kRingBudget / kStageBytes) > 8 ? 8 : (int)(kRingBudget / kStageBytes);
     static constexpr size_t kSmemBytes = 1024 + (size_t)kStages * kStageBytes + kBarrierBytes;
@@ -122,14 +126,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     using Cfg = TileCfg<BN_, MODE>;
     constexpr int CL = MODE == kSolo ? 1 : 2;
     constexpr bool PAIR = MODE == kPair;
-    constexpr int BN = Cfg::BN, kStages = Cfg::kStages;
+    constexpr int BN = Cfg::BN, kStages = Cfg::kStages, KB = Cfg::kKB;
     constexpr int kBBytes = Cfg::kBBytes, kStageBytes = Cfg::kStageBytes;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint8_t *sA = smem;                     // kStages x [BM rows][128 B], 128-byte swizzled
-    uint8_t *sB = smem + kStages * kABytes; // kStages x [kBRows rows][128 B]
-    uint64_t *bars = reinterpret_cast<uint64_t *>(sB + kStages * kBBytes);
+    uint8_t *sA = smem;                          // kStages x KB x [BM rows][128 B], swizzled
+    uint8_t *sB = smem + kStages * KB * kABytes; // kStages x KB x [kBRows rows][128 B]
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sB + kStages * KB * kBBytes);
     uint64_t *full = bars;                  // TMA -> MMA, one per stage
     uint64_t *empty = bars + kStages;       // MMA -> TMA, one per stage
     uint64_t *tfull = bars + 2 * kStages;   // MMA -> epilogue, one per accumulator
@@ -206,19 +210,25 @@ __global__ void __launch_bounds__(kThreads, 1)
             bool ok = true;
             for (int64_t t = first; ok && t < total; t += stride) {
                 const int m = (int)(t % num_mc) * CL + rank, n = (int)(t / num_mc);
-                for (int kb = 0; kb < a.k_blocks; ++kb) {
+                for (int kb = 0; kb < a.k_blocks; kb += KB) {
                     if (!wait_or_abort(&empty[s], ph ^ 1u, a.status, abort_flag)) {
                         ok = false;
                         break;
                     }
                     if constexpr (PAIR) {
-                        // Both CTAs' bytes complete on the even CTA's barrier, which it arms.
+                        // Both CTAs' bytes complete on the even CTA's barrier, which it arms
+                        // (K-blocks past H, in the last stage when k_blocks is odd, are
+                        // zero-filled and count in full).
                         if (rank == 0)
                             mbar_arrive_expect_tx(&full[s], 2 * kStageBytes);
                         const uint32_t bar0 = tc::map_to_rank(&full[s], 0);
-                        tc::tma_load_2d_pair(sA + s * kABytes, &map_h, kb * BK, m * BM, bar0);
-                        tc::tma_load_2d_pair(sB + s * kBBytes, &map_w, kb * BK,
-                                             n * BN + rank * (BN / 2), bar0);
+#pragma unroll
+                        for (int q = 0; q < KB; ++q) {
+                            tc::tma_load_2d_pair(sA + (s * KB + q) * kABytes, &map_h,
+                                                 (kb + q) * BK, m * BM, bar0);
+                            tc::tma_load_2d_pair(sB + (s * KB + q) * kBBytes, &map_w,
+                                                 (kb + q) * BK, n * BN + rank * (BN / 2), bar0);
+                        }
                     } else {
                         mbar_arrive_expect_tx(&full[s], kStageBytes);
                         tc::tma_load_2d(sA + s * kABytes, &map_h, kb * BK, m * BM, &full[s]);
@@ -255,20 +265,25 @@ __global__ void __launch_bounds__(kThreads, 1)
                     break;
                 tc::fence_after_sync();
                 const uint32_t d = tmem_base + (uint32_t)acc * kAccStride;
-                for (int kb = 0; kb < a.k_blocks; ++kb) {
+                for (int kb = 0; kb < a.k_blocks; kb += KB) {
                     if (!wait_or_abort(&full[s], ph, a.status, abort_flag)) {
                         ok = false;
                         break;
                     }
                     tc::fence_after_sync();
-                    const uint64_t ad = tc::sw128_kmajor_desc(sA + s * kABytes);
-                    const uint64_t bd = tc::sw128_kmajor_desc(sB + s * kBBytes);
 #pragma unroll
-                    for (int k = 0; k < BK / 16; ++k) {  // K = 16 per MMA: +32 B in the row
-                        if constexpr (PAIR)
-                            tc::mma_bf16_pair(d, ad + 2u * k, bd + 2u * k, idesc, (kb | k) != 0);
-                        else
-                            tc::mma_bf16(d, ad + 2u * k, bd + 2u * k, idesc, (kb | k) != 0);
+                    for (int q = 0; q < KB; ++q) {
+                        const uint64_t ad = tc::sw128_kmajor_desc(sA + (s * KB + q) * kABytes);
+                        const uint64_t bd = tc::sw128_kmajor_desc(sB + (s * KB + q) * kBBytes);
+#pragma unroll
+                        for (int k = 0; k < BK / 16; ++k) {  // K = 16 per MMA: +32 B in the row
+                            if constexpr (PAIR)
+                                tc::mma_bf16_pair(d, ad + 2u * k, bd + 2u * k, idesc,
+                                                  (kb | q | k) != 0);
+                            else
+                                tc::mma_bf16(d, ad + 2u * k, bd + 2u * k, idesc,
+                                             (kb | q | k) != 0);
+                        }
                     }
                     // The stage is free once these MMAs have read it (in a pair, in both
                     // CTAs: each refills its own half of the pair's operands).
