@@ -231,9 +231,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                     } else {
                         mbar_arrive_expect_tx(&full[s], kStageBytes);
-                        tc::tma_load_2d(sA + s * kABytes, &map_h, kb * BK, m * BM, &full[s]);
-                        tc::tma_load_2d_hint(sB + s * kBBytes, &map_w, kb * BK, n * BN,
-                                             &full[s], pol);
+#pragma unroll
+                        for (int q = 0; q < KB; ++q) {
+                            tc::tma_load_2d(sA + (s * KB + q) * kABytes, &map_h, (kb + q) * BK,
+                                            m * BM, &full[s]);
+                            tc::tma_load_2d_hint(sB + (s * KB + q) * kBBytes, &map_w,
+                                                 (kb + q) * BK, n * BN, &full[s], pol);
+                        }
                     }
                     used[s] = true;
                     last_ph[s] = ph;
@@ -431,10 +435,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 // memory that the epilogue skips.  The padded row tile costs 4 KB per K-block instead of
 // 16 KB.  A stage holds two K-blocks (two W boxes and two row boxes), five stages in all
 // (130 KB of W at h = 104 in flight per SM): per-copy overhead, not the bytes in flight,
-// limits how fast W streams here, and two blocks per stage beat one, three or four.  Each epilogue thread keeps, for every row, a running maximum, sum
-// of exp relative to it and first index over its own entry of each tile; after the last
-// tile the 128 threads' states are folded per row (a transposing butterfly in each warp,
-// then the four warps in order) into one partial per (row, CTA).
+// limits how fast W streams here, and two blocks per stage beat one, three or four.  Each
+// epilogue thread keeps, for every row, a running maximum, sum of exp relative to it and
+// first index over its own entry of each tile; after the last tile the 128 threads' states
+// are folded per row (a transposing butterfly in each warp, then the four warps in order)
+// into one partial per (row, CTA).
 constexpr int kSlabRows = 32;
 constexpr int kSlabABytes = BM * BK * 2;                 // 128 lanes; a tile fills h rows
 constexpr int kSlabBBytes = kSlabRows * BK * 2;
