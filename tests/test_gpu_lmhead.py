@@ -63,6 +63,8 @@ SHAPES = [
     (1, 3, 72, 40),
     (3, 100, 256, 2048),
     (4, 100, 128, 1000),   # three row tiles: an odd count for the cluster pairs
+    (2, 40, 192, 3000),    # three K-blocks: the pair's last two-block stage half past H
+    (2, 40, 64, 500),      # one K-block: the pair's only stage half past H
 ]
 
 
