@@ -60,6 +60,8 @@ CASES = [
     (3, 48, 16, 2048, oracle.THRESHOLD, 0.9, 16.0),
     (2, 40, 8, 1000, oracle.PROFILE, 1.0, 12.0),     # V * 2 bytes = 2000, a ragged last unit
     (1, 96, 32, 8192, oracle.PROFILE, 0.95, 18.0),
+    (2, 256, 128, 2048, oracle.PROFILE, 1.0, 16.0),  # blocks beyond 32: the CTA-per-row select
+    (1, 512, 512, 1024, oracle.FACTOR, 1.0, 16.0),   # one 512-position block
 ]
 
 
