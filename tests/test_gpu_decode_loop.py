@@ -168,13 +168,18 @@ def hidden_forward(B, Lb, H, V, w, seed, beta):
     return forward
 
 
-@pytest.mark.parametrize("mode,param", [(oracle.PROFILE, 1.0), (oracle.PROFILE, 0.75),
-                                        (oracle.FACTOR, 1.0)])
-def test_decode_loop_lmhead_against_host_loop_and_oracle(fd, orc, mode, param):
+@pytest.mark.parametrize("mode,param,Lb,gen", [(oracle.PROFILE, 1.0, 16, 32),
+                                                (oracle.PROFILE, 0.75, 16, 32),
+                                                (oracle.FACTOR, 1.0, 16, 32),
+                                                (oracle.PROFILE, 1.0, 64, 128),
+                                                (oracle.FACTOR, 1.0, 96, 192)])
+def test_decode_loop_lmhead_against_host_loop_and_oracle(fd, orc, mode, param, Lb, gen):
     """The device-resident loop with the LM head equals a host-driven loop of
     fdllm_lmhead_select calls (same kernels: bit-exact), and every step of the host loop
-    matches the oracle run on that step's tensor-core accumulators (margin >= 1e-5)."""
-    B, gen, Lb, H, V, seed, beta = 2, 32, 16, 256, 3000, 5, 20.0
+    matches the oracle run on that step's tensor-core accumulators (margin >= 1e-5).  Blocks
+    of 16 positions take the slab GEMM (B * L <= 32), blocks of 64 and 96 the tile GEMM and,
+    past 32 positions, the CTA-per-row selection."""
+    B, H, V, seed, beta = 2, 256, 3000, 5, 20.0
     w = lm_inputs(H, V)
     hidden = torch.empty((B, Lb, H), dtype=torch.bfloat16, device="cuda")
     seq_d, nfe_d, steps_d = fd.fdllm_decode_loop_lmhead(
