@@ -18,7 +18,7 @@ copy bandwidth.  At N = 1 the line also carries, measured after the timed region
 `evolving` (the serving workload with masks evolving from step to step until every row has
 finished), `per_config` (the single-block, mixed-mask, tie-group and full-sequence
 workloads, each beside the oracle on a bounded sample, and the calibration-robust rule on
-the serving workload), `lmhead` (the LM-head-fused step at B = 64 and 16) and `decode_loop`
+the serving workload), `lmhead` (the LM-head-fused step at B = 64, 32, 16 and 1) and `decode_loop`
 (a 256-token generation of 8 sequences in blocks of 32 through the device-resident loop and
 a host-driven one: NFE per block, tokens per step, tokens/s); --skip-evolving,
 --skip-per-config, --skip-lmhead and --skip-decode-loop leave them out.
@@ -677,12 +677,12 @@ def oracle_bounded(name: str, rule: str, param: float, budget_s: float, rows: in
 
 
 def run_lmhead_key(args, torch) -> dict:
-    """The LM-head-fused step at B = 64, 16 and 1 for the default line: fused ms per step,
+    """The LM-head-fused step at B = 64, 32, 16 and 1 for the default line: fused ms per step,
     the a1 path's PFLOP/s (2 R H V over the fdllm_lmhead_confidence time) against the
     measured bf16 burst peak (and the sustained one), and cuBLAS's GEMM on the same masked
     rows alone."""
     out = {}
-    for b in (64, 16, 1):
+    for b in (64, 32, 16, 1):
         a = argparse.Namespace(**vars(args))
         a.lmhead_batch, a.lmhead_vocab = b, 126464
         a.lmhead_variants = "fused,gemm,cublas_masked"

@@ -136,7 +136,7 @@ def test_main_arm_prints_one_contract_line():
     dl = d["decode_loop"]
     assert dl["identical_decisions"] is True and dl["steps"] == sum(dl["nfe_per_block"])
     assert dl["device_loop"]["tokens_per_s"] > 0
-    for b in ("B=64", "B=16"):
+    for b in ("B=64", "B=32", "B=16", "B=1"):
         lm = d["lmhead"][b]
         assert lm["fused_ms"] > 0 and 0 < lm["frac_of_burst_bf16"] < 1.3
     ev = d["evolving"]  # the serving workload with masks evolving until every row finishes
