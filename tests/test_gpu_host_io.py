@@ -94,3 +94,26 @@ def test_select_host_through_c_abi_equals_device_select(fd, orc, where, name, mo
     oref = orc.select(syn.host_bits(x), mask_np, mode, param)
     ok = oref["margin"] >= 1e-5
     assert np.array_equal(h_n.numpy()[ok], oref["n"][ok])
+
+
+def test_host_select_reports_a_nonfinite_row(fd, orc):
+    """Pinned host logits with a NaN in one masked position: through the host-buffer call
+    that batch row reports FDLLM_ROW_NONFINITE and keeps its mask, the other rows match the
+    oracle, and the library workspace's status word reads FDLLM_ERR_NONFINITE once."""
+    w = syn.WORKLOADS["target_b8_l32_bf16"]
+    x = syn.make_logits(w, seed=19, device="cpu", V=4096)
+    mask_np = np.ones((w.B, w.L), np.uint8)
+    x[3, 7, 100] = float("nan")
+    x = x.pin_memory()
+    h_mask = torch.from_numpy(mask_np.copy()).pin_memory()
+    tok, commit, n = fd.fdllm_select(x, h_mask, 0.75, fd.PROFILE)
+    assert fd.fdllm_device_status() == 3  # FDLLM_ERR_NONFINITE
+    assert fd.fdllm_device_status() == 0
+    ref = orc.select(syn.host_bits(x), mask_np, 0, 0.75)
+    assert n[3].item() == fd.ROW_NONFINITE == ref["n"][3]
+    assert commit.numpy()[3].sum() == 0 and (h_mask.numpy()[3] == 1).all()
+    ok = ref["margin"] >= 1e-5
+    ok[3] = False
+    assert ok.sum() >= 4
+    assert np.array_equal(n.numpy()[ok], ref["n"][ok])
+    assert np.array_equal(commit.numpy()[ok], ref["commit"][ok])
