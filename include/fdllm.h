@@ -129,9 +129,11 @@ fdllm_status fdllm_select_ws(const void *logits, int dtype, int B, int L, int V,
  * n* = max accepted, or 1 (the paper defines the robust certificate; this selection rule on
  * it is the library's reading).  With uniform eta and no clipping the score is the plain
  * one minus (n+1) eta (Cor. calibration-penalty).
- *   eta               uniform allowance (finite; the paper takes eta >= 0), used when
- *                     eta_per_position is NULL.
- *   eta_per_position  [B, L] fp32 device array of per-position allowances, or NULL.
+ *   eta               uniform allowance, finite and >= 0 (App. C; otherwise FDLLM_ERR_ARG),
+ *                     used when eta_per_position is NULL.
+ *   eta_per_position  [B, L] fp32 device array of per-position allowances, or NULL; a
+ *                     negative or NaN entry is read as 0 (device data: not checked on the
+ *                     host).
  * Everything else as fdllm_select (the same library workspace).  eta = 0 gives exactly
  * fdllm_select's profile rule. */
 fdllm_status fdllm_select_robust(const void *logits, int dtype, int B, int L, int V,

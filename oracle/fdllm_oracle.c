@@ -301,7 +301,9 @@ int64_t oracle_select_robust_from_conf(const double *conf, const int32_t *tok, i
             const double c_hat = conf[row0 + l];
             if (!(c_hat > 0.0 && c_hat <= 1.0))
                 invalid = 1;
-            const double eta_i = eta_pos ? eta_pos[row0 + l] : eta;
+            /* App. C takes the allowance eta >= 0; a negative or NaN allowance is read as 0 */
+            const double eta_raw = eta_pos ? eta_pos[row0 + l] : eta;
+            const double eta_i = eta_raw > 0.0 ? eta_raw : 0.0;
             /* App. C: the lower confidence max{0, c_hat - eta} */
             const double c_low = c_hat - eta_i > 0.0 ? c_hat - eta_i : 0.0;
             if (fabs(c_hat - eta_i) < clip_gap)

@@ -299,7 +299,7 @@ fdllm_status fdllm_select_robust(const void *logits, int dtype, int B, int L, in
                                         out_tokens, out_commit, out_n);
     if (st != FDLLM_OK)
         return st;
-    if (!std::isfinite(eta))
+    if (!std::isfinite(eta) || eta < 0.0)
         return FDLLM_ERR_ARG;
     const Layout lay = layout_for((int64_t)B * L, (int64_t)V * esize_of(dtype));
     cudaStream_t s = static_cast<cudaStream_t>(stream);

@@ -170,7 +170,7 @@ __global__ void __launch_bounds__(T) profile_select_kernel(const ProfileSelectAr
     auto load_row_inputs = [&]() {
         mask_byte = in_row ? __ldcg(a.mask + base + t) : (uint8_t)0;
         if (a.mode == kModeRobust && a.eta_pos != nullptr && in_row)
-            eta = __ldcg(a.eta_pos + base + t);
+            eta = fmaxf(__ldcg(a.eta_pos + base + t), 0.0f);  // negative or NaN: 0
     };
     if (early)
         load_row_inputs();
@@ -267,7 +267,7 @@ __global__ void __launch_bounds__(32) profile_select_warp_kernel(const ProfileSe
     auto load_row_inputs = [&]() {
         mask_byte = in_row ? __ldcg(a.mask + base + t) : (uint8_t)0;
         if (a.mode == kModeRobust && a.eta_pos != nullptr && in_row)
-            eta = __ldcg(a.eta_pos + base + t);
+            eta = fmaxf(__ldcg(a.eta_pos + base + t), 0.0f);  // negative or NaN: 0
     };
     if (early)
         load_row_inputs();

@@ -458,6 +458,22 @@ def pin_robust_zero_eta_is_profile(o):
         assert np.array_equal(n_r, n_p) and s_r == s_p
 
 
+def pin_robust_negative_allowance_is_zero(o):
+    """App. C takes allowances eta >= 0; the library reads a negative or NaN per-position
+    allowance as 0, so rows whose allowances are all negative or NaN decide as the plain
+    profile rule, and a row mixing such entries with zeros does too."""
+    rng = np.random.default_rng(31)
+    profiles = _random_profiles(rng, 120, 24)
+    L = max(len(p) for p in profiles)
+    eta_pos = -rng.uniform(0.01, 2.0, (len(profiles), L))
+    eta_pos[::3, ::2] = np.nan
+    eta_pos[1::3, 1::2] = 0.0
+    for f in (1.0, 0.75):
+        n_r, s_r, _ = _run_robust(o, profiles, f, 0.0, eta_pos)
+        n_p, s_p, _ = run_profiles(o, profiles, PROFILE, f)
+        assert np.array_equal(n_r, n_p) and s_r == s_p
+
+
 def pin_robust_calibration_penalty(o):
     """Cor. calibration-penalty: with uniform eta and no clipping (every c_hat >= eta),
     G^(eta)_n = G_hat_n - (n+1) eta where the robust lower bound is active, and both sides
@@ -658,6 +674,7 @@ ALL_PINS = [
     pin_matched_dominance, pin_greedy_equivalence, pin_monotone_prefix, pin_special_cases,
     pin_reveal_and_ties, pin_end_to_end, pin_robust_zero_eta_is_profile,
     pin_robust_calibration_penalty, pin_robust_bruteforce, pin_robust_monotone_and_clipped,
+    pin_robust_negative_allowance_is_zero,
     pin_bonus_terms, pin_half_widening, pin_extreme_magnitudes,
     pin_decision_margin_hand_worked, pin_decision_margin_stability,
 ]

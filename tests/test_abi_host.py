@@ -135,6 +135,7 @@ def test_select_robust_rejects(lib):
                                                              eta, None, A16, A16, A16, None)
     assert f(float("nan")) == ERR_ARG
     assert f(float("inf")) == ERR_ARG
+    assert f(-0.05) == ERR_ARG  # App. C's allowance is >= 0
     assert f(0.1, B=0) == ERR_ARG
     assert f(0.1, logits=A2) == ERR_ALIGN
 

@@ -82,3 +82,24 @@ def test_robust_full_size_serving_sample(fd, orc):
             continue
         assert n[b].item() == ref["n"][k]
         assert np.array_equal(commit[b].cpu().numpy(), ref["commit"][k])
+
+
+def test_robust_negative_and_nan_allowances_read_as_zero(fd, orc):
+    """Per-position allowances below 0 or NaN (outside App. C's eta >= 0) are read as 0:
+    against the oracle, and bit for bit the decisions with those entries set to 0."""
+    w = syn.WORKLOADS["target_b8_l32_bf16"]
+    logits = syn.make_logits(w, seed=909, device="cuda")
+    mask_np = syn.make_mask(w, seed=909)
+    rng = np.random.default_rng(9)
+    eta_pos = rng.uniform(-0.2, 0.1, (w.B, w.L))
+    eta_pos[::2, ::5] = np.nan
+    _check(fd, orc, logits, mask_np, 0.75, 0.0, eta_pos)
+    clean = np.where(np.isnan(eta_pos) | (eta_pos < 0.0), 0.0, eta_pos)
+    outs = []
+    for e in (eta_pos, clean):
+        mask = torch.from_numpy(mask_np.copy()).cuda()
+        ep = torch.from_numpy(e.astype(np.float32)).cuda()
+        outs.append([x.cpu() for x in fd.fdllm_select_robust(logits, mask, 0.75, 0.0, ep)]
+                    + [mask.cpu()])
+    for x, y in zip(*outs):
+        assert torch.equal(x, y)

@@ -51,8 +51,10 @@ MUTANTS = {
     "robust_eta_added": ("const double c_low = c_hat - eta_i > 0.0 ? c_hat - eta_i : 0.0;",
                          "const double c_low = c_hat + eta_i;"),
     "robust_ranks_by_c_hat": ("cand[m].c = c_low;", "cand[m].c = c_hat;"),
-    "robust_eta_ignored": ("const double eta_i = eta_pos ? eta_pos[row0 + l] : eta;",
+    "robust_eta_ignored": ("const double eta_i = eta_raw > 0.0 ? eta_raw : 0.0;",
                            "const double eta_i = 0.0;"),
+    "robust_negative_eta_kept": ("const double eta_i = eta_raw > 0.0 ? eta_raw : 0.0;",
+                                 "const double eta_i = eta_raw;"),
     "factor_core_drops_plus_one": ("Fn[n - 1] = (double)(n + 1) * cn - (double)n;",
                                    "Fn[n - 1] = (double)n * cn - (double)n;"),
     "bonus_index_shifted": ("bonus += c_sorted[j - 1] - cn;", "bonus += c_sorted[j] - cn;"),
