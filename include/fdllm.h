@@ -340,7 +340,9 @@ fdllm_status fdllm_decode_loop_lmhead(int B, int gen_len, int block_len, int H, 
  * Ranks n > m_b get NaN (order -1).  G_n = F_n + B_n wherever the lower bound is positive,
  * so the profile rule with margin delta behaves as the factor rule with the effective
  * factor f_eff(n).
- *   conf   [B, L] fp32 device (e.g. from fdllm_confidence), read at masked positions.
+ *   conf   [B, L] fp32 device (e.g. from fdllm_confidence), read at masked positions:
+ *          values in [0, 1], or NaN (a NaN ranks after every number, so the terms of its
+ *          rank and of every later rank are NaN); other values give unspecified terms.
  *   mask   [B, L] uint8 device, nonzero = masked (not modified).
  *   delta  the profile rule's margin (delta = 1 - param of fdllm_select), finite.
  *   out_G, out_F, out_B, out_feff  [B, L] fp64 device, each nullable; out_order [B, L]
