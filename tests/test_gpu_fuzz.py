@@ -45,7 +45,7 @@ def draw_case(seed):
 
 
 @pytest.mark.gpu
-@pytest.mark.parametrize("seed", range(32))
+@pytest.mark.parametrize("seed", range(128))
 def test_random_case_matches_oracle(fd, orc, seed):
     w, mask, mode, param = draw_case(seed)
     logits = syn.make_logits(w, seed=seed, device="cuda")
@@ -75,7 +75,7 @@ def draw_lmhead_case(seed):
 
 
 @pytest.mark.gpu
-@pytest.mark.parametrize("seed", range(16))
+@pytest.mark.parametrize("seed", range(48))
 def test_random_lmhead_case_matches_oracle(fd, orc, monkeypatch, seed):
     """The LM-head path on drawn shapes (H not a multiple of the K stage, V ragged against
     every tile), GEMM variants and tile widths: the stored logits within the fp32
@@ -108,7 +108,7 @@ def test_random_lmhead_case_matches_oracle(fd, orc, monkeypatch, seed):
 
 
 @pytest.mark.gpu
-@pytest.mark.parametrize("seed", range(12))
+@pytest.mark.parametrize("seed", range(48))
 def test_random_robust_case_matches_oracle(fd, orc, seed):
     """The calibration-robust rule on the drawn cases, with a drawn uniform allowance or a
     drawn per-position one (App. C), against the oracle's robust selector."""
