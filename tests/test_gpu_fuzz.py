@@ -122,3 +122,46 @@ def test_random_robust_case_matches_oracle(fd, orc, seed):
         _check(fd, orc, logits, mask, param, float(rng.uniform(0.0, 0.3)))
     else:
         _check(fd, orc, logits, mask, param, 0.0, rng.uniform(0.0, 0.3, (w.B, w.L)))
+
+
+def draw_large_shape_case(seed):
+    """Many rows and long blocks on small vocabularies: B * L up to 65536 and L from 1 to
+    1024 (both selection kernels, the reduction's mask compaction and work queue over many
+    rows), at sizes the oracle finishes quickly."""
+    rng = np.random.default_rng(90_000 + seed)
+    dtype = ("bf16", "fp16", "fp32")[rng.integers(3)]
+    q = 4 if dtype == "fp32" else 8
+    V = int(rng.choice([8, 16, 24, 120, 1000]))
+    V = (V + q - 1) // q * q
+    L = int(rng.choice([1, 2, 31, 32, 33, 64, 100, 257, 512, 1024]))
+    B = int(rng.integers(1, max(1, min(64, 65536 // L)) + 1))
+    peak = ("none", "uniform", "target")[rng.integers(3)]
+    lo, hi = (0.3, 4.0) if peak == "target" else (0.0, float(rng.uniform(2.0, 20.0)))
+    w = syn.Workload("fuzz_large_%d" % seed, B, L, V, dtype, 1.0, peak, lo, hi)
+    mrng = np.random.default_rng(seed)
+    frac = mrng.uniform(0.0, 1.0, size=(B, 1))
+    frac[mrng.random((B, 1)) < 0.2] = 0.0
+    mask = (mrng.random((B, L)) < frac).astype(np.uint8)
+    mode = int(rng.integers(3))
+    if mode == THRESHOLD:
+        param = float(rng.choice([0.3, 0.5, 0.9]))
+    else:
+        param = float(rng.choice([0.5, 0.75, 1.0, 2.0]))
+    return w, mask, mode, param
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("seed", range(64))
+def test_random_large_shape_case_matches_oracle(fd, orc, seed):
+    w, mask, mode, param = draw_large_shape_case(seed)
+    logits = syn.make_logits(w, seed=seed, device="cuda")
+    check_confidence(fd, orc, logits, mask)
+    check_select(fd, orc, logits, mask, mode, param)
+
+
+def test_large_shape_draws_cover_the_space():
+    """The 64 large-shape draws reach both selection kernels and thousands of rows."""
+    cases = [draw_large_shape_case(s) for s in range(64)]
+    assert min(c[0].L for c in cases) <= 32 < max(c[0].L for c in cases)
+    assert max(c[0].B * c[0].L for c in cases) >= 8192
+    assert {c[0].dtype for c in cases} == {"bf16", "fp16", "fp32"}
