@@ -223,3 +223,41 @@ def test_profile_terms_rejects_before_any_device_call(lib):
     assert call(2, 32, 0.0, mask=None) == ERR_ARG
     assert call(2, 32, float("nan")) == ERR_ARG
     assert call(2, 32, float("inf")) == ERR_ARG
+
+
+def test_c_program_builds_against_the_header_and_links(cuda_lib_path, tmp_path):
+    """A plain C99 program includes include/fdllm.h with -pedantic -Werror, takes the address
+    of every declared function (so each must be exported with C linkage), links against the
+    library and calls its host-only entry points."""
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    names = declared_functions()
+    src = tmp_path / "abi.c"
+    src.write_text(
+        "#include <stdio.h>\n#include \"fdllm.h\"\n"
+        "typedef void (*any_fn)(void);\n"
+        "static any_fn table[] = {\n"
+        + "".join("    (any_fn)%s,\n" % n for n in names)
+        + "};\n"
+        "int main(void)\n{\n"
+        "    size_t ws = fdllm_workspace_bytes(64, 32, 126464, FDLLM_BF16);\n"
+        "    printf(\"%d %zu %d %s\\n\", fdllm_version(), ws, (int)(sizeof table / sizeof *table),\n"
+        "           fdllm_status_string(FDLLM_ERR_NONFINITE));\n"
+        "    return fdllm_select(0, FDLLM_BF16, 1, 1, 8, 0, 0.75, FDLLM_PROFILE, 0, 0, 0, 0) ==\n"
+        "               FDLLM_ERR_ARG ? 0 : 1;\n"
+        "}\n")
+    exe = tmp_path / "abi"
+    libdir = os.path.dirname(cuda_lib_path)
+    r = subprocess.run([cc, "-std=c99", "-Wall", "-Wextra", "-pedantic", "-Werror",
+                        "-Wno-cast-function-type", "-I", os.path.join(ROOT, "include"),
+                        str(src), "-o", str(exe), "-L", libdir, "-lfdllm",
+                        "-Wl,-rpath," + libdir], capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    out = subprocess.run([str(exe)], capture_output=True, text=True)
+    assert out.returncode == 0, out.stderr
+    version, ws, count, text = out.stdout.split(" ", 3)
+    assert int(version) >= 100 and int(ws) > 0 and int(count) == len(names)
+    assert "non-finite" in text
