@@ -117,3 +117,94 @@ def test_host_select_reports_a_nonfinite_row(fd, orc):
     assert ok.sum() >= 4
     assert np.array_equal(n.numpy()[ok], ref["n"][ok])
     assert np.array_equal(commit.numpy()[ok], ref["commit"][ok])
+
+
+def test_c_program_selects_from_pinned_host_logits(fd, orc, cuda_lib_path, tmp_path):
+    """The host-buffer step from a plain C program, as the README shows it: page-locked
+    logits from cudaHostAlloc, one fdllm_select_host call, the results against the oracle."""
+    import os
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    cuda = os.environ.get("CUDA_HOME", "/usr/local/cuda")
+    if cc is None or not os.path.isdir(os.path.join(cuda, "include")):
+        pytest.skip("no C compiler or CUDA headers")
+    w = syn.WORKLOADS["target_b8_l32_bf16"]
+    V = 4096
+    x = syn.make_logits(w, seed=23, device="cpu", V=V)
+    bits = syn.host_bits(x)  # uint16 bf16 patterns, [B, L, V]
+    mask_np = syn.make_mask(w, seed=23)
+    (tmp_path / "logits.bin").write_bytes(np.ascontiguousarray(bits).tobytes())
+    (tmp_path / "mask.bin").write_bytes(mask_np.tobytes())
+    src = tmp_path / "step.c"
+    src.write_text(r'''
+#include <stdio.h>
+#include <stdlib.h>
+#include <string.h>
+#include <cuda_runtime.h>
+#include "fdllm.h"
+int main(int argc, char **argv)
+{
+    const int B = atoi(argv[1]), L = atoi(argv[2]), V = atoi(argv[3]);
+    const size_t n = (size_t)B * L * V;
+    uint16_t *logits = NULL;
+    if (cudaHostAlloc((void **)&logits, n * 2, cudaHostAllocDefault) != cudaSuccess)
+        return 2;
+    FILE *f = fopen(argv[4], "rb");
+    if (!f || fread(logits, 2, n, f) != n)
+        return 3;
+    fclose(f);
+    uint8_t *mask = malloc((size_t)B * L), *commit = malloc((size_t)B * L);
+    int32_t *tokens = malloc((size_t)B * L * 4), *nstar = malloc((size_t)B * 4);
+    f = fopen(argv[5], "rb");
+    if (!f || fread(mask, 1, (size_t)B * L, f) != (size_t)B * L)
+        return 4;
+    fclose(f);
+    for (int i = 0; i < B * L; ++i)
+        tokens[i] = -1;
+    fdllm_status st = fdllm_select_host(logits, FDLLM_BF16, B, L, V, mask, 0.75, FDLLM_PROFILE,
+                                        tokens, commit, nstar, 0);
+    if (st != FDLLM_OK) {
+        fprintf(stderr, "%s\n", fdllm_status_string(st));
+        return 5;
+    }
+    if (fdllm_device_status(0) != FDLLM_OK)
+        return 6;
+    f = fopen(argv[6], "wb");
+    fwrite(tokens, 4, (size_t)B * L, f);
+    fwrite(commit, 1, (size_t)B * L, f);
+    fwrite(nstar, 4, (size_t)B, f);
+    fwrite(mask, 1, (size_t)B * L, f);
+    fclose(f);
+    cudaFreeHost(logits);
+    return 0;
+}
+''')
+    exe = tmp_path / "step"
+    libdir = os.path.dirname(cuda_lib_path)
+    cudalib = os.path.join(cuda, "lib64")
+    include = os.path.join(os.path.dirname(libdir), "include")
+    r = subprocess.run([cc, "-std=c99", "-O2", "-I", include,
+                        "-I", os.path.join(cuda, "include"), str(src), "-o", str(exe),
+                        "-L", libdir, "-lfdllm", "-L", cudalib, "-lcudart",
+                        "-Wl,-rpath," + libdir, "-Wl,-rpath," + cudalib],
+                       capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    out = tmp_path / "out.bin"
+    p = subprocess.run([str(exe), str(w.B), str(w.L), str(V), str(tmp_path / "logits.bin"),
+                        str(tmp_path / "mask.bin"), str(out)], capture_output=True, text=True)
+    assert p.returncode == 0, (p.returncode, p.stderr)
+    raw = out.read_bytes()
+    BL = w.B * w.L
+    tok = np.frombuffer(raw[:4 * BL], np.int32).reshape(w.B, w.L)
+    commit = np.frombuffer(raw[4 * BL:5 * BL], np.uint8).reshape(w.B, w.L)
+    nst = np.frombuffer(raw[5 * BL:5 * BL + 4 * w.B], np.int32)
+    mask_out = np.frombuffer(raw[5 * BL + 4 * w.B:], np.uint8).reshape(w.B, w.L)
+    ref = orc.select(bits, mask_np, 0, 0.75)
+    ok = ref["margin"] >= 1e-5
+    assert ok.sum() >= w.B // 2
+    assert np.array_equal(nst[ok], ref["n"][ok])
+    assert np.array_equal(commit[ok], ref["commit"][ok])
+    assert np.array_equal(mask_out[ok], ref["mask"][ok])
+    c = ref["commit"].astype(bool) & ok[:, None]
+    assert np.array_equal(tok[c], ref["tokens"][c])
