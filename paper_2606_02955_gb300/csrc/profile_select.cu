@@ -172,11 +172,11 @@ __global__ void __launch_bounds__(T) profile_select_kernel(const ProfileSelectAr
         if (a.mode == kModeRobust && a.eta_pos != nullptr && in_row)
             eta = fmaxf(__ldcg(a.eta_pos + base + t), 0.0f);  // negative or NaN: 0
     };
+    if (threadIdx.x == 0)
+        pdl_launch_dependents();  // a following vocab reduction may start its prologue
     if (early)
         load_row_inputs();
     pdl_wait();
-    if (threadIdx.x == 0)
-        pdl_launch_dependents();  // a following vocab reduction may start its prologue
     if (!early)
         load_row_inputs();
     const bool dev_err = a.status != nullptr && (__ldcg(a.status) & kDevStatTimeout) != 0;
@@ -269,11 +269,11 @@ __global__ void __launch_bounds__(32) profile_select_warp_kernel(const ProfileSe
         if (a.mode == kModeRobust && a.eta_pos != nullptr && in_row)
             eta = fmaxf(__ldcg(a.eta_pos + base + t), 0.0f);  // negative or NaN: 0
     };
+    if (t == 0)
+        pdl_launch_dependents();  // a following vocab reduction may start its prologue
     if (early)
         load_row_inputs();
     pdl_wait();  // the producer of the partials or confidences has completed
-    if (t == 0)
-        pdl_launch_dependents();  // a following vocab reduction may start its prologue
     if (!early)
         load_row_inputs();
     // The rest of the row's loads are issued here, before any of them is used (one memory
